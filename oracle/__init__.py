@@ -1,0 +1,19 @@
+"""CPU oracle of the PTD tree-verify step.
+
+Test infrastructure: only the tests, `__graft_entry__.smoke()` and `bench.py`'s
+CPU-baseline / reference arm may import it.  The product path never does.
+"""
+from .ptd_oracle import (  # noqa: F401
+    InvalidTree,
+    ancestor_sets,
+    check_tree,
+    children_sets,
+    depths,
+    eligible_edges,
+    kv_compact,
+    topk,
+    topk_rows,
+    tree_attention,
+    verify_greedy,
+    visibility,
+)

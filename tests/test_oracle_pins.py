@@ -1,0 +1,335 @@
+"""Pins of the CPU oracle against things other than itself (no GPU needed).
+
+Each check is chosen so that a plausible slip in the oracle (a dropped ancestor, a
+wrong GQA head map, a missing context slot, a reversed tie-break, a transposed
+operand, an unsafe overlapping copy) fails at least one of them:
+  * hand-derived worked examples (tests/golden/*.json, each citing its passage);
+  * reductions to library routines: float64 torch SDPA with masks built without
+    the ancestor sets (chain = causal chunk, single node = plain decode, star),
+    np.lexsort for top-k;
+  * closed forms (identical keys -> mean of the visible values);
+  * brute force: every root path of every recursive tree with <= 6 nodes (and a
+    sample at 7 nodes) under every binary token/target assignment;
+  * invariants and metamorphic relabelling.
+"""
+import itertools
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_10661_gb300 import synthetic as syn
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _load(name):
+    with open(os.path.join(GOLD, name)) as f:
+        return json.load(f)
+
+
+def _num(x):
+    if isinstance(x, (int, float)):
+        return float(x)
+    if x.startswith("ln"):
+        return math.log(float(x[2:]))
+    return float(Fraction(x))
+
+
+# ----------------------------------------------------------------------------- tree
+
+def test_check_tree_rejects_bad_parents():
+    for bad in ([], [0], [-1, 1], [-1, 0, 2], [-1, -1], [-1, 0, 5], [1, -1]):
+        with pytest.raises(oracle.InvalidTree):
+            oracle.check_tree(bad)
+    oracle.check_tree([-1])
+    oracle.check_tree([-1, 0, 0, 1, 3])
+
+
+def test_ancestor_sets_closed_forms():
+    # chain: pi(i) = {0..i};  complete binary: |pi(i)| = floor(log2(i+1)) + 1
+    chain = [-1] + list(range(0, 9))
+    for i, s in enumerate(oracle.ancestor_sets(chain)):
+        assert s == set(range(i + 1))
+    b = syn.binary_tree(31)
+    for i, s in enumerate(oracle.ancestor_sets(b)):
+        assert len(s) == int(math.floor(math.log2(i + 1))) + 1
+        # every member's own ancestors are a subset (closure)
+        assert all(((j - 1) // 2 in s) for j in s if j > 0)
+
+
+# ------------------------------------------------------------------------ attention
+
+def test_attention_worked_example():
+    g = _load("attention_worked.json")
+    C, scale, parents = g["ctx_len"], g["scale"], g["parents"]
+    q = np.stack([np.array(g["q_head0"], float), np.array(g["q_head1"], float)], axis=1)  # [T,2,D]
+    k = np.array([[_num(x) for x in r] for r in g["k"]])[:, None, :]
+    v = np.array([[_num(x) for x in r] for r in g["v"]])[:, None, :]
+    o = oracle.tree_attention(q, k, v, parents, C, scale)
+    exp0 = np.array([[_num(x) for x in r] for r in g["o_head0"]])
+    exp1 = np.array([[_num(x) for x in r] for r in g["o_head1"]])
+    np.testing.assert_allclose(o[:, 0, :], exp0, rtol=0, atol=1e-13)
+    np.testing.assert_allclose(o[:, 1, :], exp1, rtol=0, atol=1e-13)
+
+
+def _sdpa(q, k, v, mask, scale):
+    """float64 torch SDPA: q [T,H,D], k/v [N,H,D], mask [T,N] bool (True = attend)."""
+    qt = torch.from_numpy(q).permute(1, 0, 2)[None]
+    kt = torch.from_numpy(k).permute(1, 0, 2)[None]
+    vt = torch.from_numpy(v).permute(1, 0, 2)[None]
+    o = torch.nn.functional.scaled_dot_product_attention(
+        qt, kt, vt, attn_mask=torch.from_numpy(mask), scale=scale)
+    return o[0].permute(1, 0, 2).numpy()
+
+
+def _rand_qkv(seed, T, C, Hq, Hkv, D):
+    g = np.random.default_rng(seed)
+    return (g.standard_normal((T, Hq, D)), g.standard_normal((C + T, Hkv, D)),
+            g.standard_normal((C + T, Hkv, D)))
+
+
+@pytest.mark.parametrize("C", [0, 1, 7, 40])
+def test_chain_tree_is_causal_chunk(C):
+    T, H, D = 9, 3, 16
+    q, k, v = _rand_qkv(1 + C, T, C, H, H, D)
+    parents = [-1] + list(range(T - 1))
+    mask = np.tril(np.ones((T, C + T), bool), k=C)       # causal over an appended chunk
+    o = oracle.tree_attention(q, k, v, parents, C)
+    np.testing.assert_allclose(o, _sdpa(q, k, v, mask, 1 / math.sqrt(D)), rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("C", [0, 5, 300])
+def test_single_node_is_plain_decode(C):
+    H, D = 4, 32
+    q, k, v = _rand_qkv(7 + C, 1, C, H, H, D)
+    o = oracle.tree_attention(q, k, v, [-1], C)
+    mask = np.ones((1, C + 1), bool)
+    np.testing.assert_allclose(o, _sdpa(q, k, v, mask, 1 / math.sqrt(D)), rtol=1e-12, atol=1e-12)
+
+
+def test_star_tree_sees_context_root_self():
+    T, C, H, D = 6, 11, 2, 8
+    q, k, v = _rand_qkv(3, T, C, H, H, D)
+    parents = [-1] + [0] * (T - 1)
+    mask = np.zeros((T, C + T), bool)
+    mask[:, :C + 1] = True                               # context and the root
+    mask[np.arange(T), C + np.arange(T)] = True          # itself
+    o = oracle.tree_attention(q, k, v, parents, C)
+    np.testing.assert_allclose(o, _sdpa(q, k, v, mask, 1 / math.sqrt(D)), rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("G", [1, 4, 8])
+def test_gqa_matches_repeated_kv_heads(G):
+    """Query head h uses KV head h // G: equals MHA with each KV head repeated G times.
+    The mask is the complete binary tree's, built from (i-1)//2 without ancestor sets."""
+    T, C, Hkv, D = 15, 20, 2, 16
+    q, k, v = _rand_qkv(11 * G, T, C, Hkv * G, Hkv, D)
+    parents = syn.binary_tree(T)
+    mask = np.zeros((T, C + T), bool)
+    mask[:, :C] = True
+    for i in range(T):
+        a = i
+        while True:
+            mask[i, C + a] = True
+            if a == 0:
+                break
+            a = (a - 1) // 2
+    o = oracle.tree_attention(q, k, v, parents, C)
+    kr, vr = np.repeat(k, G, axis=1), np.repeat(v, G, axis=1)
+    np.testing.assert_allclose(o, _sdpa(q, kr, vr, mask, 1 / math.sqrt(D)), rtol=1e-12, atol=1e-12)
+
+
+def test_identical_keys_give_mean_of_visible_values():
+    """All scores equal -> uniform weights over the C + depth(i) + 1 visible slots."""
+    T, C, D = 15, 5, 4
+    g = np.random.default_rng(5)
+    q = g.standard_normal((T, 1, D))
+    k = np.tile(g.standard_normal((1, 1, D)), (C + T, 1, 1))
+    v = g.standard_normal((C + T, 1, D))
+    parents = syn.binary_tree(T)
+    o = oracle.tree_attention(q, k, v, parents, C)
+    for i in range(T):
+        anc, a = [], i
+        while True:
+            anc.append(a)
+            if a == 0:
+                break
+            a = (a - 1) // 2
+        rows = list(range(C)) + [C + a for a in anc]
+        np.testing.assert_allclose(o[i, 0], v[rows, 0].mean(axis=0), rtol=1e-12, atol=1e-12)
+
+
+def test_relabelling_permutes_outputs():
+    """Another topological order of the same tree permutes the outputs accordingly."""
+    cfg = syn.shrink(syn.CONFIGS["llama2-7b-layer"], hq=2, hkv=2, d=16, ctx=(13, 13), vocab=50)
+    w = syn.Workload(cfg, 3)
+    par = w.trees[0]
+    T = len(par)
+    C = int(w.ctx_lens[0])
+    g = np.random.default_rng(0)
+    q, k, v = _rand_qkv(9, T, C, 2, 2, 16)
+    o = oracle.tree_attention(q, k, v, par, C)
+    # DFS preorder (children in reverse) is another topological order
+    kids = oracle.children_sets(par)
+    order, stack = [], [0]
+    while stack:
+        n = stack.pop()
+        order.append(n)
+        stack.extend(kids[n])
+    new_of = {old: new for new, old in enumerate(order)}
+    par2 = [-1 if par[old] < 0 else new_of[int(par[old])] for old in order]
+    q2 = q[order]
+    k2 = np.concatenate([k[:C], k[C + np.array(order)]])
+    v2 = np.concatenate([v[:C], v[C + np.array(order)]])
+    o2 = oracle.tree_attention(q2, k2, v2, par2, C)
+    np.testing.assert_allclose(o2, o[order], rtol=1e-12, atol=1e-12)
+    del g
+
+
+# ----------------------------------------------------------------------------- top-k
+
+def test_topk_worked_example():
+    g = _load("topk_worked.json")
+    row = np.array(g["row"])
+    for c in g["cases"]:
+        idx, val = oracle.topk(row, c["k"])
+        assert idx.tolist() == c["idx"]
+        assert val.tolist() == c["val"]
+
+
+def test_topk_matches_lexsort_with_ties():
+    g = np.random.default_rng(17)
+    for trial in range(40):
+        V = int(g.integers(1, 3000))
+        row = np.round(g.standard_normal(V) * 3, 1)        # many exact ties
+        row[g.integers(0, V, size=min(V, 5))] = 0.0
+        row[g.integers(0, V, size=min(V, 5))] = -0.0
+        k = int(g.integers(1, min(V, 16) + 1))
+        order = np.lexsort((np.arange(V), -row))[:k]       # primary -value, secondary index
+        idx, val = oracle.topk(row, k)
+        assert idx.tolist() == order.tolist()
+        assert np.array_equal(val, row[order])
+
+
+def test_topk_brute_force_rank():
+    """rank(j) = #{i : x_i > x_j or (x_i == x_j and i < j)}; top-k = ranks 0..k-1 in rank order."""
+    g = np.random.default_rng(23)
+    for _ in range(30):
+        V = int(g.integers(1, 60))
+        row = g.integers(-3, 4, size=V).astype(float)
+        k = int(g.integers(1, V + 1))
+        rank = [sum(1 for i in range(V) if row[i] > row[j] or (row[i] == row[j] and i < j)) for j in range(V)]
+        expect = sorted(range(V), key=lambda j: rank[j])[:k]
+        assert oracle.topk(row, k)[0].tolist() == expect
+
+
+def test_topk_bf16_rows_widen_exactly():
+    bits = syn.bf16_bits(np.random.default_rng(2).standard_normal((3, 500)).astype(np.float32))
+    x = syn.widen(bits, "bf16")
+    idx, val = oracle.topk_rows(x, 4)
+    for r in range(3):
+        order = np.lexsort((np.arange(500), -x[r]))[:4]
+        assert idx[r].tolist() == order.tolist()
+
+
+# ---------------------------------------------------------------------------- verify
+
+def test_verify_worked_examples():
+    for c in _load("verify_worked.json")["cases"]:
+        I = oracle.eligible_edges(c["parents"], c["tokens"], c["target"])
+        assert sorted(map(list, I)) == c["eligible_edges"]
+        path, n, bonus = oracle.verify_greedy(c["parents"], c["tokens"], c["target"])
+        assert path == c["path"] and n == c["accept_len"] and bonus == c["bonus"]
+
+
+def _brute_force(parents, tokens, target):
+    """Enumerate every root path (one per end node); keep eligible ones; longest, then lex-min."""
+    best = None
+    for end in range(len(parents)):
+        path = [end]
+        while parents[path[-1]] >= 0:
+            path.append(parents[path[-1]])
+        path.reverse()
+        if all(tokens[c] == target[p] for p, c in zip(path, path[1:])):
+            if best is None or len(path) > len(best) or (len(path) == len(best) and path < best):
+                best = path
+    return best, len(best), target[best[-1]]
+
+
+def _recursive_trees(n):
+    for tail in itertools.product(*[range(i) for i in range(1, n)]):
+        yield [-1, *tail]
+
+
+@pytest.mark.parametrize("n", [1, 2, 3, 4, 5, 6])
+def test_verify_brute_force_exhaustive(n):
+    for parents in _recursive_trees(n):
+        for toks in itertools.product((0, 1), repeat=n - 1):
+            tokens = [0, *toks]
+            for target in itertools.product((0, 1), repeat=n):
+                assert oracle.verify_greedy(parents, tokens, target) == _brute_force(parents, tokens, list(target))
+
+
+def test_verify_brute_force_seven_nodes_sampled():
+    g = np.random.default_rng(7)
+    trees = list(_recursive_trees(7))
+    for parents in trees:
+        for _ in range(24):
+            tokens = [0] + g.integers(0, 2, size=6).tolist()
+            target = g.integers(0, 2, size=7).tolist()
+            assert oracle.verify_greedy(parents, tokens, target) == _brute_force(parents, tokens, target)
+
+
+@pytest.mark.parametrize("name", syn.CONFIG_ORDER)
+def test_verify_invariants_on_workloads(name):
+    cfg = syn.CONFIGS[name]
+    if cfg.vocab > 40000:
+        cfg = syn.shrink(cfg, vocab=4000)
+    w = syn.Workload(cfg, 1)
+    logits = syn.widen(w.logits, cfg.dtype)
+    idx, _ = oracle.topk_rows(logits, 1)
+    for b in range(cfg.batch):
+        sl = w.nodes_of(b)
+        par, tok, tgt = w.trees[b], w.tokens[sl], idx[sl, 0]
+        path, n, bonus = oracle.verify_greedy(par, tok, tgt)
+        d = oracle.depths(par)
+        assert 1 <= n <= d.max() + 1                       # accepted edges <= tree depth
+        assert path[0] == 0
+        for p, c in zip(path, path[1:]):
+            assert par[c] == p and tok[c] == tgt[p]        # a root path of eligible edges
+        assert not any(tok[c] == tgt[path[-1]] for c in oracle.children_sets(par)[path[-1]])
+        assert bonus == tgt[path[-1]]
+
+
+# --------------------------------------------------------------------------- compact
+
+def test_compact_worked_example():
+    g = _load("compact_worked.json")
+    slots = np.array(g["slots_before"])[:, None]
+    new, new_ctx = oracle.kv_compact(slots, g["path"], g["ctx_len"])
+    assert new_ctx == g["new_ctx"]
+    assert new[:new_ctx, 0].tolist() == g["slots_after_prefix"]
+
+
+def test_compact_matches_gather_and_keeps_prefix():
+    g = np.random.default_rng(4)
+    for _ in range(50):
+        C, T = int(g.integers(0, 20)), int(g.integers(1, 30))
+        parents = [-1] + [int(g.integers(0, i)) for i in range(1, T)]
+        # a random root path
+        end = int(g.integers(0, T))
+        path = [end]
+        while parents[path[-1]] >= 0:
+            path.append(parents[path[-1]])
+        path.reverse()
+        cache = g.standard_normal((C + T + 3, 2, 4))
+        new, nc = oracle.kv_compact(cache, path, C)
+        assert nc == C + len(path)
+        assert np.array_equal(new[:C], cache[:C])
+        assert np.array_equal(new[C:nc], cache[C + np.array(path)])
