@@ -1,0 +1,227 @@
+/*
+ * ptd.h -- C ABI of the Progressive Tree Drafting (PTD) tree-verify step on one GPU.
+ *
+ * One step of PTD (Alg. 1, steps 2 and 5-6) runs the target model once over the
+ * committed prefix X followed by a rooted token tree (the draft tree T and the
+ * retrieved candidate tree C_X hang below the current token, Sec. 3.2), reads the
+ * greedy token of every tree node, accepts the longest root path whose edges are
+ * eligible, and appends it to X.  This library exposes the data-parallel part of
+ * that step as four calls:
+ *
+ *   ptd_tree_attention   tree-masked attention, ancestor-only visibility (Sec. 3.1)
+ *   ptd_topk_draft       per-node top-k of the logits: draft tokens d_v, width
+ *                        control, greedy verification tokens V_n (Sec. 3.1, 3.2)
+ *   ptd_verify_greedy    eligible edges I and accepted sequence X' (Sec. 3.2)
+ *   ptd_kv_compact       move the accepted nodes' K/V behind the prefix (Alg. 1 step 6)
+ *
+ * Conventions shared by every call
+ *   - Pointers are DEVICE pointers unless a comment says "host".  The caller owns
+ *     all memory; the library never allocates, frees or synchronises.  Scratch
+ *     space, where a call needs any, is passed in by the caller.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Every call only enqueues work on that stream and returns.
+ *   - Errors the host can see (null pointer, bad size, unsupported shape) return
+ *     synchronously and enqueue nothing.  Errors only the device can see (an
+ *     invalid parent array) are reported through `dev_status` (one int32 in device
+ *     memory, written with atomicMax of the status code, so the caller zeroes it
+ *     before the step and reads it after); the affected sequence's outputs are then
+ *     defined (zeros, accept_len 0) instead of garbage.
+ *   - A failed kernel launch returns PTD_ERR_CUDA.  No C++ exception crosses the ABI.
+ *
+ * Tree layout (ptd_tree): B trees stored back to back; tree b owns nodes
+ * [node_offsets[b], node_offsets[b+1]); parents are tree-local indices with
+ * parents[first] = -1 and 0 <= parents[i] < i (topological order, e.g. BFS).
+ * Node 0 of a tree is the current input token; node i of tree b has its K/V at
+ * cache slot ctx_lens[b] + i, right after the b-th committed prefix.
+ */
+#ifndef PTD_H_
+#define PTD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  PTD_OK = 0,
+  PTD_ERR_INVALID_ARG = 1,   /* null pointer, size out of range, inconsistent shapes      */
+  PTD_ERR_INVALID_TREE = 2,  /* (device) a parent array is not a topological rooted tree  */
+  PTD_ERR_UNSUPPORTED = 3,   /* valid but not implemented (dtype / head_dim combination)  */
+  PTD_ERR_CUDA = 4,          /* a CUDA runtime call or kernel launch failed              */
+  PTD_ERR_TIMEOUT = 5,       /* (device) a bounded on-chip wait gave up; outputs invalid  */
+  PTD_ERR_WORKSPACE = 6      /* workspace pointer null or smaller than required          */
+} ptd_status;
+
+typedef enum { PTD_F32 = 0, PTD_BF16 = 1 } ptd_dtype;
+
+/* Maximum nodes of one tree (the ancestor bitmask of a node is 4 x 32 bits). */
+#define PTD_MAX_TREE_NODES 128
+/* Maximum k of ptd_topk_draft. */
+#define PTD_MAX_TOPK 16
+
+/* A batch of draft/candidate trees (Sec. 3.1 "Tree Construction": every node has a
+ * unique parent P(v); node v sees pi(v) = {v} U pi(P(v))). */
+typedef struct {
+  int32_t batch;               /* host: B >= 1                                        */
+  int32_t total_nodes;         /* host: N_tot = node_offsets[B]                       */
+  int32_t max_nodes;           /* host: max_b T_b, 1..PTD_MAX_TREE_NODES              */
+  int32_t max_ctx;             /* host: upper bound of every ctx_lens[b] (>= 0)       */
+  const int32_t* node_offsets; /* [B+1], node_offsets[0] = 0, non-decreasing          */
+  const int32_t* parents;      /* [N_tot], tree-local parent index, -1 for the root   */
+  const int32_t* ctx_lens;     /* [B], committed prefix length C_b                    */
+} ptd_tree;
+
+/* The per-layer K/V cache of the target model.
+ * Contiguous (page_size == 0): k, v are [num_layers][B][seq_capacity][Hkv][D].
+ * Paged (page_size in {16, 32, 64, 128}): k, v are [num_layers][num_pages][page_size][Hkv][D]
+ *   and slot s of sequence b lives in page block_table[b * max_pages + s / page_size]
+ *   (the same page index in every layer).
+ * Element type `dtype`; rows of one slot (all KV heads) are contiguous. */
+typedef struct {
+  void* k;
+  void* v;
+  ptd_dtype dtype;
+  int32_t num_layers;
+  int32_t num_kv_heads;        /* Hkv                                                  */
+  int32_t head_dim;            /* D: 128 for bf16; 32, 64 or 128 for f32               */
+  int32_t page_size;           /* 0 = contiguous                                       */
+  int32_t seq_capacity;        /* contiguous: slots per sequence (>= C_b + T_b)        */
+  int32_t num_pages;           /* paged: pages per layer                               */
+  const int32_t* block_table;  /* paged: [B][max_pages]                                */
+  int32_t max_pages;           /* paged: entries per block-table row                   */
+} ptd_kv_cache;
+
+/* Bytes of scratch `ptd_tree_attention` wants for these shapes (0 if it needs none).
+ * Passing less (even 0 with a NULL pointer) is allowed: the call then uses fewer
+ * key splits, down to one split which needs no scratch. */
+size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache,
+                                    int32_t num_q_heads, int32_t num_layers);
+
+/* Tree-masked attention (Sec. 3.1 ancestor-only visibility; Sec. 3.2 one pass over
+ * [X; T; C_X]).  For every layer l in [layer_begin, layer_begin + num_layers), tree b,
+ * node i and query head h (KV head h / (Hq / Hkv)):
+ *     out[l'][n][h] = sum_j softmax_j(scale * <q[l'][n][h], K[l][b][j]>) V[l][b][j]
+ * over the slots j in [0, C_b) U { C_b + a : a in pi(i) }, where n = node_offsets[b] + i
+ * and l' = l - layer_begin.
+ *   q, out: [num_layers][N_tot][num_q_heads][D], element type = cache->dtype (fp32
+ *           accumulation; bf16 output rounded to nearest even).
+ *   scale:  <= 0 selects 1/sqrt(D).
+ *   workspace/workspace_bytes: scratch from ptd_attention_workspace_size (may be less).
+ *   dev_status: device int32, atomicMax'ed with PTD_ERR_INVALID_TREE if a tree is
+ *           invalid (that tree's outputs are zero) or PTD_ERR_TIMEOUT.
+ * The tree's own K/V must already be in slots C_b .. C_b + T_b - 1 (position
+ * encoding is applied by the caller before the call). */
+ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache,
+                              int32_t layer_begin, int32_t num_layers,
+                              const void* q, int32_t num_q_heads, float scale, void* out,
+                              void* workspace, size_t workspace_bytes,
+                              int32_t* dev_status, void* stream);
+
+/* Per-node top-k of the logits (Sec. 3.1 "Progressive Expansion": each node's draft
+ * token d_v; "Width Control": at most k children; Sec. 3.2: greedy V_n = entry 0).
+ *   logits: [rows][row_stride] of `dtype`, the first `vocab` entries of a row are used.
+ *   out_idx: [rows][k] int32, out_val: [rows][k] fp32 (exact value of the logit).
+ *   Order: value descending; equal values by lower index first; -0.0 equals +0.0.
+ *   NaN logits are not supported (their placement is unspecified).
+ *   1 <= k <= min(PTD_MAX_TOPK, vocab). */
+ptd_status ptd_topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab,
+                          int64_t row_stride, int32_t k, int32_t* out_idx, float* out_val,
+                          void* stream);
+
+/* Greedy verification (Sec. 3.2): with V_n = target[n * target_stride] (the greedy
+ * token of node n, e.g. column 0 of ptd_topk_draft's out_idx with stride k), the
+ * eligible edges are I = {(n, c) : c child of n, tokens[c] = V_n}; the accepted path is
+ * the longest root path n_0 = 0, n_1, ..., n_m with every edge in I (ties: the
+ * lexicographically smallest node sequence), and X' = (n_0, ..., n_m, V_{n_m}).
+ *   tokens: [N_tot] token of each node;  target: greedy token per node (stride in int32s).
+ *   accepted_nodes: [B][max_nodes] tree-local node ids of the path (entries >= accept_len
+ *       are set to -1);  accept_len: [B] = m + 1 (0 if the tree is invalid);
+ *   bonus_token: [B] = V_{n_m} (-1 if the tree is invalid). */
+ptd_status ptd_verify_greedy(const ptd_tree* tree, const int32_t* tokens, const int32_t* target,
+                             int32_t target_stride, int32_t* accepted_nodes, int32_t* accept_len,
+                             int32_t* bonus_token, int32_t* dev_status, void* stream);
+
+/* KV-cache compaction (Alg. 1 step 6: X' joins the prefix): for every layer, K and V,
+ * slot C_b + j receives the pre-call content of slot C_b + accepted_nodes[b][j] for
+ * j < accept_len[b]; slots below C_b are untouched; new_ctx_lens[b] = C_b + accept_len[b]
+ * (C_b when accept_len[b] = 0).  Overlapping sources and destinations are handled
+ * (the result equals a copy from a snapshot).  Slots >= new_ctx_lens[b] are left with
+ * unspecified content.  accepted_nodes must be a root path of tree b (as written by
+ * ptd_verify_greedy); it is read with stride tree->max_nodes. */
+ptd_status ptd_kv_compact(const ptd_tree* tree, const ptd_kv_cache* cache,
+                          const int32_t* accepted_nodes, const int32_t* accept_len,
+                          int32_t* new_ctx_lens, void* stream);
+
+/* One whole tree-verify step on device buffers: attention over all cache layers,
+ * top-k of the logits, greedy verification on top-k column 0, KV compaction.
+ * Equivalent to the four calls above in that order on `stream`. */
+typedef struct {
+  const void* q;               /* [L][N_tot][Hq][D]                                    */
+  int32_t num_q_heads;
+  float scale;                 /* <= 0: 1/sqrt(D)                                      */
+  void* attn_out;              /* [L][N_tot][Hq][D]                                    */
+  const void* logits;          /* [N_tot][vocab] of logits_dtype                       */
+  ptd_dtype logits_dtype;
+  int32_t vocab;
+  int32_t k;
+  const int32_t* tokens;       /* [N_tot]                                              */
+  int32_t* topk_idx;           /* [N_tot][k]                                           */
+  float* topk_val;             /* [N_tot][k]                                           */
+  int32_t* accepted_nodes;     /* [B][max_nodes]                                       */
+  int32_t* accept_len;         /* [B]                                                  */
+  int32_t* bonus_token;        /* [B]                                                  */
+  int32_t* new_ctx_lens;       /* [B]                                                  */
+  int32_t* dev_status;         /* [1]                                                  */
+  void* workspace;
+  size_t workspace_bytes;
+} ptd_step_args;
+
+ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
+                                const ptd_step_args* args, void* stream);
+
+/* The same step fed from and drained to HOST memory (pinned for asynchronous copies):
+ * copies the host inputs into the device buffers named by `tree`, `cache` and `args`,
+ * runs ptd_tree_verify_step, and copies the small results back.  Contiguous caches only.
+ * Host inputs: q_h [L][N_tot][Hq][D]; logits_h [N_tot][vocab]; tokens_h [N_tot];
+ *   parents_h [N_tot]; node_offsets_h [B+1]; ctx_lens_h [B] (also used on the host to
+ *   place the tree rows); tree_k_h, tree_v_h [L][N_tot][Hkv][D] (node n of tree b goes to
+ *   slot ctx_lens_h[b] + (n - node_offsets_h[b])).
+ * Host outputs: topk_idx_h, topk_val_h [N_tot][k]; accepted_h [B][max_nodes];
+ *   accept_len_h, bonus_h, new_ctx_h [B]; status_h [1].
+ * Returns after enqueueing; the host outputs are valid after the stream synchronises. */
+typedef struct {
+  const void* q_h;
+  const void* logits_h;
+  const int32_t* tokens_h;
+  const int32_t* parents_h;
+  const int32_t* node_offsets_h;
+  const int32_t* ctx_lens_h;
+  const void* tree_k_h;
+  const void* tree_v_h;
+  int32_t* topk_idx_h;
+  float* topk_val_h;
+  int32_t* accepted_h;
+  int32_t* accept_len_h;
+  int32_t* bonus_h;
+  int32_t* new_ctx_h;
+  int32_t* status_h;
+} ptd_host_io;
+
+ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* cache,
+                                     const ptd_step_args* args, const ptd_host_io* io,
+                                     void* stream);
+
+/* Number of kernels the last successful call of each entry point enqueued on this
+ * host thread (a diagnostic for launch accounting). */
+int32_t ptd_last_launch_count(void);
+
+/* Static description of a status code. */
+const char* ptd_status_string(ptd_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PTD_H_ */

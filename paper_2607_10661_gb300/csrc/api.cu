@@ -1,0 +1,376 @@
+// C ABI of the PTD tree-verify step: host-side argument checks, scratch sizing, TMA
+// descriptor encoding and kernel launches.  No allocation, no synchronisation: every
+// call enqueues on the caller's stream (declared in include/ptd.h).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstddef>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/ptd.h"
+#include "attention.cuh"
+#include "topk.cuh"
+#include "verify_compact.cuh"
+
+namespace {
+
+thread_local int32_t g_last_launches = 0;
+
+constexpr int kMaxSplits = 16;
+constexpr int kMaxDevices = 64;
+
+int num_sms_of_current_device() {
+  static int cache[kMaxDevices] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (dev >= 0 && dev < kMaxDevices && cache[dev] > 0) return cache[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+  if (dev >= 0 && dev < kMaxDevices) cache[dev] = n;
+  return n;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t dtype_size(ptd_dtype d) { return d == PTD_BF16 ? 2 : 4; }
+
+ptd_status check_tree(const ptd_tree* t) {
+  if (!t || t->batch < 1 || t->total_nodes < 1 || t->max_nodes < 1 || t->max_nodes > PTD_MAX_TREE_NODES ||
+      t->max_ctx < 0 || !t->node_offsets || !t->parents || !t->ctx_lens)
+    return PTD_ERR_INVALID_ARG;
+  if ((int64_t)t->total_nodes > (int64_t)t->batch * t->max_nodes) return PTD_ERR_INVALID_ARG;
+  return PTD_OK;
+}
+
+ptd_status check_cache(const ptd_kv_cache* c) {
+  if (!c || !c->k || !c->v || c->num_layers < 1 || c->num_kv_heads < 1 || c->head_dim < 1) return PTD_ERR_INVALID_ARG;
+  if (c->dtype != PTD_BF16 && c->dtype != PTD_F32) return PTD_ERR_INVALID_ARG;
+  if (c->page_size < 0) return PTD_ERR_INVALID_ARG;
+  if (c->page_size == 0) {
+    if (c->seq_capacity < 1) return PTD_ERR_INVALID_ARG;
+  } else {
+    if (c->page_size != 16 && c->page_size != 32 && c->page_size != 64 && c->page_size != 128)
+      return PTD_ERR_UNSUPPORTED;
+    if (c->num_pages < 1 || c->max_pages < 1 || !c->block_table) return PTD_ERR_INVALID_ARG;
+  }
+  if (!aligned16(c->k) || !aligned16(c->v)) return PTD_ERR_INVALID_ARG;
+  if (((size_t)c->num_kv_heads * c->head_dim * dtype_size(c->dtype)) % 16 != 0) return PTD_ERR_UNSUPPORTED;
+  return PTD_OK;
+}
+
+int64_t cache_rows_per_layer(const ptd_kv_cache* c, int batch) {
+  return c->page_size > 0 ? (int64_t)c->num_pages * c->page_size : (int64_t)batch * c->seq_capacity;
+}
+
+bool use_tensor_cores(const ptd_kv_cache* c) { return c->dtype == PTD_BF16 && c->head_dim == 128; }
+
+// Number of 256-row M-tile pairs per (tree, KV head) and work units of the tensor-core path.
+void tc_geometry(const ptd_tree* t, const ptd_kv_cache* c, int hq, int layers, int* pairs, int* units,
+                 int* n_kt_max) {
+  const int G = hq / c->num_kv_heads;
+  const int rows = t->max_nodes * G;
+  const int tiles = (rows + 127) / 128;
+  *pairs = (tiles + 1) / 2;
+  *units = layers * t->batch * c->num_kv_heads * (*pairs);
+  *n_kt_max = (t->max_ctx + t->max_nodes + 127) / 128;
+}
+
+// Split count: minimise (waves of CTAs) x (key tiles per CTA + fixed cost); one split
+// needs no scratch and no combine pass, so it wins ties.
+int choose_splits(int units, int n_kt, int sms) {
+  int best = 1;
+  double best_cost = 1e300;
+  for (int s = 1; s <= kMaxSplits && s <= n_kt; ++s) {
+    const double waves = std::ceil((double)units * s / sms);
+    const double cost = waves * (std::ceil((double)n_kt / s) + 2.0) + (s > 1 ? 1.0 : 0.0);
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best = s;
+    }
+  }
+  return best;
+}
+
+size_t split_workspace_bytes(int units, int splits, int head_dim) {
+  if (splits <= 1) return 0;
+  return (size_t)units * splits * 256 * ((size_t)head_dim + 2) * sizeof(float);
+}
+
+ptd_status cuda_status(cudaError_t e) { return e == cudaSuccess ? PTD_OK : PTD_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+const char* ptd_status_string(ptd_status s) {
+  switch (s) {
+    case PTD_OK:
+      return "ok";
+    case PTD_ERR_INVALID_ARG:
+      return "invalid argument";
+    case PTD_ERR_INVALID_TREE:
+      return "invalid tree (parent array is not a rooted tree in topological order)";
+    case PTD_ERR_UNSUPPORTED:
+      return "unsupported shape or dtype";
+    case PTD_ERR_CUDA:
+      return "CUDA error";
+    case PTD_ERR_TIMEOUT:
+      return "device wait timed out";
+    case PTD_ERR_WORKSPACE:
+      return "workspace missing or too small";
+  }
+  return "unknown status";
+}
+
+int32_t ptd_last_launch_count(void) { return g_last_launches; }
+
+size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t num_q_heads,
+                                    int32_t num_layers) {
+  if (check_tree(tree) != PTD_OK || check_cache(cache) != PTD_OK || num_q_heads < 1 || num_layers < 1 ||
+      num_q_heads % cache->num_kv_heads != 0 || !use_tensor_cores(cache))
+    return 0;
+  int pairs, units, n_kt;
+  tc_geometry(tree, cache, num_q_heads, num_layers, &pairs, &units, &n_kt);
+  const int s = choose_splits(units, n_kt, num_sms_of_current_device());
+  return split_workspace_bytes(units, s, cache->head_dim);
+}
+
+ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
+                              int32_t num_layers, const void* q, int32_t num_q_heads, float scale, void* out,
+                              void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  ptd_status st = check_tree(tree);
+  if (st != PTD_OK) return st;
+  if ((st = check_cache(cache)) != PTD_OK) return st;
+  if (!q || !out || !dev_status || num_q_heads < 1 || num_layers < 1 || layer_begin < 0 ||
+      layer_begin + num_layers > cache->num_layers || num_q_heads % cache->num_kv_heads != 0)
+    return PTD_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(out)) return PTD_ERR_INVALID_ARG;
+  const int D = cache->head_dim;
+  ptd::AttnParams p = {};
+  p.q = q;
+  p.out = out;
+  p.node_offsets = tree->node_offsets;
+  p.parents = tree->parents;
+  p.ctx_lens = tree->ctx_lens;
+  p.block_table = cache->block_table;
+  p.k = cache->k;
+  p.v = cache->v;
+  p.dev_status = dev_status;
+  p.batch = tree->batch;
+  p.hq = num_q_heads;
+  p.hkv = cache->num_kv_heads;
+  p.group = num_q_heads / cache->num_kv_heads;
+  p.head_dim = D;
+  p.layer_begin = layer_begin;
+  p.layers = num_layers;
+  p.n_total = tree->total_nodes;
+  p.max_nodes = tree->max_nodes;
+  p.page_size = cache->page_size;
+  p.seq_capacity = cache->seq_capacity;
+  p.num_pages = cache->num_pages;
+  p.max_pages = cache->max_pages;
+  const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)D);
+  p.scale = sc;
+  p.scale_log2 = sc * 1.4426950408889634f;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  if (cache->dtype == PTD_F32) {
+    if (D != 32 && D != 64 && D != 128) return PTD_ERR_UNSUPPORTED;
+    p.splits = 1;
+    p.pairs = 1;
+    st = cuda_status(ptd::launch_tree_attn_simt(p, s));
+    if (st == PTD_OK) g_last_launches = 1;
+    return st;
+  }
+  if (!use_tensor_cores(cache)) return PTD_ERR_UNSUPPORTED;
+
+  int pairs, units, n_kt;
+  tc_geometry(tree, cache, num_q_heads, num_layers, &pairs, &units, &n_kt);
+  if (units <= 0) return PTD_ERR_INVALID_ARG;
+  int splits = choose_splits(units, n_kt, num_sms_of_current_device());
+  while (splits > 1 && (workspace == nullptr || split_workspace_bytes(units, splits, D) > workspace_bytes)) --splits;
+  p.pairs = pairs;
+  p.splits = splits;
+  if (splits > 1) {
+    if (!aligned16(workspace)) return PTD_ERR_WORKSPACE;
+    p.part_o = static_cast<float*>(workspace);
+    p.part_ml = p.part_o + (size_t)units * splits * 256 * D;
+  }
+
+  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+  if (!enc) return PTD_ERR_CUDA;
+  const int64_t rows_per_layer = cache_rows_per_layer(cache, tree->batch);
+  const cuuint64_t gdim[3] = {(cuuint64_t)D, (cuuint64_t)cache->num_kv_heads,
+                              (cuuint64_t)(rows_per_layer * cache->num_layers)};
+  const cuuint64_t gstride[2] = {(cuuint64_t)D * 2, (cuuint64_t)cache->num_kv_heads * D * 2};
+  const cuuint32_t box[3] = {64, 1, (cuuint32_t)(cache->page_size > 0 ? cache->page_size : 128)};
+  const cuuint32_t estride[3] = {1, 1, 1};
+  CUtensorMap map_k, map_v;
+  if (enc(&map_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, cache->k, gdim, gstride, box, estride,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return PTD_ERR_CUDA;
+  if (enc(&map_v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, cache->v, gdim, gstride, box, estride,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return PTD_ERR_CUDA;
+
+  if ((st = cuda_status(ptd::launch_tree_attn_tc(map_k, map_v, p, units, s))) != PTD_OK) return st;
+  int launches = 1;
+  if (splits > 1) {
+    if ((st = cuda_status(ptd::launch_attn_combine(p, units, s))) != PTD_OK) return st;
+    ++launches;
+  }
+  g_last_launches = launches;
+  return PTD_OK;
+}
+
+ptd_status ptd_topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab, int64_t row_stride,
+                          int32_t k, int32_t* out_idx, float* out_val, void* stream) {
+  g_last_launches = 0;
+  if (!logits || !out_idx || !out_val || rows < 1 || vocab < 1 || row_stride < vocab || k < 1 ||
+      k > PTD_MAX_TOPK || k > vocab)
+    return PTD_ERR_INVALID_ARG;
+  if (dtype != PTD_BF16 && dtype != PTD_F32) return PTD_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(logits) % dtype_size(dtype)) != 0) return PTD_ERR_INVALID_ARG;
+  const ptd_status st = cuda_status(ptd::launch_topk(logits, dtype == PTD_BF16, rows, vocab, row_stride, k, out_idx,
+                                                     out_val, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+ptd_status ptd_verify_greedy(const ptd_tree* tree, const int32_t* tokens, const int32_t* target,
+                             int32_t target_stride, int32_t* accepted_nodes, int32_t* accept_len,
+                             int32_t* bonus_token, int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  ptd_status st = check_tree(tree);
+  if (st != PTD_OK) return st;
+  if (!tokens || !target || target_stride < 1 || !accepted_nodes || !accept_len || !bonus_token || !dev_status)
+    return PTD_ERR_INVALID_ARG;
+  st = cuda_status(ptd::launch_verify(tree->node_offsets, tree->parents, tokens, target, target_stride, tree->batch,
+                                      tree->total_nodes, tree->max_nodes, accepted_nodes, accept_len, bonus_token,
+                                      dev_status, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+ptd_status ptd_kv_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* accepted_nodes,
+                          const int32_t* accept_len, int32_t* new_ctx_lens, void* stream) {
+  g_last_launches = 0;
+  ptd_status st = check_tree(tree);
+  if (st != PTD_OK) return st;
+  if ((st = check_cache(cache)) != PTD_OK) return st;
+  if (!accepted_nodes || !accept_len || !new_ctx_lens) return PTD_ERR_INVALID_ARG;
+  if (new_ctx_lens == tree->ctx_lens) return PTD_ERR_INVALID_ARG;   // other CTAs still read ctx_lens
+  const int row_bytes = cache->num_kv_heads * cache->head_dim * (int)dtype_size(cache->dtype);
+  st = cuda_status(ptd::launch_compact(cache->k, cache->v, row_bytes, cache->num_layers, tree->batch,
+                                       cache->page_size, cache->seq_capacity, cache->num_pages, cache->block_table,
+                                       cache->max_pages, tree->ctx_lens, accepted_nodes, accept_len,
+                                       tree->max_nodes, new_ctx_lens, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a,
+                                void* stream) {
+  if (!a) return PTD_ERR_INVALID_ARG;
+  int total = 0;
+  ptd_status st = ptd_tree_attention(tree, cache, 0, cache ? cache->num_layers : 0, a->q, a->num_q_heads, a->scale,
+                                     a->attn_out, a->workspace, a->workspace_bytes, a->dev_status, stream);
+  if (st != PTD_OK) return st;
+  total += g_last_launches;
+  st = ptd_topk_draft(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
+                      a->topk_val, stream);
+  if (st != PTD_OK) return st;
+  total += g_last_launches;
+  st = ptd_verify_greedy(tree, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len, a->bonus_token,
+                         a->dev_status, stream);
+  if (st != PTD_OK) return st;
+  total += g_last_launches;
+  st = ptd_kv_compact(tree, cache, a->accepted_nodes, a->accept_len, a->new_ctx_lens, stream);
+  if (st != PTD_OK) return st;
+  total += g_last_launches;
+  g_last_launches = total;
+  return PTD_OK;
+}
+
+ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a,
+                                     const ptd_host_io* io, void* stream) {
+  if (!a || !io) return PTD_ERR_INVALID_ARG;
+  ptd_status st = check_tree(tree);
+  if (st != PTD_OK) return st;
+  if ((st = check_cache(cache)) != PTD_OK) return st;
+  if (cache->page_size != 0) return PTD_ERR_UNSUPPORTED;
+  if (!io->q_h || !io->logits_h || !io->tokens_h || !io->parents_h || !io->node_offsets_h || !io->ctx_lens_h ||
+      !io->tree_k_h || !io->tree_v_h || !io->topk_idx_h || !io->topk_val_h || !io->accepted_h ||
+      !io->accept_len_h || !io->bonus_h || !io->new_ctx_h || !io->status_h)
+    return PTD_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int B = tree->batch, N = tree->total_nodes, L = cache->num_layers;
+  const size_t es = dtype_size(cache->dtype);
+  const size_t slot_bytes = (size_t)cache->num_kv_heads * cache->head_dim * es;
+  const size_t qbytes = (size_t)L * N * a->num_q_heads * cache->head_dim * es;
+  const size_t lbytes = (size_t)N * a->vocab * dtype_size(a->logits_dtype);
+  auto h2d = [&](void* dst, const void* src, size_t n) {
+    return cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s);
+  };
+  cudaError_t e = cudaSuccess;
+  if (e == cudaSuccess) e = h2d(const_cast<void*>(a->q), io->q_h, qbytes);
+  if (e == cudaSuccess) e = h2d(const_cast<void*>(a->logits), io->logits_h, lbytes);
+  if (e == cudaSuccess) e = h2d(const_cast<int32_t*>(a->tokens), io->tokens_h, (size_t)N * 4);
+  if (e == cudaSuccess) e = h2d(const_cast<int32_t*>(tree->parents), io->parents_h, (size_t)N * 4);
+  if (e == cudaSuccess) e = h2d(const_cast<int32_t*>(tree->node_offsets), io->node_offsets_h, (size_t)(B + 1) * 4);
+  if (e == cudaSuccess) e = h2d(const_cast<int32_t*>(tree->ctx_lens), io->ctx_lens_h, (size_t)B * 4);
+  if (e == cudaSuccess) e = cudaMemsetAsync(a->dev_status, 0, 4, s);
+  // the tree's own K/V rows go to slots C_b .. C_b + T_b - 1 of every layer
+  const size_t layer_pitch = (size_t)B * cache->seq_capacity * slot_bytes;
+  for (int b = 0; b < B && e == cudaSuccess; ++b) {
+    const int off = io->node_offsets_h[b], T = io->node_offsets_h[b + 1] - off, C = io->ctx_lens_h[b];
+    if (T < 1 || C < 0 || C + T > cache->seq_capacity) return PTD_ERR_INVALID_ARG;
+    const size_t dst_off = ((size_t)b * cache->seq_capacity + C) * slot_bytes;
+    const size_t src_off = (size_t)off * slot_bytes;
+    for (int kv = 0; kv < 2 && e == cudaSuccess; ++kv) {
+      uint8_t* dst = static_cast<uint8_t*>(kv ? cache->v : cache->k) + dst_off;
+      const uint8_t* src = static_cast<const uint8_t*>(kv ? io->tree_v_h : io->tree_k_h) + src_off;
+      e = cudaMemcpy2DAsync(dst, layer_pitch, src, (size_t)N * slot_bytes, (size_t)T * slot_bytes, (size_t)L,
+                            cudaMemcpyHostToDevice, s);
+    }
+  }
+  if (e != cudaSuccess) return PTD_ERR_CUDA;
+  st = ptd_tree_verify_step(tree, cache, a, stream);
+  if (st != PTD_OK) return st;
+  const int32_t launches = g_last_launches;
+  auto d2h = [&](void* dst, const void* src, size_t n) {
+    return cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, s);
+  };
+  if (e == cudaSuccess) e = d2h(io->topk_idx_h, a->topk_idx, (size_t)N * a->k * 4);
+  if (e == cudaSuccess) e = d2h(io->topk_val_h, a->topk_val, (size_t)N * a->k * 4);
+  if (e == cudaSuccess) e = d2h(io->accepted_h, a->accepted_nodes, (size_t)B * tree->max_nodes * 4);
+  if (e == cudaSuccess) e = d2h(io->accept_len_h, a->accept_len, (size_t)B * 4);
+  if (e == cudaSuccess) e = d2h(io->bonus_h, a->bonus_token, (size_t)B * 4);
+  if (e == cudaSuccess) e = d2h(io->new_ctx_h, a->new_ctx_lens, (size_t)B * 4);
+  if (e == cudaSuccess) e = d2h(io->status_h, a->dev_status, 4);
+  g_last_launches = launches;
+  return e == cudaSuccess ? PTD_OK : PTD_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,10 @@
+// Internal launcher of the per-node top-k kernel (not part of the C ABI).
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+namespace ptd {
+cudaError_t launch_topk(const void* logits, bool bf16, int64_t rows, int vocab, int64_t row_stride, int k,
+                        int32_t* out_idx, float* out_val, cudaStream_t stream);
+}  // namespace ptd

@@ -1,0 +1,79 @@
+"""Device-resident buffers of one tree-verify step for a synthetic workload.
+
+Uploads a `synthetic.Workload` (trees, Q, K/V cache, logits, draft tokens) to one GPU and
+owns every output buffer, so tests and the benchmark can run the step through the C ABI
+(`ptd.tree_verify_step`) or one call at a time.  Layout only: no arithmetic of the step.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import ptd
+from . import synthetic as syn
+
+
+def to_torch(a: np.ndarray, dtype: str) -> torch.Tensor:
+    """Host numpy array (bf16 bit patterns or fp32) as a torch CPU tensor of the matching dtype."""
+    if dtype == "bf16":
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32))
+
+
+class DeviceWorkload:
+    def __init__(self, w: syn.Workload, device="cuda:0", with_step_buffers: bool = True):
+        self.w = w
+        c = w.cfg
+        self.device = torch.device(device)
+        dev = self.device
+        self.tdtype = torch.bfloat16 if c.dtype == "bf16" else torch.float32
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.node_offsets = torch.tensor(w.node_offsets, **i32)
+        self.parents = torch.tensor(w.parents, **i32)
+        self.ctx_lens = torch.tensor(w.ctx_lens, **i32)
+        self.tree = ptd.Tree(self.node_offsets, self.parents, self.ctx_lens, w.max_nodes, w.max_ctx)
+        shape = (c.layers, *w.cache_shape())
+        self.k = torch.empty(shape, dtype=self.tdtype, device=dev)
+        self.v = torch.empty(shape, dtype=self.tdtype, device=dev)
+        self.q = torch.empty((c.layers, w.n_total, c.hq, c.d), dtype=self.tdtype, device=dev)
+        for l in range(c.layers):
+            kl, vl = w.kv_layer(l)
+            self.k[l].copy_(to_torch(kl, c.dtype))
+            self.v[l].copy_(to_torch(vl, c.dtype))
+            self.q[l].copy_(to_torch(w.q_layer(l), c.dtype))
+        self.block_table = torch.tensor(w.block_table, **i32) if c.page_size else None
+        self.cache = ptd.KVCache(self.k, self.v, c.hkv, c.d, c.page_size, self.block_table)
+        self.logits = to_torch(w.logits, c.dtype).to(dev)
+        self.tokens = torch.tensor(w.tokens, **i32)
+        self.attn_out = torch.zeros_like(self.q)
+        self.topk_idx = torch.zeros((w.n_total, c.k), **i32)
+        self.topk_val = torch.zeros((w.n_total, c.k), dtype=torch.float32, device=dev)
+        self.accepted = torch.zeros((c.batch, w.max_nodes), **i32)
+        self.accept_len = torch.zeros(c.batch, **i32)
+        self.bonus = torch.zeros(c.batch, **i32)
+        self.new_ctx = torch.zeros(c.batch, **i32)
+        self.dev_status = torch.zeros(1, **i32)
+        nbytes = ptd.attention_workspace_size(self.tree, self.cache, c.hq)
+        self.workspace = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=dev) if nbytes else None
+        self.bufs = ptd.StepBuffers(self.q, c.hq, self.attn_out, self.logits, c.k, self.tokens, self.topk_idx,
+                                    self.topk_val, self.accepted, self.accept_len, self.bonus, self.new_ctx,
+                                    self.dev_status, self.workspace) if with_step_buffers else None
+
+    # ---- the whole step, or one call at a time ------------------------------------
+    def step(self, stream=None) -> int:
+        self.dev_status.zero_()
+        return ptd.tree_verify_step(self.tree, self.cache, self.bufs, stream)
+
+    def attention(self, stream=None) -> int:
+        return ptd.tree_attention(self.tree, self.cache, self.q, self.attn_out, self.w.cfg.hq, self.dev_status,
+                                  workspace=self.workspace, stream=stream)
+
+    def topk(self, stream=None) -> int:
+        return ptd.topk_draft(self.logits, self.w.cfg.k, self.topk_idx, self.topk_val, stream=stream)
+
+    def verify(self, stream=None) -> int:
+        return ptd.verify_greedy(self.tree, self.tokens, self.topk_idx, self.w.cfg.k, self.accepted,
+                                 self.accept_len, self.bonus, self.dev_status, stream=stream)
+
+    def compact(self, stream=None) -> int:
+        return ptd.kv_compact(self.tree, self.cache, self.accepted, self.accept_len, self.new_ctx, stream=stream)

@@ -1,0 +1,67 @@
+"""The C ABI library builds, loads and exports every function include/ptd.h declares;
+host-side argument checks reject bad calls before touching the GPU (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import __graft_entry__
+    from paper_2607_10661_gb300 import ptd
+
+    __graft_entry__.build()
+    return ptd.lib()
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "ptd.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(ptd_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declares_the_four_steps():
+    names = _declared_functions()
+    for n in ("ptd_tree_attention", "ptd_topk_draft", "ptd_verify_greedy", "ptd_kv_compact"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2607_10661_gb300 import ptd
+
+    names = _declared_functions()
+    assert names, "no declarations parsed"
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(ptd.EXPORTED)
+
+
+def test_status_strings(lib):
+    from paper_2607_10661_gb300 import ptd
+
+    for s in range(7):
+        assert ptd.status_string(s)
+    assert ptd.status_string(0) == "ok"
+
+
+def test_host_checks_reject_without_gpu(lib):
+    from paper_2607_10661_gb300 import ptd
+
+    null = ctypes.c_void_p(0)
+    assert lib.ptd_topk_draft(null, ptd.BF16, 4, 100, 100, 2, null, null, null) == ptd.INVALID_ARG
+    assert lib.ptd_tree_attention(None, None, 0, 1, null, 8, 0.0, null, null, 0, null, null) == ptd.INVALID_ARG
+    assert lib.ptd_verify_greedy(None, null, null, 1, null, null, null, null, null) == ptd.INVALID_ARG
+    assert lib.ptd_kv_compact(None, None, null, null, null, null) == ptd.INVALID_ARG
+    t = ptd._Tree(1, 200, 200, 0, 8, 8, 8)          # max_nodes above 128
+    c = ptd._Cache(16, 16, ptd.BF16, 1, 8, 128, 0, 300, 0, None, 0)
+    assert lib.ptd_tree_attention(ctypes.byref(t), ctypes.byref(c), 0, 1, 16, 32, 0.0, 16, None, 0, 16,
+                                  None) == ptd.INVALID_ARG
+    t = ptd._Tree(1, 10, 10, 0, 8, 8, 8)
+    c = ptd._Cache(16, 16, ptd.BF16, 1, 8, 128, 24, 0, 4, 8, 4)   # page size 24 is not supported
+    assert lib.ptd_tree_attention(ctypes.byref(t), ctypes.byref(c), 0, 1, 16, 32, 0.0, 16, None, 0, 16,
+                                  None) == ptd.UNSUPPORTED
+    assert lib.ptd_attention_workspace_size(ctypes.byref(t), ctypes.byref(c), 32, 1) == 0

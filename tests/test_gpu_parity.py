@@ -1,0 +1,409 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Bit-exact: top-k indices and values, accepted paths / lengths / bonus tokens, compacted
+cache bytes.  Attention: max-abs 2e-2 and mean-abs 2e-3 for bf16 inputs with fp32
+accumulation, 1e-4 for fp32, plus a relative-RMS bound of 1e-2 and small / peaked
+contexts, because at long contexts one wrongly (un)masked tree key moves an output by
+only ~1/C (far below 2e-2).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_10661_gb300 import ptd
+from paper_2607_10661_gb300 import synthetic as syn
+from paper_2607_10661_gb300.harness import DeviceWorkload, to_torch
+
+pytestmark = pytest.mark.gpu
+
+BF16_MAX, BF16_MEAN, REL_RMS = 2e-2, 2e-3, 1e-2
+F32_MAX = 1e-4
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+
+    __graft_entry__.build()
+
+
+def _attn_ref(w, layer, b, heads=None):
+    """Oracle attention of tree b in one layer ([T, Hq, D]); optionally one KV group only."""
+    c = w.cfg
+    q = syn.widen(w.q_layer(layer), c.dtype)[w.nodes_of(b)]
+    kc, vc = (syn.widen(x, c.dtype) for x in w.kv_layer(layer))
+    k, v = w.seq_view(kc, b), w.seq_view(vc, b)
+    if heads is not None:
+        G = c.hq // c.hkv
+        kvh = heads // G
+        q = q[:, kvh * G:(kvh + 1) * G]
+        k, v = k[:, kvh:kvh + 1], v[:, kvh:kvh + 1]
+    return oracle.tree_attention(q, k, v, w.trees[b], int(w.ctx_lens[b]))
+
+
+def _check_attn(got, ref, dtype, what=""):
+    err = np.abs(got - ref)
+    if dtype == "f32":
+        assert err.max() <= F32_MAX, (what, err.max())
+        return
+    assert err.max() <= BF16_MAX, (what, err.max())
+    assert err.mean() <= BF16_MEAN, (what, err.mean())
+    rel = np.sqrt((err ** 2).mean() / max((ref ** 2).mean(), 1e-30))
+    assert rel <= REL_RMS, (what, rel)
+
+
+def _run_attention(w):
+    dw = DeviceWorkload(w, with_step_buffers=False)
+    dw.attention()
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == 0
+    return dw, dw.attn_out.float().cpu().numpy()
+
+
+# ------------------------------------------------------------------------------ attention
+
+ATTN_CASES = {
+    # name: (base config, overrides) -- sizes the oracle finishes in seconds, spanning several
+    # 128-key tiles, a ragged tail, one and two M tiles, splits and the paged layout
+    "tiny-fp32": ("tiny-fp32", {}),
+    "fp32-d128-gqa": ("tiny-fp32", dict(hq=8, hkv=2, d=128, ctx=(300, 300))),
+    "llama2-layer-short": ("llama2-7b-layer", dict(hq=8, hkv=8, ctx=(333, 333), vocab=100)),
+    "llama3-gqa-2layers": ("llama3-8b-gqa", dict(layers=2, ctx=(1000, 1000), vocab=100)),
+    "llama3-gqa-ctx0": ("llama3-8b-gqa", dict(layers=1, ctx=(0, 0), vocab=100)),
+    "llama3-gqa-ctx1": ("llama3-8b-gqa", dict(layers=1, ctx=(1, 1), vocab=100)),
+    "llama3-gqa-ctx7": ("llama3-8b-gqa", dict(layers=1, ctx=(7, 7), vocab=100)),
+    "llama3-gqa-ctx65": ("llama3-8b-gqa", dict(layers=1, ctx=(65, 65), vocab=100)),
+    "llama3-gqa-ctx128": ("llama3-8b-gqa", dict(layers=1, ctx=(128, 128), vocab=100)),
+    "batched-paged-short": ("batched-paged", dict(ctx=(100, 700), vocab=100)),
+    "long-context-short": ("long-context", dict(ctx=(3000, 3000), vocab=100)),
+    "chain-128": ("llama3-8b-gqa", dict(layers=1, ctx=(50, 50), vocab=100, tree="chain", nodes=(128, 128))),
+    "single-node": ("llama3-8b-gqa", dict(layers=1, ctx=(200, 200), vocab=100, tree="chain", nodes=(1, 1))),
+    "mha-g1-t64": ("llama2-7b-layer", dict(hq=4, hkv=4, ctx=(129, 129), vocab=100, tree="chain",
+                                           nodes=(64, 64))),
+}
+
+
+@pytest.mark.parametrize("case", list(ATTN_CASES))
+def test_attention_matches_oracle(case):
+    base, over = ATTN_CASES[case]
+    w = syn.Workload(syn.shrink(syn.CONFIGS[base], **over), 11)
+    dw, got = _run_attention(w)
+    for l in range(w.cfg.layers):
+        for b in range(w.cfg.batch):
+            ref = _attn_ref(w, l, b)
+            _check_attn(got[l][w.nodes_of(b)], ref, w.cfg.dtype, f"{case} l{l} b{b}")
+
+
+def test_attention_peaked_context_exposes_mask():
+    """Committed-context keys made to score very low: outputs are dominated by the tree
+    keys, so a wrongly (un)masked ancestor changes an output by O(1)."""
+    cfg = syn.shrink(syn.CONFIGS["llama3-8b-gqa"], layers=1, ctx=(257, 257), vocab=100)
+    w = syn.Workload(cfg, 5)
+    dw = DeviceWorkload(w, with_step_buffers=False)
+    C = int(w.ctx_lens[0])
+    q = syn.widen(w.q_layer(0), "bf16")
+    kc, vc = (syn.widen(x, "bf16") for x in w.kv_layer(0))
+    # context keys = -4 * mean query direction of their group, so scores are strongly negative
+    G = cfg.hq // cfg.hkv
+    for h in range(cfg.hkv):
+        dirn = q[:, h * G:(h + 1) * G].mean(axis=(0, 1))
+        kc[0, :C, h] = -4.0 * dirn / np.linalg.norm(dirn) * np.sqrt(cfg.d)
+    kbits = syn.bf16_bits(kc.astype(np.float32))
+    dw.k[0].copy_(to_torch(kbits, "bf16"))
+    kc = syn.widen(kbits, "bf16")
+    dw.attention()
+    torch.cuda.synchronize()
+    ref = oracle.tree_attention(q, w.seq_view(kc, 0), w.seq_view(vc, 0), w.trees[0], C)
+    got = dw.attn_out[0].float().cpu().numpy()
+    _check_attn(got, ref, "bf16", "peaked")
+    # and the tree part really dominates: dropping the ancestors changes the answer a lot
+    flat = oracle.tree_attention(q, w.seq_view(kc, 0), w.seq_view(vc, 0), [-1] + [0] * (w.n_total - 1), C)
+    assert np.abs(flat - ref).max() > 0.1
+
+
+def test_attention_full_size_llama3_sampled():
+    """32 layers, context 8192, 63 nodes, the launch the benchmark times; oracle on a sample
+    of (layer, KV group) pairs."""
+    w = syn.Workload(syn.CONFIGS["llama3-8b-gqa"], 1000)
+    dw, got = _run_attention(w)
+    G = w.cfg.hq // w.cfg.hkv
+    for l, kvh in ((0, 0), (13, 5), (31, 7)):
+        ref = _attn_ref(w, l, 0, heads=kvh * G)
+        _check_attn(got[l][:, kvh * G:(kvh + 1) * G], ref, "bf16", f"l{l} kv{kvh}")
+
+
+def test_attention_full_size_long_context_sampled():
+    w = syn.Workload(syn.CONFIGS["long-context"], 5000)
+    dw, got = _run_attention(w)
+    G = w.cfg.hq // w.cfg.hkv
+    for kvh in (0, 6):
+        ref = _attn_ref(w, 0, 0, heads=kvh * G)
+        _check_attn(got[0][:, kvh * G:(kvh + 1) * G], ref, "bf16", f"kv{kvh}")
+
+
+def test_attention_full_size_batched_paged():
+    w = syn.Workload(syn.CONFIGS["batched-paged"], 4000)
+    dw, got = _run_attention(w)
+    for b in range(w.cfg.batch):
+        ref = _attn_ref(w, 0, b, heads=(b % w.cfg.hkv) * (w.cfg.hq // w.cfg.hkv))
+        G = w.cfg.hq // w.cfg.hkv
+        kvh = b % w.cfg.hkv
+        _check_attn(got[0][w.nodes_of(b)][:, kvh * G:(kvh + 1) * G], ref, "bf16", f"b{b}")
+
+
+def test_attention_invalid_tree_reports_and_zeroes():
+    cfg = syn.shrink(syn.CONFIGS["llama3-8b-gqa"], layers=1, ctx=(100, 100), vocab=100)
+    w = syn.Workload(cfg, 2)
+    dw = DeviceWorkload(w, with_step_buffers=False)
+    bad = w.parents.copy()
+    bad[5] = 7                                  # parent after the child
+    dw.parents.copy_(torch.tensor(bad))
+    dw.attn_out.fill_(1.0)
+    dw.attention()
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == ptd.INVALID_TREE
+    assert float(dw.attn_out.abs().max()) == 0.0
+
+
+# ------------------------------------------------------------------------------ top-k
+
+@pytest.mark.parametrize("name", syn.CONFIG_ORDER)
+def test_topk_matches_oracle(name):
+    w = syn.Workload(syn.CONFIGS[name], 21)
+    dev = torch.device("cuda:0")
+    logits = to_torch(w.logits, w.cfg.dtype).to(dev)
+    k = w.cfg.k
+    idx = torch.zeros((w.n_total, k), dtype=torch.int32, device=dev)
+    val = torch.zeros((w.n_total, k), dtype=torch.float32, device=dev)
+    ptd.topk_draft(logits, k, idx, val)
+    torch.cuda.synchronize()
+    ref_i, ref_v = oracle.topk_rows(syn.widen(w.logits, w.cfg.dtype), k)
+    assert np.array_equal(idx.cpu().numpy(), ref_i)
+    assert np.array_equal(val.cpu().numpy().astype(np.float64), ref_v)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("vocab,k", [(1, 1), (7, 3), (9, 9), (1001, 16), (32003, 5), (128256, 1), (152067, 16)])
+def test_topk_edge_cases(dtype, vocab, k):
+    g = np.random.default_rng(vocab + k)
+    rows = 37
+    x = np.round(g.standard_normal((rows, vocab)) * 2, 1).astype(np.float32)   # many ties
+    x[:, ::5] = 0.0
+    x[:, 3::7] = -0.0
+    x[0] = 1.5                                                                 # a constant row
+    if dtype == "bf16":
+        bits = syn.bf16_bits(x)
+        host, wide = bits, syn.widen(bits, "bf16")
+    else:
+        host, wide = x, x.astype(np.float64)
+    # row stride not a multiple of 8 elements: rows start at every alignment
+    stride = vocab + 3
+    pad = np.zeros((rows, stride), dtype=host.dtype)
+    pad[:, :vocab] = host
+    t = to_torch(pad, dtype).cuda()
+    idx = torch.zeros((rows, k), dtype=torch.int32, device="cuda")
+    val = torch.zeros((rows, k), dtype=torch.float32, device="cuda")
+    st = ptd.lib().ptd_topk_draft(t.data_ptr(), ptd.BF16 if dtype == "bf16" else ptd.F32, rows, vocab, stride, k,
+                                  idx.data_ptr(), val.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    assert st == ptd.OK
+    torch.cuda.synchronize()
+    ref_i, ref_v = oracle.topk_rows(wide, k)
+    assert np.array_equal(idx.cpu().numpy(), ref_i)
+    assert np.array_equal(val.cpu().numpy().astype(np.float64), ref_v)
+
+
+def test_topk_rejects_bad_k():
+    t = torch.zeros((2, 10), dtype=torch.bfloat16, device="cuda")
+    idx = torch.zeros((2, 17), dtype=torch.int32, device="cuda")
+    val = torch.zeros((2, 17), dtype=torch.float32, device="cuda")
+    with pytest.raises(ptd.PtdError):
+        ptd.topk_draft(t, 17, idx, val)
+    with pytest.raises(ptd.PtdError):
+        ptd.topk_draft(t, 11, idx, val)
+
+
+# ------------------------------------------------------------------------------ verify
+
+def _verify_gpu(trees, tokens, target, max_nodes=None):
+    dev = "cuda"
+    offs = np.zeros(len(trees) + 1, np.int32)
+    offs[1:] = np.cumsum([len(t) for t in trees])
+    max_nodes = max_nodes or max(len(t) for t in trees)
+    tree = ptd.Tree(torch.tensor(offs, device=dev), torch.tensor(np.concatenate(trees).astype(np.int32), device=dev),
+                    torch.zeros(len(trees), dtype=torch.int32, device=dev), max_nodes, 0)
+    B = len(trees)
+    acc = torch.full((B, max_nodes), 77, dtype=torch.int32, device=dev)
+    alen = torch.zeros(B, dtype=torch.int32, device=dev)
+    bonus = torch.zeros(B, dtype=torch.int32, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    ptd.verify_greedy(tree, torch.tensor(tokens, dtype=torch.int32, device=dev),
+                      torch.tensor(target, dtype=torch.int32, device=dev), 1, acc, alen, bonus, st)
+    torch.cuda.synchronize()
+    return acc.cpu().numpy(), alen.cpu().numpy(), bonus.cpu().numpy(), int(st.item())
+
+
+def _expect_verify(trees, tokens, target, acc, alen, bonus):
+    off = 0
+    for b, par in enumerate(trees):
+        T = len(par)
+        path, n, bo = oracle.verify_greedy(par, tokens[off:off + T], target[off:off + T])
+        assert alen[b] == n and bonus[b] == bo, (b, n, alen[b])
+        assert acc[b, :n].tolist() == path
+        assert (acc[b, n:] == -1).all()
+        off += T
+
+
+@pytest.mark.parametrize("name", syn.CONFIG_ORDER)
+def test_verify_on_workloads(name):
+    cfg = syn.CONFIGS[name]
+    w = syn.Workload(syn.shrink(cfg, vocab=min(cfg.vocab, 3000)), 31)
+    idx, _ = oracle.topk_rows(syn.widen(w.logits, w.cfg.dtype), 1)
+    acc, alen, bonus, st = _verify_gpu(w.trees, w.tokens, idx[:, 0], w.max_nodes)
+    assert st == 0
+    _expect_verify(w.trees, w.tokens, idx[:, 0], acc, alen, bonus)
+
+
+def test_verify_random_trees_dense_matches_and_ties():
+    """Small alphabet: many eligible edges, duplicate sibling tokens (ties broken by the
+    lexicographically smallest path), batch of ragged trees up to 128 nodes."""
+    g = np.random.default_rng(3)
+    for trial in range(20):
+        trees, toks, tgts = [], [], []
+        for b in range(int(g.integers(1, 9))):
+            T = int(g.choice([1, 2, 3, 7, 31, 64, 127, 128]))
+            par = np.array([-1] + [int(g.integers(max(0, i - 4), i)) for i in range(1, T)], np.int32)
+            trees.append(par)
+            toks.append(g.integers(0, 2, size=T))
+            tgts.append(g.integers(0, 2, size=T))
+        tokens, target = np.concatenate(toks).astype(np.int32), np.concatenate(tgts).astype(np.int32)
+        acc, alen, bonus, st = _verify_gpu(trees, tokens, target)
+        assert st == 0
+        _expect_verify(trees, tokens, target, acc, alen, bonus)
+
+
+def test_verify_full_chain_accepts_all_128():
+    par = np.arange(-1, 127, dtype=np.int32)
+    tokens = np.arange(128, dtype=np.int32)
+    target = np.arange(1, 129, dtype=np.int32)      # V_n = token of node n+1
+    acc, alen, bonus, st = _verify_gpu([par], tokens, target)
+    assert st == 0 and alen[0] == 128 and bonus[0] == 128 and acc[0].tolist() == list(range(128))
+
+
+def test_verify_invalid_tree():
+    good = np.array([-1, 0, 0, 1], np.int32)
+    bad = np.array([-1, 0, 3, 1], np.int32)
+    acc, alen, bonus, st = _verify_gpu([good, bad], np.zeros(8, np.int32), np.zeros(8, np.int32))
+    assert st == ptd.INVALID_TREE
+    assert alen[1] == 0 and bonus[1] == -1 and (acc[1] == -1).all()
+    assert alen[0] == 3   # the valid tree is still verified (all tokens and targets 0)
+
+
+# ------------------------------------------------------------------------------ compaction
+
+@pytest.mark.parametrize("name", ["llama3-8b-gqa", "batched-paged", "tiny-fp32"])
+def test_compact_matches_oracle(name):
+    cfg = syn.CONFIGS[name]
+    over = dict(vocab=min(cfg.vocab, 2000))
+    if name == "llama3-8b-gqa":
+        over.update(layers=3, ctx=(300, 300))
+    w = syn.Workload(syn.shrink(cfg, **over), 41)
+    cfg = w.cfg
+    dw = DeviceWorkload(w, with_step_buffers=False)
+    # a chosen root path per tree: the deepest node's ancestors (long, overlapping copies)
+    B, M = cfg.batch, w.max_nodes
+    acc = np.full((B, M), -1, np.int32)
+    alen = np.zeros(B, np.int32)
+    for b, par in enumerate(w.trees):
+        d = oracle.depths(par)
+        end = int(np.argmax(d))
+        path = [end]
+        while par[path[-1]] >= 0:
+            path.append(int(par[path[-1]]))
+        path.reverse()
+        acc[b, :len(path)] = path
+        alen[b] = len(path)
+    k_before, v_before = dw.k.cpu(), dw.v.cpu()
+    dw.accepted.copy_(torch.tensor(acc))
+    dw.accept_len.copy_(torch.tensor(alen))
+    dw.compact()
+    torch.cuda.synchronize()
+    k_after, v_after = dw.k.cpu(), dw.v.cpu()
+    assert dw.new_ctx.cpu().numpy().tolist() == (w.ctx_lens + alen).tolist()
+    for before, after in ((k_before, k_after), (v_before, v_after)):
+        bb = before.view(torch.int16).numpy() if before.dtype == torch.bfloat16 else before.numpy()
+        aa = after.view(torch.int16).numpy() if after.dtype == torch.bfloat16 else after.numpy()
+        for l in range(cfg.layers):
+            for b in range(B):
+                C = int(w.ctx_lens[b])
+                n = int(alen[b])
+                seq_b = w.seq_view(bb[l], b)
+                seq_a = w.seq_view(aa[l], b)
+                ref, new_ctx = oracle.kv_compact(seq_b, acc[b, :n], C)
+                assert np.array_equal(seq_a[:new_ctx], ref[:new_ctx])
+
+
+# ------------------------------------------------------------------------------ whole step
+
+@pytest.mark.parametrize("case", ["tiny-fp32", "llama3-gqa-2layers", "batched-paged-short"])
+def test_whole_step_matches_oracle(case):
+    base, over = ATTN_CASES[case]
+    cfg = syn.shrink(syn.CONFIGS[base], **over)
+    w = syn.Workload(cfg, 51)
+    dw = DeviceWorkload(w)
+    k_before = dw.k.cpu()
+    n = dw.step()
+    assert n >= 4
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == 0
+    got = dw.attn_out.float().cpu().numpy()
+    for b in range(cfg.batch):
+        _check_attn(got[0][w.nodes_of(b)], _attn_ref(w, 0, b), cfg.dtype, f"step b{b}")
+    idx_ref, _ = oracle.topk_rows(syn.widen(w.logits, cfg.dtype), cfg.k)
+    assert np.array_equal(dw.topk_idx.cpu().numpy(), idx_ref)
+    kb = k_before.view(torch.int16).numpy() if k_before.dtype == torch.bfloat16 else k_before.numpy()
+    ka = dw.k.cpu()
+    ka = ka.view(torch.int16).numpy() if ka.dtype == torch.bfloat16 else ka.numpy()
+    for b, par in enumerate(w.trees):
+        sl = w.nodes_of(b)
+        path, nacc, bonus = oracle.verify_greedy(par, w.tokens[sl], idx_ref[sl, 0])
+        assert int(dw.accept_len[b]) == nacc and int(dw.bonus[b]) == bonus
+        assert dw.accepted[b, :nacc].cpu().tolist() == path
+        ref, new_ctx = oracle.kv_compact(w.seq_view(kb[0], b), path, int(w.ctx_lens[b]))
+        assert int(dw.new_ctx[b]) == new_ctx
+        assert np.array_equal(w.seq_view(ka[0], b)[:new_ctx], ref[:new_ctx])
+
+
+def test_host_step_matches_device_step():
+    """ptd_tree_verify_step_host (pinned host inputs and outputs) gives the device step's results."""
+    cfg = syn.shrink(syn.CONFIGS["llama3-8b-gqa"], layers=2, ctx=(700, 700), vocab=3000)
+    w = syn.Workload(cfg, 61)
+    dw = DeviceWorkload(w)
+    N, L = w.n_total, cfg.layers
+    C = int(w.ctx_lens[0])
+    pin = lambda t: t.contiguous().pin_memory()
+    tree_k = pin(torch.stack([dw.k[l, 0, C:C + N] for l in range(L)]).cpu())
+    tree_v = pin(torch.stack([dw.v[l, 0, C:C + N] for l in range(L)]).cpu())
+    io_t = dict(q_h=pin(dw.q.cpu()), logits_h=pin(dw.logits.cpu()), tokens_h=pin(dw.tokens.cpu()),
+                parents_h=pin(dw.parents.cpu()), node_offsets_h=pin(dw.node_offsets.cpu()),
+                ctx_lens_h=pin(dw.ctx_lens.cpu()), tree_k_h=tree_k, tree_v_h=tree_v,
+                topk_idx_h=pin(torch.zeros((N, cfg.k), dtype=torch.int32)),
+                topk_val_h=pin(torch.zeros((N, cfg.k), dtype=torch.float32)),
+                accepted_h=pin(torch.zeros((1, w.max_nodes), dtype=torch.int32)),
+                accept_len_h=pin(torch.zeros(1, dtype=torch.int32)), bonus_h=pin(torch.zeros(1, dtype=torch.int32)),
+                new_ctx_h=pin(torch.zeros(1, dtype=torch.int32)), status_h=pin(torch.zeros(1, dtype=torch.int32)))
+    io = ptd.HostIO(**io_t)
+    # scramble the device inputs: the host call must overwrite them
+    dw.q.zero_()
+    dw.logits.zero_()
+    n = ptd.tree_verify_step_host(dw.tree, dw.cache, dw.bufs, io)
+    assert n >= 4
+    torch.cuda.synchronize()
+    idx_ref, _ = oracle.topk_rows(syn.widen(w.logits, cfg.dtype), cfg.k)
+    assert np.array_equal(io_t["topk_idx_h"].numpy(), idx_ref)
+    path, nacc, bonus = oracle.verify_greedy(w.trees[0], w.tokens, idx_ref[:, 0])
+    assert int(io_t["accept_len_h"][0]) == nacc and int(io_t["bonus_h"][0]) == bonus
+    assert io_t["accepted_h"][0, :nacc].tolist() == path
+    assert int(io_t["new_ctx_h"][0]) == C + nacc and int(io_t["status_h"][0]) == 0
+    got = dw.attn_out.float().cpu().numpy()
+    _check_attn(got[1], _attn_ref(w, 1, 0), "bf16", "host step")
