@@ -1,0 +1,409 @@
+"""Benchmark of the PTD tree-verify step on GB300.
+
+One step = the whole hot path on one batch of synthetic input: tree-masked attention over
+all 32 layers of the KV cache, per-node top-k of the logits, greedy verification and KV
+compaction, through the C ABI (libptd.so), on the Llama-3-8B-shaped GQA workload
+(32 query / 8 KV heads, head dim 128, committed context 8192, 63-node draft tree,
+vocabulary 128256, top-4).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints one JSON line (rank 0).  `value` is whole-job steps/s with inputs resident in HBM;
+`e2e` is the same metric through ptd_tree_verify_step_host with pinned host buffers (per
+step: host->device inputs, the step, device->host results, then a stream sync).
+Every step reads ~1.13 GB (more than the 129 MB L2), so no step finds the previous one's
+data in L2.  Under torchrun each rank runs an independent replica (the step has no
+cross-sequence exchange), timing is max over ranks, and value sums all ranks' steps.
+`--impl reference` times the CPU oracle on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "llama3-8b-gqa"
+MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0
+
+
+def _workload_desc(cfg) -> str:
+    return (f"{cfg.name}: {cfg.layers} layers, {cfg.hq}q/{cfg.hkv}kv heads, head_dim {cfg.d}, "
+            f"context {cfg.ctx[0]}, draft tree {cfg.nodes[0]} nodes (branching {','.join(map(str, cfg.branching))} "
+            f"pruned), vocab {cfg.vocab}, top-{cfg.k}, batch {cfg.batch}")
+
+
+def step_bytes(w) -> dict:
+    """Algorithmic bytes of one step: every byte the step must move at least once."""
+    c = w.cfg
+    es = 2 if c.dtype == "bf16" else 4
+    kv = sum(int(s) for s in w.seq_lens) * c.hkv * c.d * es * 2 * c.layers   # K and V, context + tree
+    qo = 2 * c.layers * w.n_total * c.hq * c.d * es                          # Q read, O written
+    logits = w.n_total * c.vocab * es
+    return dict(kv=kv, qo=qo, logits=logits, attention=kv + qo, roofline=kv + logits)
+
+
+def attention_flops(w) -> float:
+    """QK^T and PV over every visible key (context plus the node's ancestors)."""
+    c = w.cfg
+    total = 0
+    for b, par in enumerate(w.trees):
+        depth = np.zeros(len(par), np.int64)
+        for i in range(1, len(par)):
+            depth[i] = depth[par[i]] + 1
+        keys = len(par) * int(w.ctx_lens[b]) + int((depth + 1).sum())
+        total += keys
+    return 4.0 * c.d * c.hq * c.layers * total
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    QUERY = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float) -> dict:
+        rows = []
+        for ts, line in self.lines:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                rows.append((ts, float(parts[0]), float(parts[1]), parts[3:]))
+            except ValueError:
+                continue
+        inside = [r for r in rows if t0 <= r[0] <= t1] or rows
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in inside:
+            for n, v in zip(names, r[3][1:5]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": float(np.median([r[1] for r in inside])), "sm_max_mhz": max(r[2] for r in inside),
+                "reasons": sorted(reasons), "samples": len(inside)}
+
+
+def _peak_hbm():
+    try:
+        with open(MEASURED_PEAKS) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ----------------------------------------------------------------------------- GPU arm
+def run_gpu(args, rank: int, world: int, dist):
+    import torch
+
+    from paper_2607_10661_gb300 import ptd
+    from paper_2607_10661_gb300 import synthetic as syn
+    from paper_2607_10661_gb300.harness import DeviceWorkload
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    import __graft_entry__
+
+    if rank == 0 or not os.path.exists(ptd.LIB_PATH):
+        __graft_entry__.build()
+    if dist is not None:
+        dist.barrier()
+    cfg = syn.CONFIGS[WORKLOAD]
+    if args.layers:
+        cfg = syn.shrink(cfg, layers=args.layers)
+    w = syn.Workload(cfg, 1000 + rank)
+    dw = DeviceWorkload(w, device=f"cuda:{local}")
+    stream = torch.cuda.current_stream()
+    nb = step_bytes(w)
+
+    def one_step(ev=None):
+        n = 0
+        if ev is not None:
+            ev[0].record(stream)
+        n += dw.attention()
+        if ev is not None:
+            ev[1].record(stream)
+        n += dw.topk()
+        n += dw.verify()
+        n += dw.compact()
+        return n
+
+    dw.dev_status.zero_()              # sticky status word: cleared once, read after the run
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.5)
+    for _ in range(args.warmup):
+        one_step()
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == 0, ptd.status_string(int(dw.dev_status.item()))
+
+    K = args.steps
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    start.record(stream)
+    launches = 0
+    for i in range(K):
+        launches += one_step(evs[i])
+    end.record(stream)
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    if dist is not None:
+        dist.barrier()
+    ms = start.elapsed_time(end)
+    attn_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    clocks = sampler.summary(t_wall0, t_wall1)
+    sampler.stop()
+    status = int(dw.dev_status.item())
+
+    # ---- end to end: pinned host inputs and outputs through ptd_tree_verify_step_host
+    N, L = w.n_total, cfg.layers
+    C = int(w.ctx_lens[0])
+    pin = lambda t: t.contiguous().pin_memory()
+    io_t = dict(q_h=pin(dw.q.cpu()), logits_h=pin(dw.logits.cpu()), tokens_h=pin(dw.tokens.cpu()),
+                parents_h=pin(dw.parents.cpu()), node_offsets_h=pin(dw.node_offsets.cpu()),
+                ctx_lens_h=pin(dw.ctx_lens.cpu()),
+                tree_k_h=pin(dw.k[:, 0, C:C + N].cpu()), tree_v_h=pin(dw.v[:, 0, C:C + N].cpu()),
+                topk_idx_h=pin(torch.zeros((N, cfg.k), dtype=torch.int32)),
+                topk_val_h=pin(torch.zeros((N, cfg.k), dtype=torch.float32)),
+                accepted_h=pin(torch.zeros((cfg.batch, w.max_nodes), dtype=torch.int32)),
+                accept_len_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
+                bonus_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
+                new_ctx_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
+                status_h=pin(torch.zeros(1, dtype=torch.int32)))
+    io = ptd.HostIO(**io_t)
+    h2d = sum(io_t[n].numel() * io_t[n].element_size() for n in
+              ("q_h", "logits_h", "tokens_h", "parents_h", "node_offsets_h", "ctx_lens_h", "tree_k_h", "tree_v_h"))
+    d2h = sum(io_t[n].numel() * io_t[n].element_size() for n in
+              ("topk_idx_h", "topk_val_h", "accepted_h", "accept_len_h", "bonus_h", "new_ctx_h", "status_h"))
+    for _ in range(3):
+        ptd.tree_verify_step_host(dw.tree, dw.cache, dw.bufs, io)
+        stream.synchronize()
+    Ke = max(10, K // 5)
+    if dist is not None:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(Ke):
+        ptd.tree_verify_step_host(dw.tree, dw.cache, dw.bufs, io)
+        stream.synchronize()             # the host reads the step's result before the next step
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    e2e_ok = int(io_t["status_h"][0]) == 0
+
+    if dist is not None:
+        t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device=f"cuda:{local}")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, e2e_ms = float(t[0]), float(t[1])
+
+    peak, peak_kind = _peak_hbm()
+    achieved = nb["attention"] / (attn_ms * 1e-3) / 1e9
+    ms_step = ms / K
+    value = world * K / (ms * 1e-3)
+    flops = attention_flops(w)
+    out = {
+        "metric": "tree-verify steps/sec (HBM GB/s and fraction of ~8 TB/s alongside)",
+        "value": round(value, 3),
+        "unit": "steps/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) Q/K/V, N(0,2) logits with a planted +6 token, random pruned tree)",
+        "config": {"workload": _workload_desc(cfg), "batch": cfg.batch, "layers": cfg.layers,
+                   "context": cfg.ctx[0], "tree_nodes": w.n_total, "vocab": cfg.vocab, "k": cfg.k,
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "l2": "inputs larger than L2 (%.2f GB read per step vs 129 MB L2)" % (nb["roofline"] / 1e9)},
+        "step_roofline_bytes": nb["roofline"],
+        "hbm_gbs": round(nb["roofline"] / (ms_step * 1e-3) / 1e9, 1),
+        "hbm_frac_of_8tbs": round(nb["roofline"] / (ms_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4),
+        "hbm_frac_of_measured": round(nb["roofline"] / (ms_step * 1e-3) / 1e9 / peak, 4),
+        "roofline": {"bound": "hbm", "kernel": "tree_attn_tc_kernel", "achieved": round(achieved, 1),
+                     "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "traffic": None, "bytes_per_launch": nb["attention"],
+                     "avg_launch_ms": round(attn_ms, 5),
+                     "tensor_tflops": round(flops / (attn_ms * 1e-3) / 1e12, 1)},
+        "clocks": clocks,
+        "e2e": {"value": round(world * Ke / (e2e_ms * 1e-3), 3), "unit": "steps/s", "steps": Ke,
+                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "status_ok": e2e_ok},
+        "gpu_launches": int(launches),
+        "status": ptd.status_string(status),
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
+    return out
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+_SAMPLE_CODE = r"""
+import json, sys, time
+sys.path.insert(0, {root!r})
+import numpy as np
+import oracle
+from paper_2607_10661_gb300 import synthetic as syn
+cfg = syn.CONFIGS[{workload!r}]
+w = syn.Workload(cfg, 1000)
+G, C, L, H = cfg.hq // cfg.hkv, int(w.ctx_lens[0]), cfg.layers, cfg.hkv
+lg = syn.widen(w.logits, "bf16")
+cache = {{}}
+def layer(l):
+    if l not in cache:
+        cache.clear()
+        kl, vl = w.kv_layer(l)
+        cache[l] = (syn.widen(w.q_layer(l), "bf16"), w.seq_view(syn.widen(kl, "bf16"), 0),
+                    w.seq_view(syn.widen(vl, "bf16"), 0))
+    return cache[l]
+per_step = []
+deadline = time.time() + {budget}
+for i in range({warmup} + {steps}):
+    u = i % (L * H)
+    q, k, v = layer(u // H)
+    h = u % H
+    t0 = time.time()
+    oracle.tree_attention(q[:, h * G:(h + 1) * G], k[:, h:h + 1], v[:, h:h + 1], w.trees[0], C)
+    t1 = time.time()
+    idx, _ = oracle.topk(lg[i % w.n_total], cfg.k)
+    t2 = time.time()
+    target = np.full(w.n_total, int(idx[0]), np.int64)
+    path, n, bonus = oracle.verify_greedy(w.trees[0], w.tokens, target)
+    t3 = time.time()
+    oracle.kv_compact(k if i % 2 == 0 else v, path, C)
+    t4 = time.time()
+    if i >= {warmup}:
+        per_step.append((t1 - t0) * L * H + (t2 - t1) * w.n_total + (t3 - t2) + (t4 - t3) * 2 * L)
+    if time.time() > deadline and len(per_step) > 0:
+        break
+print(json.dumps(dict(per_step=per_step)))
+"""
+
+SAMPLE_DESC = ("per sample: one of the 256 (layer, KV head) attention units, one of the 63 top-k rows, the "
+               "whole verification and compaction of one of the 64 layer K/V tensors, timed single-threaded "
+               "(BLAS pinned to one thread) and scaled by those counts to one full step")
+
+
+def oracle_samples(steps: int, warmup: int, budget_s: float):
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    code = _SAMPLE_CODE.format(root=ROOT, workload=WORKLOAD, budget=float(budget_s), steps=int(steps),
+                               warmup=int(warmup))
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
+                       timeout=budget_s * 4 + 300)
+    if r.returncode != 0:
+        raise RuntimeError(r.stderr[-500:])
+    return json.loads(r.stdout.strip().splitlines()[-1])["per_step"]
+
+
+def cpu_baseline(budget_s: float) -> dict:
+    """The oracle as it stands on a bounded sample of the workload (about budget_s of CPU)."""
+    try:
+        per = oracle_samples(10000, 1, budget_s)
+    except Exception as e:  # reported, never fatal for the GPU line
+        return {"value": None, "unit": "steps/s", "cores": 1, "kind": "oracle", "error": str(e)[-300:]}
+    sec = float(np.mean(per))
+    return {"value": 1.0 / sec, "unit": "steps/s", "cores": 1, "kind": "oracle",
+            "sample": f"{len(per)} samples; " + SAMPLE_DESC, "seconds_per_step": sec}
+
+
+def run_reference(args):
+    """--impl reference: the CPU oracle on the host cores, one bounded sample per step; the
+    run stops early (reporting the steps it timed) once about 150 s of samples are taken."""
+    from paper_2607_10661_gb300 import synthetic as syn
+
+    cfg = syn.CONFIGS[WORKLOAD]
+    try:
+        per = oracle_samples(args.steps, min(args.warmup, 1), 150.0)
+    except Exception as e:
+        return {"impl": "reference", "unavailable": "oracle sample failed: " + str(e)[-200:]}
+    sec = float(np.mean(per))
+    value = 1.0 / sec
+    return {
+        "impl": "reference",
+        "metric": "tree-verify steps/sec (HBM GB/s and fraction of ~8 TB/s alongside)",
+        "value": value, "unit": "steps/s", "n_gpus": args.gpus, "steps": len(per), "warmup": min(args.warmup, 1),
+        "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic", "config": {"workload": _workload_desc(cfg)},
+        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{len(per)} samples; " + SAMPLE_DESC},
+        "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ptd", choices=["ptd", "reference"])
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling captures)")
+    ap.add_argument("--cpu-seconds", type=float, default=20.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args)), flush=True)
+        return
+    dist = None
+    if world > 1:
+        import torch.distributed as dist_mod
+
+        dist_mod.init_process_group("nccl")
+        dist = dist_mod
+    out = run_gpu(args, rank, world, dist)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -11,18 +11,21 @@
 // one (layer, tree, KV head) and a contiguous range of 128-key tiles (a KV split).  Each
 // K/V tile is loaded from HBM once by TMA and used by both M tiles.
 //
-// Warp roles (384 threads):
-//   warp 0      TMA producer: K, V tiles into a 3-slot ring (K_j, V_j, K_j+1, ...).
+// Warp roles (320 threads):
+//   warp 0      TMA producer: K, V tiles into a 5-slot ring (K_j, V_j, K_j+1, ...).
 //   warp 1      TMEM allocator and MMA issuer (one thread issues tcgen05.mma):
-//                 S_t = Q_t K_j^T    (SS: Q and K in shared memory, fp32 in TMEM)
-//                 O_t += P_t V_j     (SS: P written to shared memory by the softmax warps)
+//                 S_t = Q_t K_j^T    (Q and K from shared memory, fp32 S in TMEM)
+//                 O_t += P_t V_j     (P from TMEM, where the softmax wrote it over S_t;
+//                                     V from shared memory)
 //               in the order S_0, S_1 | PV_0, S_0', PV_1, S_1' | ... so the softmax of one
 //               M tile overlaps the tensor work of the other.
-//   warps 4-7   softmax of M tile 0 (thread = row = TMEM lane), warps 8-11 of M tile 1:
-//               masked row max, lazy rescaling of O (only when the running max grows by
-//               more than 2^8), exp2, P to shared memory in the 128-byte swizzled K-major
-//               layout the MMA reads, row sum; at the end O / l (or a split partial).
-// TMEM: S_0 | S_1 | O_0 | O_1, 128 fp32 columns each = all 512 columns of the SM.
+//   warps 2-5   softmax of M tile 0, warps 6-9 of M tile 1 (thread = row = TMEM lane
+//               (warp % 4) * 32 + lane): row max, lazy rescaling of O (only when the
+//               running max grows by more than 2^8), exp2, bf16 P back into TMEM, row sum;
+//               at the end O / l (or a split partial).  Tiles that lie entirely inside the
+//               committed prefix skip the mask arithmetic.
+// TMEM: S_0 | S_1 | O_0 | O_1, 128 fp32 columns each = all 512 columns of the SM; P_t
+// takes the first 64 columns of S_t (two bf16 per column).
 // The ancestor mask of a row's node (up to 128 bits) lives in 4 registers of its thread.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -36,13 +39,13 @@
 namespace ptd {
 namespace tc {
 
-constexpr int kThreads = 384;
-constexpr int kSlots = 3;
+constexpr int kThreads = 320;
+constexpr int kSlots = 5;
 constexpr uint32_t kTileBytes = 32768;   // 128 rows x 128 bf16
 constexpr uint32_t kHalfBytes = 16384;   // 128 rows x 64 bf16 (one 128-byte swizzle column)
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffP = 2 * kTileBytes;
-constexpr uint32_t kOffRing = 4 * kTileBytes;
+constexpr uint32_t kOffRing = 2 * kTileBytes;
+constexpr uint32_t kOffScratch = kOffRing + (kSlots - 1) * kTileBytes;   // setup only
 constexpr uint32_t kOffBar = kOffRing + kSlots * kTileBytes;
 constexpr uint32_t kNumBars = 2 * kSlots + 7;
 constexpr uint32_t kOffTmemPtr = kOffBar + kNumBars * 8;
@@ -150,9 +153,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
   }
 
-  // ---- tree: validate and build ancestor masks (scratch in the P region)
-  int* par_s = reinterpret_cast<int*>(smem + kOffP);
-  uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + kOffP + 512);
+  // ---- tree: validate and build ancestor masks (scratch in the last ring slot)
+  int* par_s = reinterpret_cast<int*>(smem + kOffScratch);
+  uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + kOffScratch + 512);
   bool bad = false;
   if (threadIdx.x < T) {
     const int pp = p.parents[node0 + threadIdx.x];
@@ -178,9 +181,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
 
   // ---- softmax-thread identity, ancestor mask and Q row
-  const bool is_sm = warp >= 4;
-  const int t = is_sm ? (warp - 4) >> 2 : 0;
-  const int row = ((warp - 4) & 3) * 32 + lane;
+  const bool is_sm = warp >= 2;
+  const int t = is_sm ? (warp - 2) >> 2 : 0;
+  const int row = (warp & 3) * 32 + lane;   // = TMEM lane this warp may access
   const int grow = (2 * mp + t) * 128 + row;
   const int node = grow / G;
   const int g = grow - node * G;
@@ -195,8 +198,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   const size_t qo_row = row_valid ? ((((size_t)lq * p.n_total + node0 + node) * p.hq + (size_t)hkv * G + g) * 128)
                                   : 0;
-  __syncthreads();   // scratch reads done before Q / P writes
-
   if (active_t && !invalid) {
     const uint32_t qrow = base + kOffQ + (uint32_t)t * kTileBytes + (uint32_t)row * 128u;
     const uint4* src = reinterpret_cast<const uint4*>(p.q) + qo_row / 8;
@@ -209,7 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   fence_proxy_async_smem();
-  __syncthreads();
+  __syncthreads();   // Q visible to the tensor core; the scratch slot is free again
   tc_fence_after();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffTmemPtr);
 
@@ -271,17 +272,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // drain the copies already issued (bounded) before the CTA can exit
         for (int back = 1; back <= kSlots && it - back >= 0; ++back) {
           const int i2 = it - back;
-          const unsigned long long t_start = globaltimer_ns();
-          while (!mbar_try_wait(full_bar(i2 % kSlots), (uint32_t)((i2 / kSlots) & 1)) &&
-                 globaltimer_ns() - t_start < 100000000ull) {
-          }
+          mbar_drain(full_bar(i2 % kSlots), (uint32_t)((i2 / kSlots) & 1), 100000000ull);
         }
       }
     }
   } else if (warp == 1) {
     // ================================================================ MMA issuer
     if (n_local > 0) {
-      const uint32_t q_base = base + kOffQ, p_base = base + kOffP, ring = base + kOffRing;
+      const uint32_t q_base = base + kOffQ, ring = base + kOffRing;
       auto issue_s = [&](int tt, int slot) {
         const uint32_t d = tmem + (uint32_t)tt * 128u;
 #pragma unroll
@@ -294,13 +292,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       auto issue_pv = [&](int tt, int slot, bool acc) {
         const uint32_t d = tmem + 256u + (uint32_t)tt * 128u;
+        const uint32_t a = tmem + (uint32_t)tt * 128u;   // P: 16 keys = 8 packed columns per step
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t koff = (uint32_t)(kk >> 2) * kHalfBytes + (uint32_t)(kk & 3) * 32u;
-          const uint64_t a = smem_desc_sw128(p_base + (uint32_t)tt * kTileBytes + koff, 16, 1024);
           const uint64_t bd = smem_desc_sw128(ring + (uint32_t)slot * kTileBytes + (uint32_t)kk * 2048u,
                                               kHalfBytes, 1024);
-          mma_bf16_ss(d, a, bd, kIdescPV, (acc || kk > 0) ? 1u : 0u);
+          mma_bf16_ts(d, a + (uint32_t)kk * 8u, bd, kIdescPV, (acc || kk > 0) ? 1u : 0u);
         }
       };
       bool ok = true;
@@ -382,67 +379,85 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     const uint32_t tS = tmem + lane_base + (uint32_t)t * 128u;
     const uint32_t tO = tmem + lane_base + 256u + (uint32_t)t * 128u;
-    const uint32_t prow = base + kOffP + (uint32_t)t * kTileBytes + (uint32_t)row * 128u;
+    const unsigned long long sl2x2 = f2_pack(sl2, sl2);
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     uint32_t r[32];
+    uint32_t sv[128];   // the thread's whole S row: one TMEM wait per tile
     for (int jj = 0; jj < n_local; ++jj) {
       if (!(ok = mbar_wait_warp(sfull_bar(t), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
       tc_fence_after();
+      tmem_ld32(tS + 0u, *reinterpret_cast<uint32_t(*)[32]>(sv + 0));
+      tmem_ld32(tS + 32u, *reinterpret_cast<uint32_t(*)[32]>(sv + 32));
+      tmem_ld32(tS + 64u, *reinterpret_cast<uint32_t(*)[32]>(sv + 64));
+      tmem_ld32(tS + 96u, *reinterpret_cast<uint32_t(*)[32]>(sv + 96));
+      tmem_ld_wait();
       const int t0 = (kt_begin + jj) * 128;
-      const bool need_mask = t0 + 128 > C;
-      float mx = -INFINITY;
+      const bool need_mask = t0 + 128 > C;   // warp-uniform
+      if (need_mask) {
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        tmem_ld32(tS + (uint32_t)c * 32u, r);
-        tmem_ld_wait();
-        const uint32_t vw = need_mask ? vis_word(t0 + c * 32 - C, am0, am1, am2, am3) : 0xFFFFFFFFu;
+        for (int c = 0; c < 4; ++c) {
+          const uint32_t vw = vis_word(t0 + c * 32 - C, am0, am1, am2, am3);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const float s = ((vw >> e) & 1u) ? __uint_as_float(r[e]) : -INFINITY;
-          mx = fmaxf(mx, s);
+          for (int e = 0; e < 32; ++e)
+            sv[c * 32 + e] = ((vw >> e) & 1u) ? sv[c * 32 + e] : __float_as_uint(-INFINITY);
         }
+      }
+      // row max of the visible scores (masked entries are -inf)
+      float mx;
+      {
+        float a0 = -INFINITY, a1 = -INFINITY, a2 = -INFINITY, a3 = -INFINITY;
+#pragma unroll
+        for (int e = 0; e < 128; e += 8) {
+          a0 = fmax3(a0, __uint_as_float(sv[e + 0]), __uint_as_float(sv[e + 1]));
+          a1 = fmax3(a1, __uint_as_float(sv[e + 2]), __uint_as_float(sv[e + 3]));
+          a2 = fmax3(a2, __uint_as_float(sv[e + 4]), __uint_as_float(sv[e + 5]));
+          a3 = fmax3(a3, __uint_as_float(sv[e + 6]), __uint_as_float(sv[e + 7]));
+        }
+        mx = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3));
       }
       const float m_tile = mx * sl2;
-      if (m_tile > m_run + kRescaleLog2) {
-        if (jj > 0) {
-          const float alpha = ptx_exp2(m_run - m_tile);
-          l_run *= alpha;
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            tmem_ld32(tO + (uint32_t)c * 32u, r);
-            tmem_ld_wait();
-#pragma unroll
-            for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-            tmem_st32(tO + (uint32_t)c * 32u, r);
-          }
-          tmem_st_wait();
-        }
-        m_run = m_tile;
-      }
+      // lazy rescaling: move the reference max only when it grows by more than 2^8
+      const bool rescale = m_tile > m_run + kRescaleLog2;
+      const float alpha = (rescale && jj > 0) ? ptx_exp2(m_run - m_tile) : 1.f;
+      if (rescale) m_run = m_tile;
       const float m_use = m_run == -INFINITY ? 0.f : m_run;
+      const unsigned long long negm = f2_pack(-m_use, -m_use);
+      // P = 2^(s * scale * log2e - m) (masked: 2^-inf = 0), bf16 into the first 64 columns of S_t
+      unsigned long long sum = f2_pack(0.f, 0.f);
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        tmem_ld32(tS + (uint32_t)c * 32u, r);
-        tmem_ld_wait();
-        const uint32_t vw = need_mask ? vis_word(t0 + c * 32 - C, am0, am1, am2, am3) : 0xFFFFFFFFu;
-        uint32_t pk[16];
+      for (int c = 0; c < 8; ++c) {
+        uint32_t pk[8];
 #pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          const float p0 = ((vw >> e) & 1u) ? ptx_exp2(fmaf(__uint_as_float(r[e]), sl2, -m_use)) : 0.f;
-          const float p1 = ((vw >> (e + 1)) & 1u) ? ptx_exp2(fmaf(__uint_as_float(r[e + 1]), sl2, -m_use)) : 0.f;
-          l_run += p0 + p1;
+        for (int e = 0; e < 16; e += 2) {
+          const unsigned long long x = f2_fma(
+              f2_pack(__uint_as_float(sv[c * 16 + e]), __uint_as_float(sv[c * 16 + e + 1])), sl2x2, negm);
+          float x0, x1;
+          f2_unpack(x, x0, x1);
+          const float p0 = ptx_exp2(x0), p1 = ptx_exp2(x1);
+          sum = f2_add(sum, f2_pack(p0, p1));
           pk[e >> 1] = pack_bf16x2(p0, p1);
         }
+        tmem_st8(tS + (uint32_t)c * 8u, pk);
+      }
+      {
+        float s0, s1;
+        f2_unpack(sum, s0, s1);
+        l_run = l_run * alpha + (s0 + s1);
+      }
+      if (rescale && jj > 0) {
+        // O_t is idle here: PV_t of the previous tile completed before S_t of this one
+#pragma unroll 1
+        for (int c = 0; c < 8; ++c) {
+          uint32_t o16[16];
+          tmem_ld16(tO + (uint32_t)c * 16u, o16);
+          tmem_ld_wait();
 #pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          const int cc = c * 4 + q4;            // 16-byte chunk 0..15 of the row
-          const int half = cc >> 3, j = cc & 7;
-          st_shared_v4(prow + (uint32_t)half * kHalfBytes + (uint32_t)((j ^ (row & 7)) << 4), pk[q4 * 4 + 0],
-                       pk[q4 * 4 + 1], pk[q4 * 4 + 2], pk[q4 * 4 + 3]);
+          for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
+          tmem_st16(tO + (uint32_t)c * 16u, o16);
         }
       }
-      fence_proxy_async_smem();
+      tmem_st_wait();
       tc_fence_before();
       mbar_arrive(pfull_bar(t));
     }
