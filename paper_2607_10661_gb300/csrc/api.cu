@@ -253,7 +253,7 @@ ptd_status ptd_topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int
   if (dtype != PTD_BF16 && dtype != PTD_F32) return PTD_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(logits) % dtype_size(dtype)) != 0) return PTD_ERR_INVALID_ARG;
   const ptd_status st = cuda_status(ptd::launch_topk(logits, dtype == PTD_BF16, rows, vocab, row_stride, k, out_idx,
-                                                     out_val, static_cast<cudaStream_t>(stream)));
+                                                     out_val, nullptr, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }

@@ -81,6 +81,23 @@ struct ThreadList {
       }
     }
   }
+  // Insert a full key (any index order): larger key first, ties impossible (distinct indices).
+  __device__ __forceinline__ void push_key(uint64_t key) {
+    const uint32_t o = (uint32_t)(key >> 32), i = ~(uint32_t)key;
+    if (key <= make_key(ord[KM - 1], idx[KM - 1])) return;
+    ord[KM - 1] = o;
+    idx[KM - 1] = i;
+#pragma unroll
+    for (int s = KM - 1; s > 0; --s) {
+      if (make_key(ord[s], idx[s]) > make_key(ord[s - 1], idx[s - 1])) {
+        const uint32_t to = ord[s], ti = idx[s];
+        ord[s] = ord[s - 1];
+        idx[s] = idx[s - 1];
+        ord[s - 1] = to;
+        idx[s - 1] = ti;
+      }
+    }
+  }
   __device__ __forceinline__ uint64_t head() const { return make_key(ord[0], idx[0]); }
   __device__ __forceinline__ void pop() {
 #pragma unroll
@@ -215,14 +232,214 @@ __global__ void __launch_bounds__(kThreads) topk_cluster_kernel(const T* __restr
   }
 }
 
-template <int KM, typename T>
+// ------------------------------------------------------------------ bf16 fast path
+// Each CTA stages its contiguous slice of the row (up to kSliceVec 16-byte vectors) into
+// shared memory with bulk asynchronous copies, so the row is read from HBM exactly once,
+// then makes three passes over shared memory:
+//   1. every thread's maximum;
+//   2. T = the k-th largest thread maximum.  The k threads holding those maxima own k
+//      distinct elements >= T, so every element of the CTA's top-k is >= T;
+//   3. elements >= T become candidates (exact 64-bit keys); the CTA's top-k is selected
+//      among them.
+// A slice with more than kCandCap candidates (many ties at the threshold, e.g. a constant
+// row) is selected exactly with per-thread sorted lists instead.
+constexpr int kSliceVec = 4096;            // 64 KB of bf16 logits per CTA
+constexpr int kCandCap = 1024;
+constexpr uint32_t kChunkBytes = 16384;    // bytes per bulk copy
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// k rounds of "largest key wins" over one key per lane; lane s < k ends with the s-th largest.
+__device__ __forceinline__ uint64_t warp_topk_of_one(uint64_t key, int k, int lane) {
+  uint64_t mine = key, out = 0ull;
+  for (int s = 0; s < k; ++s) {
+    const uint64_t best = warp_max_u64(mine);
+    if (mine == best) mine = 0ull;
+    if (lane == s) out = best;
+  }
+  return out;
+}
+
+template <int KM>
+__global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16* __restrict__ logits,
+                                                             int64_t rows, int vocab, int64_t row_stride, int k,
+                                                             int32_t* __restrict__ out_idx,
+                                                             float* __restrict__ out_val, int32_t* dev_status) {
+  extern __shared__ __align__(128) uint4 slice[];
+  __shared__ uint64_t warp_keys[kWarps][KM];
+  __shared__ uint64_t cta_keys[KM];
+  __shared__ uint64_t cand[kCandCap];
+  __shared__ int ncand;
+  __shared__ float thr_s;
+  __shared__ __align__(8) uint64_t bar_s;
+  __shared__ int abort_s;
+
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = (int)cluster.block_rank();
+  const int csize = (int)cluster.num_blocks();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tid = threadIdx.x;
+  const uint32_t bar = smem_u32(&bar_s);
+  if (tid == 0) {
+    mbar_init(bar, 1);
+    abort_s = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  uint32_t phase = 0;
+
+  for (int64_t r = blockIdx.y; r < rows; r += gridDim.y, phase ^= 1u) {
+    const __nv_bfloat16* row = logits + r * row_stride;
+    const uintptr_t addr = reinterpret_cast<uintptr_t>(row);
+    int a0 = (int)(((16 - (addr & 15)) & 15) / 2);
+    if (a0 > vocab) a0 = vocab;
+    const int nvec = (vocab - a0) / 8;
+    const int a1 = a0 + nvec * 8;
+    const int per = (nvec + csize - 1) / csize;
+    const int v_begin = min(nvec, rank * per), v_end = min(nvec, v_begin + per);
+    const int nv = v_end - v_begin;
+    const uint4* vrow = reinterpret_cast<const uint4*>(row + a0) + v_begin;
+    const bool own_head = rank == 0 && tid == 0;
+    const bool own_tail = rank == csize - 1 && tid == kThreads - 1;
+
+    if (tid == 0) {
+      fence_proxy_async_smem();   // the previous row's reads of the slice precede this copy
+      const uint32_t total = (uint32_t)nv * 16u;
+      mbar_arrive_expect_tx(bar, total);
+      for (uint32_t off = 0; off < total; off += kChunkBytes) {
+        const uint32_t n = total - off < kChunkBytes ? total - off : kChunkBytes;
+        bulk_load(smem_u32(slice) + off, reinterpret_cast<const uint8_t*>(vrow) + off, n, bar);
+      }
+    }
+    // head / tail scalars while the copy is in flight
+    float tmax = -INFINITY;
+    if (own_head)
+      for (int i = 0; i < a0; ++i) tmax = fmaxf(tmax, Vec<__nv_bfloat16>::scalar(row + i));
+    if (own_tail)
+      for (int i = a1; i < vocab; ++i) tmax = fmaxf(tmax, Vec<__nv_bfloat16>::scalar(row + i));
+    mbar_wait(bar, phase, &abort_s, dev_status);   // bounded: a lost copy only flags PTD_ERR_TIMEOUT
+
+    // pass 1: thread maximum
+    for (int v = tid; v < nv; v += kThreads) {
+      const uint4 x = slice[v];
+      tmax = fmax3(tmax, bf16_lo(x.x), bf16_hi(x.x));
+      tmax = fmax3(tmax, bf16_lo(x.y), bf16_hi(x.y));
+      tmax = fmax3(tmax, bf16_lo(x.z), bf16_hi(x.z));
+      tmax = fmax3(tmax, bf16_lo(x.w), bf16_hi(x.w));
+    }
+    const bool has_elems = tid < nv || (own_head && a0 > 0) || (own_tail && a1 < vocab);
+
+    // pass 2: T = k-th largest thread maximum (over threads that own elements)
+    {
+      const uint64_t key = has_elems ? make_key(ordered_bits(tmax), (uint32_t)tid) : 0ull;
+      const uint64_t wk = warp_topk_of_one(key, k, lane);
+      if (lane < k) warp_keys[warp][lane] = wk;
+      if (tid == 0) ncand = 0;
+      __syncthreads();
+      if (warp == 0) {
+        int cur = 0;
+        uint64_t kth = 0ull;
+        for (int s = 0; s < k; ++s) {
+          const uint64_t mine = (lane < kWarps && cur < k) ? warp_keys[lane][cur] : 0ull;
+          const uint64_t best = warp_max_u64(mine);
+          if (lane < kWarps && mine == best && best != 0ull) ++cur;
+          kth = best;
+        }
+        if (lane == 0) thr_s = kth != 0ull ? from_ordered((uint32_t)(kth >> 32)) : -INFINITY;
+      }
+      __syncthreads();
+    }
+    const float thr = thr_s;
+
+    // pass 3: candidates >= T
+    auto offer = [&](float f, uint32_t gidx) {
+      if (f >= thr) {
+        const int pos = atomicAdd(&ncand, 1);
+        if (pos < kCandCap) cand[pos] = make_key(ordered_bits(f), gidx);
+      }
+    };
+    for (int v = tid; v < nv; v += kThreads) {
+      const uint4 x = slice[v];
+      float vm = fmax3(bf16_lo(x.x), bf16_hi(x.x), bf16_lo(x.y));
+      vm = fmax3(vm, bf16_hi(x.y), bf16_lo(x.z));
+      vm = fmax3(vm, bf16_hi(x.z), bf16_lo(x.w));
+      vm = fmaxf(vm, bf16_hi(x.w));
+      if (vm >= thr) {
+        const uint32_t gi = (uint32_t)(a0 + (v_begin + v) * 8);
+        const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          offer(bf16_lo(w[q]), gi + 2 * q);
+          offer(bf16_hi(w[q]), gi + 2 * q + 1);
+        }
+      }
+    }
+    if (own_head)
+      for (int i = 0; i < a0; ++i) offer(Vec<__nv_bfloat16>::scalar(row + i), (uint32_t)i);
+    if (own_tail)
+      for (int i = a1; i < vocab; ++i) offer(Vec<__nv_bfloat16>::scalar(row + i), (uint32_t)i);
+    __syncthreads();
+    const int nc = ncand;
+
+    // CTA top-k: from the candidates, or exactly from every element on overflow
+    ThreadList<KM> list;
+    list.init();
+    if (nc <= kCandCap) {
+      for (int i = tid; i < nc; i += kThreads) list.push_key(cand[i]);
+    } else {
+      if (own_head)
+        for (int i = 0; i < a0; ++i) list.push(ordered_bits(Vec<__nv_bfloat16>::scalar(row + i)), (uint32_t)i);
+      for (int v = tid; v < nv; v += kThreads) {
+        float f[8];
+        Vec<__nv_bfloat16>::unpack(slice[v], f);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) list.push(ordered_bits(f[e]), (uint32_t)(a0 + (v_begin + v) * 8 + e));
+      }
+      if (own_tail)
+        for (int i = a1; i < vocab; ++i) list.push(ordered_bits(Vec<__nv_bfloat16>::scalar(row + i)), (uint32_t)i);
+    }
+    for (int s = 0; s < k; ++s) {
+      const uint64_t mine = list.head();
+      const uint64_t best = warp_max_u64(mine);
+      if (mine == best) list.pop();
+      if (lane == 0) warp_keys[warp][s] = best;
+    }
+    __syncthreads();   // also: every thread is done reading the slice
+    if (warp == 0) {
+      int cur = 0;
+      for (int s = 0; s < k; ++s) {
+        const uint64_t mine = (lane < kWarps && cur < k) ? warp_keys[lane][cur] : 0ull;
+        const uint64_t best = warp_max_u64(mine);
+        if (lane < kWarps && mine == best && best != 0ull) ++cur;
+        if (lane == 0) cta_keys[s] = best;
+      }
+    }
+    cluster.sync();
+    if (rank == 0 && warp == 0) {
+      const uint64_t* remote = lane < csize ? cluster.map_shared_rank(cta_keys, lane) : nullptr;
+      int cur = 0;
+      for (int s = 0; s < k; ++s) {
+        const uint64_t mine = (lane < csize && cur < k) ? remote[cur] : 0ull;
+        const uint64_t best = warp_max_u64(mine);
+        if (lane < csize && mine == best && best != 0ull) ++cur;
+        if (lane == 0) {
+          out_idx[r * k + s] = (int32_t)(~(uint32_t)(best & 0xFFFFFFFFull));
+          out_val[r * k + s] = from_ordered((uint32_t)(best >> 32));
+        }
+      }
+    }
+    cluster.sync();
+  }
+}
+
+template <int KM, typename T, bool kFast>
 cudaError_t launch_km(const T* logits, int64_t rows, int vocab, int64_t row_stride, int k, int32_t* out_idx,
-                      float* out_val, int cluster, cudaStream_t stream) {
+                      float* out_val, int cluster, int32_t* dev_status, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   const int64_t gy = rows < 65535 ? rows : 65535;
   cfg.gridDim = dim3((unsigned)cluster, (unsigned)gy, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -231,32 +448,58 @@ cudaError_t launch_km(const T* logits, int64_t rows, int vocab, int64_t row_stri
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, topk_cluster_kernel<KM, T>, logits, rows, vocab, row_stride, k, out_idx,
-                            out_val);
+  if constexpr (kFast) {
+    const int nvec = vocab / 8 + 1;
+    const int per = (nvec + cluster - 1) / cluster;
+    cfg.dynamicSmemBytes = (size_t)per * 16;
+    cudaError_t e = cudaFuncSetAttribute(topk_bf16_kernel<KM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSliceVec * 16);
+    if (e != cudaSuccess) return e;
+    return cudaLaunchKernelEx(&cfg, topk_bf16_kernel<KM>, logits, rows, vocab, row_stride, k, out_idx, out_val,
+                              dev_status);
+  } else {
+    cfg.dynamicSmemBytes = 0;
+    return cudaLaunchKernelEx(&cfg, topk_cluster_kernel<KM, T>, logits, rows, vocab, row_stride, k, out_idx,
+                              out_val);
+  }
 }
 
-template <typename T>
+template <typename T, bool kFast>
 cudaError_t launch_t(const T* logits, int64_t rows, int vocab, int64_t row_stride, int k, int32_t* out_idx,
-                     float* out_val, cudaStream_t stream) {
-  // enough CTAs per row to keep HBM busy, at most one portable cluster (8 CTAs)
-  const int per_cta = (int)(16384 / sizeof(T)) * 2;   // ~32 KB of logits per CTA
-  int cluster = (vocab + per_cta - 1) / per_cta;
+                     float* out_val, int32_t* dev_status, cudaStream_t stream) {
+  int cluster;
+  if (kFast) {
+    const int nvec = vocab / 8 + 1;
+    cluster = (nvec + kSliceVec - 1) / kSliceVec;   // slices of at most 64 KB
+  } else {
+    const int per_cta = (int)(16384 / sizeof(T)) * 2;   // ~32 KB of logits per CTA
+    cluster = (vocab + per_cta - 1) / per_cta;
+  }
   cluster = cluster < 1 ? 1 : (cluster > kMaxCluster ? kMaxCluster : cluster);
-  if (k <= 1) return launch_km<1>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, stream);
-  if (k <= 2) return launch_km<2>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, stream);
-  if (k <= 4) return launch_km<4>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, stream);
-  if (k <= 8) return launch_km<8>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, stream);
-  return launch_km<16>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, stream);
+#define PTD_TOPK_LAUNCH(KMV) \
+  return launch_km<KMV, T, kFast>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, dev_status, stream)
+  if (k <= 1) PTD_TOPK_LAUNCH(1);
+  if (k <= 2) PTD_TOPK_LAUNCH(2);
+  if (k <= 4) PTD_TOPK_LAUNCH(4);
+  if (k <= 8) PTD_TOPK_LAUNCH(8);
+  PTD_TOPK_LAUNCH(16);
+#undef PTD_TOPK_LAUNCH
 }
 
 }  // namespace topk
 
 cudaError_t launch_topk(const void* logits, bool bf16, int64_t rows, int vocab, int64_t row_stride, int k,
-                        int32_t* out_idx, float* out_val, cudaStream_t stream) {
-  if (bf16)
-    return topk::launch_t(static_cast<const __nv_bfloat16*>(logits), rows, vocab, row_stride, k, out_idx,
-                          out_val, stream);
-  return topk::launch_t(static_cast<const float*>(logits), rows, vocab, row_stride, k, out_idx, out_val, stream);
+                        int32_t* out_idx, float* out_val, int32_t* dev_status, cudaStream_t stream) {
+  if (bf16) {
+    // the shared-memory path covers rows up to kMaxCluster slices of kSliceVec vectors
+    if ((int64_t)vocab / 8 + 1 <= (int64_t)topk::kMaxCluster * topk::kSliceVec)
+      return topk::launch_t<__nv_bfloat16, true>(static_cast<const __nv_bfloat16*>(logits), rows, vocab,
+                                                 row_stride, k, out_idx, out_val, dev_status, stream);
+    return topk::launch_t<__nv_bfloat16, false>(static_cast<const __nv_bfloat16*>(logits), rows, vocab, row_stride,
+                                                k, out_idx, out_val, dev_status, stream);
+  }
+  return topk::launch_t<float, false>(static_cast<const float*>(logits), rows, vocab, row_stride, k, out_idx,
+                                      out_val, dev_status, stream);
 }
 
 }  // namespace ptd

@@ -6,5 +6,5 @@
 
 namespace ptd {
 cudaError_t launch_topk(const void* logits, bool bf16, int64_t rows, int vocab, int64_t row_stride, int k,
-                        int32_t* out_idx, float* out_val, cudaStream_t stream);
+                        int32_t* out_idx, float* out_val, int32_t* dev_status, cudaStream_t stream);
 }  // namespace ptd
