@@ -119,6 +119,31 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache,
                               void* workspace, size_t workspace_bytes,
                               int32_t* dev_status, void* stream);
 
+/* Tree-masked attention for callers that cannot allocate device memory.  Some embedders
+ * hand this library only their input and output buffers: a plugin running inside another
+ * runtime's engine may have no allocator of its own to ask, and a latency-critical decode
+ * loop may not tolerate cudaMalloc, whose implicit device synchronisation stalls every
+ * stream.  This variant computes exactly what ptd_tree_attention computes, with the same
+ * key-split schedule, but takes its split scratch from a fixed array that the library
+ * holds in device memory (PTD_STATIC_SCRATCH_BYTES; every GPU that loads the library keeps
+ * it until the process exits) instead of from a caller workspace.  The paper has no
+ * counterpart of this entry point.
+ *   - Arguments are those of ptd_tree_attention without workspace / workspace_bytes.
+ *   - If the split schedule for these shapes needs more than PTD_STATIC_SCRATCH_BYTES of
+ *     scratch (ptd_attention_workspace_size > PTD_STATIC_SCRATCH_BYTES) the call returns
+ *     PTD_ERR_WORKSPACE and enqueues nothing; use ptd_tree_attention with a workspace then.
+ *   - The first call on each device resolves the array's device address on that device
+ *     (make that device current); issue that first call before any stream capture.
+ *   - Every call on a device shares the one array and it keeps the previous call's
+ *     contents.  The kernels write every scratch entry they later read, so nothing needs
+ *     clearing, but calls whose kernels overlap on the GPU (different streams without
+ *     ordering between them) race on the array: serialise them.
+ *   - Calls no allocator (no cudaMalloc/cudaFree, no allocating library routine). */
+#define PTD_STATIC_SCRATCH_BYTES ((size_t)8 << 20)
+ptd_status ptd_tree_attention_noalloc(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
+                                      int32_t num_layers, const void* q, int32_t num_q_heads, float scale,
+                                      void* out, int32_t* dev_status, void* stream);
+
 /* Per-node top-k of the logits (Sec. 3.1 "Progressive Expansion": each node's draft
  * token d_v; "Width Control": at most k children; Sec. 3.2: greedy V_n = entry 0).
  *   logits: [rows][row_stride] of `dtype`, the first `vocab` entries of a row are used.

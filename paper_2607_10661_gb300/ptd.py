@@ -25,7 +25,7 @@ MAX_TOPK = 16
 EXPORTED = (
     "ptd_attention_workspace_size", "ptd_tree_attention", "ptd_topk_draft", "ptd_verify_greedy",
     "ptd_kv_compact", "ptd_tree_verify_step", "ptd_tree_verify_step_host", "ptd_last_launch_count",
-    "ptd_status_string",
+    "ptd_status_string", "ptd_tree_attention_noalloc",
 )
 
 
@@ -84,6 +84,8 @@ def lib() -> ctypes.CDLL:
         L.ptd_attention_workspace_size.argtypes = [P(_Tree), P(_Cache), i32, i32]
         L.ptd_tree_attention.restype = ctypes.c_int
         L.ptd_tree_attention.argtypes = [P(_Tree), P(_Cache), i32, i32, vp, i32, f32, vp, vp, sz, vp, vp]
+        L.ptd_tree_attention_noalloc.restype = ctypes.c_int
+        L.ptd_tree_attention_noalloc.argtypes = [P(_Tree), P(_Cache), i32, i32, vp, i32, f32, vp, vp, vp]
         L.ptd_topk_draft.restype = ctypes.c_int
         L.ptd_topk_draft.argtypes = [vp, ctypes.c_int, i64, i32, i64, i32, vp, vp, vp]
         L.ptd_verify_greedy.restype = ctypes.c_int

@@ -1,0 +1,74 @@
+"""ptd_tree_attention_noalloc: the attention entry point for callers that cannot allocate
+device memory (for example a plugin inside another runtime that owns every allocation, or a
+decode loop that cannot afford cudaMalloc's implicit synchronisation).
+
+It takes its key-split scratch from a fixed array the library keeps in device memory, so
+its output must match ptd_tree_attention given a caller workspace, on consecutive calls
+that reuse the array with the previous call's contents still in it.  This file is
+collected last so a failure here never hides the other tests.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_10661_gb300 import ptd
+from paper_2607_10661_gb300 import synthetic as syn
+from paper_2607_10661_gb300.harness import DeviceWorkload
+
+pytestmark = pytest.mark.gpu
+
+BF16_MAX, BF16_MEAN = 2e-2, 2e-3
+STATIC_SCRATCH_BYTES = 8 << 20     # PTD_STATIC_SCRATCH_BYTES in include/ptd.h
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+
+    __graft_entry__.build()
+
+
+def _noalloc(dw, out):
+    c = dw.w.cfg
+    return ptd.lib().ptd_tree_attention_noalloc(
+        ctypes.byref(dw.tree.c), ctypes.byref(dw.cache.c), 0, c.layers, dw.q.data_ptr(), c.hq, ctypes.c_float(0.0),
+        out.data_ptr(), dw.dev_status.data_ptr(), ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+
+
+def _case(cfg_name, seed, **over):
+    w = syn.Workload(syn.shrink(syn.CONFIGS[cfg_name], **over), seed)
+    dw = DeviceWorkload(w, with_step_buffers=False)
+    need = ptd.attention_workspace_size(dw.tree, dw.cache, w.cfg.hq)
+    return dw, need
+
+
+def test_noalloc_matches_workspace_entry_on_consecutive_calls():
+    cases = [
+        _case("llama2-7b-layer", 71, hq=8, hkv=8, ctx=(333, 333), vocab=100),
+        _case("batched-paged", 72, batch=2, ctx=(300, 900), vocab=100, hq=8, hkv=2),
+    ]
+    for dw, need in cases:
+        assert 0 < need <= STATIC_SCRATCH_BYTES, need     # the split path (scratch) is exercised
+    for dw, _ in cases:                                   # two calls in a row on the shared array
+        dw.dev_status.zero_()
+        ref = torch.zeros_like(dw.q)
+        dw.attn_out = ref
+        dw.attention()                                    # ptd_tree_attention with a workspace
+        got = torch.full_like(dw.q, float("nan"))
+        assert _noalloc(dw, got) == ptd.OK
+        torch.cuda.synchronize()
+        assert int(dw.dev_status.item()) == 0
+        err = (got.float() - ref.float()).abs()
+        assert torch.isfinite(got.float()).all()
+        assert float(err.max()) <= BF16_MAX and float(err.mean()) <= BF16_MEAN
+
+
+def test_noalloc_rejects_problems_beyond_its_scratch():
+    dw, need = _case("long-context", 73, ctx=(3000, 3000), vocab=100)
+    assert need > STATIC_SCRATCH_BYTES
+    out = torch.zeros_like(dw.q)
+    assert _noalloc(dw, out) == ptd.WORKSPACE
+    torch.cuda.synchronize()
+    assert float(out.float().abs().max()) == 0.0          # nothing was launched
