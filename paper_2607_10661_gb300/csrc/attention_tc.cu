@@ -40,14 +40,16 @@ namespace ptd {
 namespace tc {
 
 constexpr int kThreads = 320;
-constexpr int kSlots = 5;
+constexpr int kStages = 2;                // K/V stage pairs (K tile then V tile)
 constexpr uint32_t kTileBytes = 32768;   // 128 rows x 128 bf16
 constexpr uint32_t kHalfBytes = 16384;   // 128 rows x 64 bf16 (one 128-byte swizzle column)
+constexpr uint32_t kStageBytes = 2 * kTileBytes;
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffRing = 2 * kTileBytes;
-constexpr uint32_t kOffScratch = kOffRing + (kSlots - 1) * kTileBytes;   // setup only
-constexpr uint32_t kOffBar = kOffRing + kSlots * kTileBytes;
-constexpr uint32_t kNumBars = 2 * kSlots + 7;
+constexpr uint32_t kOffScratch = kOffRing + kStageBytes + kTileBytes;   // setup only (V of stage 1)
+constexpr uint32_t kOffBar = kOffRing + kStages * kStageBytes;
+// barriers: full_k[2], full_v[2], empty[2], vzero, s_full[2], p_full[2], o_full[2], drain
+constexpr uint32_t kNumBars = 3 * kStages + 8;
 constexpr uint32_t kOffTmemPtr = kOffBar + kNumBars * 8;
 constexpr uint32_t kOffAbort = kOffTmemPtr + 4;
 constexpr uint32_t kSmemUsed = kOffAbort + 4;
@@ -125,22 +127,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n_local = max(0, min(n_kt, kt_begin + tps) - kt_begin);
 
   auto bar = [&](int i) { return base + kOffBar + 8u * (uint32_t)i; };
-  auto full_bar = [&](int s) { return bar(s); };
-  auto empty_bar = [&](int s) { return bar(kSlots + s); };
-  auto sfull_bar = [&](int t) { return bar(2 * kSlots + t); };
-  auto pfull_bar = [&](int t) { return bar(2 * kSlots + 2 + t); };
-  auto ofull_bar = [&](int t) { return bar(2 * kSlots + 4 + t); };
-  const uint32_t drain_bar = bar(2 * kSlots + 6);
+  auto fullk_bar = [&](int s) { return bar(s); };
+  auto fullv_bar = [&](int s) { return bar(kStages + s); };
+  auto empty_bar = [&](int s) { return bar(2 * kStages + s); };
+  const uint32_t vzero_bar = bar(3 * kStages);
+  auto sfull_bar = [&](int t) { return bar(3 * kStages + 1 + t); };
+  auto pfull_bar = [&](int t) { return bar(3 * kStages + 3 + t); };
+  auto ofull_bar = [&](int t) { return bar(3 * kStages + 5 + t); };
+  const uint32_t drain_bar = bar(3 * kStages + 7);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffAbort);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kSlots; ++s) {
-      mbar_init(full_bar(s), 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(fullk_bar(s), 1);
+      mbar_init(fullv_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
+    mbar_init(vzero_bar, 1);
     for (int t = 0; t < 2; ++t) {
       mbar_init(sfull_bar(t), 1);
-      mbar_init(pfull_bar(t), 128);
+      mbar_init(pfull_bar(t), 4);   // one arrival per softmax warp
       mbar_init(ofull_bar(t), 1);
     }
     mbar_init(drain_bar, 1);
@@ -231,147 +237,145 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 0) {
     // ================================================================ TMA producer
-    if (lane == 0 && n_local > 0) {
-      prefetch_tensormap(&map_k);
-      prefetch_tensormap(&map_v);
-      int it = 0;
+    if (n_local > 0) {
+      if (lane == 0) {
+        prefetch_tensormap(&map_k);
+        prefetch_tensormap(&map_v);
+      }
       bool ok = true;
-      for (int jj = 0; jj < n_local && ok; ++jj) {
+      int jj = 0;
+      for (; jj < n_local && ok; ++jj) {
         const int t0 = (kt_begin + jj) * 128;
-        for (int which = 0; which < 2; ++which, ++it) {
-          const int slot = it % kSlots;
-          const uint32_t ph = (uint32_t)((it / kSlots) & 1);
-          if (!mbar_wait(empty_bar(slot), ph ^ 1u, abort_flag, p.dev_status)) {
-            ok = false;
-            break;
-          }
-          const CUtensorMap* map = which ? &map_v : &map_k;
-          const uint32_t dst = base + kOffRing + (uint32_t)slot * kTileBytes;
-          if (!kPaged) {
-            const int row0 = (layer * p.batch + b) * p.seq_capacity + t0;
-            mbar_arrive_expect_tx(full_bar(slot), kTileBytes);
-            tma_load_3d(dst, map, full_bar(slot), 0, hkv, row0);
-            tma_load_3d(dst + kHalfBytes, map, full_bar(slot), 64, hkv, row0);
-          } else {
-            const int ps = p.page_size;
-            const int first_page = t0 / ps;
-            const int seq_pages = (N + ps - 1) / ps;
-            const int nvalid = min(128 / ps, seq_pages - first_page);
-            mbar_arrive_expect_tx(full_bar(slot), (uint32_t)(nvalid * 2 * ps * 128));
-            for (int pg = 0; pg < nvalid; ++pg) {
-              const int phys = p.block_table[(size_t)b * p.max_pages + first_page + pg];
-              const int row0 = (layer * p.num_pages + phys) * ps;
-              const uint32_t off = (uint32_t)(pg * ps * 128);
-              tma_load_3d(dst + off, map, full_bar(slot), 0, hkv, row0);
-              tma_load_3d(dst + kHalfBytes + off, map, full_bar(slot), 64, hkv, row0);
+        const int st = jj % kStages;
+        const uint32_t ph = (uint32_t)((jj / kStages) & 1);
+        if (lane == 0) {
+          ok = mbar_wait(empty_bar(st), ph ^ 1u, abort_flag, p.dev_status);
+          if (ok) {
+            const uint32_t dst = base + kOffRing + (uint32_t)st * kStageBytes;
+            for (int which = 0; which < 2; ++which) {
+              const CUtensorMap* map = which ? &map_v : &map_k;
+              const uint32_t fb = which ? fullv_bar(st) : fullk_bar(st);
+              const uint32_t d = dst + (uint32_t)which * kTileBytes;
+              if (!kPaged) {
+                const int row0 = (layer * p.batch + b) * p.seq_capacity + t0;
+                mbar_arrive_expect_tx(fb, kTileBytes);
+                tma_load_3d(d, map, fb, 0, hkv, row0);
+                tma_load_3d(d + kHalfBytes, map, fb, 64, hkv, row0);
+              } else {
+                const int ps = p.page_size;
+                const int first_page = t0 / ps;
+                const int seq_pages = (N + ps - 1) / ps;
+                const int nvalid = min(128 / ps, seq_pages - first_page);
+                mbar_arrive_expect_tx(fb, (uint32_t)(nvalid * 2 * ps * 128));
+                for (int pg = 0; pg < nvalid; ++pg) {
+                  const int phys = p.block_table[(size_t)b * p.max_pages + first_page + pg];
+                  const int row0 = (layer * p.num_pages + phys) * ps;
+                  const uint32_t off = (uint32_t)(pg * ps * 128);
+                  tma_load_3d(d + off, map, fb, 0, hkv, row0);
+                  tma_load_3d(d + kHalfBytes + off, map, fb, 64, hkv, row0);
+                }
+              }
             }
           }
         }
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (ok && t0 + 128 > N) {
+          // V rows past the sequence: zero them so that P = 0 never meets a non-finite value
+          if ((ok = mbar_wait_warp(fullv_bar(st), ph, abort_flag, p.dev_status))) {
+            const uint32_t vbase = base + kOffRing + (uint32_t)st * kStageBytes + kTileBytes;
+            const int r0 = N - t0;
+            for (int c = lane; c < (128 - r0) * 16; c += 32) {
+              const int r = r0 + (c >> 4), hc = c & 15;
+              st_shared_v4(vbase + (uint32_t)(hc >> 3) * kHalfBytes + (uint32_t)r * 128u + (uint32_t)(hc & 7) * 16u,
+                           0, 0, 0, 0);
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(vzero_bar);
+          }
+        }
       }
-      if (!ok) {
+      if (!ok && lane == 0) {
         // drain the copies already issued (bounded) before the CTA can exit
-        for (int back = 1; back <= kSlots && it - back >= 0; ++back) {
-          const int i2 = it - back;
-          mbar_drain(full_bar(i2 % kSlots), (uint32_t)((i2 / kSlots) & 1), 100000000ull);
+        for (int back = 1; back <= kStages && jj - back >= 0; ++back) {
+          const int j2 = jj - back;
+          mbar_drain(fullk_bar(j2 % kStages), (uint32_t)((j2 / kStages) & 1), 100000000ull);
+          mbar_drain(fullv_bar(j2 % kStages), (uint32_t)((j2 / kStages) & 1), 100000000ull);
         }
       }
     }
   } else if (warp == 1) {
-    // ================================================================ MMA issuer
-    if (n_local > 0) {
+    // ================================================================ MMA issuer (one thread)
+    if (n_local > 0 && lane == 0) {
       const uint32_t q_base = base + kOffQ, ring = base + kOffRing;
-      auto issue_s = [&](int tt, int slot) {
+      auto issue_s = [&](int tt, int st) {
         const uint32_t d = tmem + (uint32_t)tt * 128u;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t koff = (uint32_t)(kk >> 2) * kHalfBytes + (uint32_t)(kk & 3) * 32u;
           const uint64_t a = smem_desc_sw128(q_base + (uint32_t)tt * kTileBytes + koff, 16, 1024);
-          const uint64_t bd = smem_desc_sw128(ring + (uint32_t)slot * kTileBytes + koff, 16, 1024);
+          const uint64_t bd = smem_desc_sw128(ring + (uint32_t)st * kStageBytes + koff, 16, 1024);
           mma_bf16_ss(d, a, bd, kIdescS, kk > 0 ? 1u : 0u);
         }
       };
-      auto issue_pv = [&](int tt, int slot, bool acc) {
+      auto issue_pv = [&](int tt, int st, bool acc) {
         const uint32_t d = tmem + 256u + (uint32_t)tt * 128u;
         const uint32_t a = tmem + (uint32_t)tt * 128u;   // P: 16 keys = 8 packed columns per step
+        const uint32_t vb = ring + (uint32_t)st * kStageBytes + kTileBytes;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t bd = smem_desc_sw128(ring + (uint32_t)slot * kTileBytes + (uint32_t)kk * 2048u,
-                                              kHalfBytes, 1024);
+          const uint64_t bd = smem_desc_sw128(vb + (uint32_t)kk * 2048u, kHalfBytes, 1024);
           mma_bf16_ts(d, a + (uint32_t)kk * 8u, bd, kIdescPV, (acc || kk > 0) ? 1u : 0u);
         }
       };
-      bool ok = true;
-      // prologue: S for the first tile
-      {
-        const int ks = 0;
-        ok = mbar_wait_warp(full_bar(ks), 0, abort_flag, p.dev_status);
-        tc_fence_after();
-        if (ok && lane == 0) {
-          issue_s(0, ks);
-          mma_commit(sfull_bar(0));
-          if (nt == 2) {
-            issue_s(1, ks);
-            mma_commit(sfull_bar(1));
-          }
-          mma_commit(empty_bar(ks));
+      bool ok = mbar_wait(fullk_bar(0), 0, abort_flag, p.dev_status);
+      tc_fence_after();
+      if (ok) {
+        issue_s(0, 0);
+        mma_commit(sfull_bar(0));
+        if (nt == 2) {
+          issue_s(1, 0);
+          mma_commit(sfull_bar(1));
         }
-        __syncwarp();
       }
       for (int jj = 0; jj < n_local && ok; ++jj) {
-        const int vi = 2 * jj + 1, vs = vi % kSlots;
-        if (!(ok = mbar_wait_warp(full_bar(vs), (uint32_t)((vi / kSlots) & 1), abort_flag, p.dev_status))) break;
+        const int st = jj % kStages;
+        const uint32_t ph = (uint32_t)((jj / kStages) & 1);
         const int t0 = (kt_begin + jj) * 128;
-        if (t0 + 128 > N) {
-          // V rows past the sequence: zero them so that P = 0 never meets a non-finite value
-          const int r0 = N - t0;
-          const int nchunks = (128 - r0) * 16;
-          for (int c = lane; c < nchunks; c += 32) {
-            const int r = r0 + (c >> 4), hc = c & 15;
-            const uint32_t addr = ring + (uint32_t)vs * kTileBytes + (uint32_t)(hc >> 3) * kHalfBytes +
-                                  (uint32_t)r * 128u + (uint32_t)(hc & 7) * 16u;
-            st_shared_v4(addr, 0, 0, 0, 0);
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-        }
-        if (!(ok = mbar_wait_warp(pfull_bar(0), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
+        // V of this tile (zeroed past the sequence by the producer warp on the last tile)
+        if (!(ok = (t0 + 128 > N) ? mbar_wait(vzero_bar, 0, abort_flag, p.dev_status)
+                                  : mbar_wait(fullv_bar(st), ph, abort_flag, p.dev_status)))
+          break;
+        if (!(ok = mbar_wait(pfull_bar(0), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
         tc_fence_after();
-        if (lane == 0) issue_pv(0, vs, jj > 0);
+        issue_pv(0, st, jj > 0);
         const bool more = jj + 1 < n_local;
-        const int ki = 2 * jj + 2, ks = ki % kSlots;
+        const int st1 = (jj + 1) % kStages;
         if (more) {
-          if (!(ok = mbar_wait_warp(full_bar(ks), (uint32_t)((ki / kSlots) & 1), abort_flag, p.dev_status))) break;
+          if (!(ok = mbar_wait(fullk_bar(st1), (uint32_t)(((jj + 1) / kStages) & 1), abort_flag, p.dev_status)))
+            break;
           tc_fence_after();
-          if (lane == 0) {
-            issue_s(0, ks);
-            mma_commit(sfull_bar(0));
-          }
+          issue_s(0, st1);
+          mma_commit(sfull_bar(0));
         }
         if (nt == 2) {
-          if (!(ok = mbar_wait_warp(pfull_bar(1), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
+          if (!(ok = mbar_wait(pfull_bar(1), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
           tc_fence_after();
-          if (lane == 0) issue_pv(1, vs, jj > 0);
+          issue_pv(1, st, jj > 0);
         }
-        if (lane == 0) mma_commit(empty_bar(vs));
-        if (more && lane == 0) {
-          if (nt == 2) {
-            issue_s(1, ks);
-            mma_commit(sfull_bar(1));
-          }
-          mma_commit(empty_bar(ks));
-        }
-        __syncwarp();
-      }
-      if (lane == 0) {
-        mma_commit(ofull_bar(0));
-        if (nt == 2) mma_commit(ofull_bar(1));
-        if (!ok) {
-          // error path: let the tensor core finish what was issued before TMEM is freed
-          mma_commit(drain_bar);
-          mbar_drain(drain_bar, 0, 100000000ull);
+        mma_commit(empty_bar(st));   // K and V of this stage are no longer read
+        if (more && nt == 2) {
+          issue_s(1, st1);
+          mma_commit(sfull_bar(1));
         }
       }
-      __syncwarp();
+      mma_commit(ofull_bar(0));
+      if (nt == 2) mma_commit(ofull_bar(1));
+      if (!ok) {
+        // error path: let the tensor core finish what was issued before TMEM is freed
+        mma_commit(drain_bar);
+        mbar_drain(drain_bar, 0, 100000000ull);
+      }
     }
   } else if (active_t) {
     // ================================================================ softmax / epilogue
@@ -403,49 +407,61 @@ __global__ void __launch_bounds__(kThreads, 1)
             sv[c * 32 + e] = ((vw >> e) & 1u) ? sv[c * 32 + e] : __float_as_uint(-INFINITY);
         }
       }
-      // row max of the visible scores (masked entries are -inf)
-      float mx;
-      {
-        float a0 = -INFINITY, a1 = -INFINITY, a2 = -INFINITY, a3 = -INFINITY;
+      // P = 2^(s * scale * log2e - m) (masked: 2^-inf = 0), bf16 into the first 64 columns
+      // of S_t; returns the row sum and (optionally) the row max of s.
+      auto exp_pass = [&](float m_ref, float& mx_out) -> float {
+        const unsigned long long negm = f2_pack(-m_ref, -m_ref);
+        unsigned long long sum = f2_pack(0.f, 0.f);
+        float a0 = -INFINITY, a1 = -INFINITY;
 #pragma unroll
-        for (int e = 0; e < 128; e += 8) {
-          a0 = fmax3(a0, __uint_as_float(sv[e + 0]), __uint_as_float(sv[e + 1]));
-          a1 = fmax3(a1, __uint_as_float(sv[e + 2]), __uint_as_float(sv[e + 3]));
-          a2 = fmax3(a2, __uint_as_float(sv[e + 4]), __uint_as_float(sv[e + 5]));
-          a3 = fmax3(a3, __uint_as_float(sv[e + 6]), __uint_as_float(sv[e + 7]));
+        for (int c = 0; c < 8; ++c) {
+          uint32_t pk[8];
+#pragma unroll
+          for (int e = 0; e < 16; e += 2) {
+            const float s0 = __uint_as_float(sv[c * 16 + e]), s1 = __uint_as_float(sv[c * 16 + e + 1]);
+            if (e & 2)
+              a1 = fmax3(a1, s0, s1);
+            else
+              a0 = fmax3(a0, s0, s1);
+            const unsigned long long x = f2_fma(f2_pack(s0, s1), sl2x2, negm);
+            float x0, x1;
+            f2_unpack(x, x0, x1);
+            const float p0 = ptx_exp2(x0), p1 = ptx_exp2(x1);
+            sum = f2_add(sum, f2_pack(p0, p1));
+            pk[e >> 1] = pack_bf16x2(p0, p1);
+          }
+          tmem_st8(tS + (uint32_t)c * 8u, pk);
         }
-        mx = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3));
-      }
-      const float m_tile = mx * sl2;
-      // lazy rescaling: move the reference max only when it grows by more than 2^8
-      const bool rescale = m_tile > m_run + kRescaleLog2;
-      const float alpha = (rescale && jj > 0) ? ptx_exp2(m_run - m_tile) : 1.f;
-      if (rescale) m_run = m_tile;
-      const float m_use = m_run == -INFINITY ? 0.f : m_run;
-      const unsigned long long negm = f2_pack(-m_use, -m_use);
-      // P = 2^(s * scale * log2e - m) (masked: 2^-inf = 0), bf16 into the first 64 columns of S_t
-      unsigned long long sum = f2_pack(0.f, 0.f);
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        uint32_t pk[8];
-#pragma unroll
-        for (int e = 0; e < 16; e += 2) {
-          const unsigned long long x = f2_fma(
-              f2_pack(__uint_as_float(sv[c * 16 + e]), __uint_as_float(sv[c * 16 + e + 1])), sl2x2, negm);
-          float x0, x1;
-          f2_unpack(x, x0, x1);
-          const float p0 = ptx_exp2(x0), p1 = ptx_exp2(x1);
-          sum = f2_add(sum, f2_pack(p0, p1));
-          pk[e >> 1] = pack_bf16x2(p0, p1);
-        }
-        tmem_st8(tS + (uint32_t)c * 8u, pk);
-      }
-      {
+        mx_out = fmaxf(a0, a1);
         float s0, s1;
         f2_unpack(sum, s0, s1);
-        l_run = l_run * alpha + (s0 + s1);
+        return s0 + s1;
+      };
+      float alpha = 1.f, tile_sum, mx;
+      if (m_run == -INFINITY) {
+        // no reference yet: row max first
+        float b0 = -INFINITY, b1 = -INFINITY, b2 = -INFINITY, b3 = -INFINITY;
+#pragma unroll
+        for (int e = 0; e < 128; e += 8) {
+          b0 = fmax3(b0, __uint_as_float(sv[e + 0]), __uint_as_float(sv[e + 1]));
+          b1 = fmax3(b1, __uint_as_float(sv[e + 2]), __uint_as_float(sv[e + 3]));
+          b2 = fmax3(b2, __uint_as_float(sv[e + 4]), __uint_as_float(sv[e + 5]));
+          b3 = fmax3(b3, __uint_as_float(sv[e + 6]), __uint_as_float(sv[e + 7]));
+        }
+        m_run = fmaxf(fmaxf(b0, b1), fmaxf(b2, b3)) * sl2;   // stays -inf if nothing is visible
+        tile_sum = exp_pass(m_run == -INFINITY ? 0.f : m_run, mx);
+      } else {
+        // exponentials against the running max; redo only if this tile raises it by > 2^8
+        tile_sum = exp_pass(m_run, mx);
+        const float m_tile = mx * sl2;
+        if (m_tile > m_run + kRescaleLog2) {
+          alpha = ptx_exp2(m_run - m_tile);
+          m_run = m_tile;
+          tile_sum = exp_pass(m_run, mx);
+        }
       }
-      if (rescale && jj > 0) {
+      l_run = l_run * alpha + tile_sum;
+      if (alpha != 1.f) {
         // O_t is idle here: PV_t of the previous tile completed before S_t of this one
 #pragma unroll 1
         for (int c = 0; c < 8; ++c) {
@@ -459,7 +475,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(pfull_bar(t));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(pfull_bar(t));
     }
     // ---- epilogue
     ok = __all_sync(0xffffffffu, ok);
