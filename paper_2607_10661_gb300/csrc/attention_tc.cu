@@ -384,94 +384,91 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tS = tmem + lane_base + (uint32_t)t * 128u;
     const uint32_t tO = tmem + lane_base + 256u + (uint32_t)t * 128u;
     const unsigned long long sl2x2 = f2_pack(sl2, sl2);
+    // Reference max m_run (log2 units) against which P = 2^(s*scale*log2e - m_run) is taken.
+    // It only moves up, and only when a 32-column chunk exceeds it by more than 2^8; then the
+    // row sum, O and the P chunks already written for this tile are rescaled (rare).
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     uint32_t r[32];
-    uint32_t sv[128];   // the thread's whole S row: one TMEM wait per tile
     for (int jj = 0; jj < n_local; ++jj) {
       if (!(ok = mbar_wait_warp(sfull_bar(t), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
       tc_fence_after();
-      tmem_ld32(tS + 0u, *reinterpret_cast<uint32_t(*)[32]>(sv + 0));
-      tmem_ld32(tS + 32u, *reinterpret_cast<uint32_t(*)[32]>(sv + 32));
-      tmem_ld32(tS + 64u, *reinterpret_cast<uint32_t(*)[32]>(sv + 64));
-      tmem_ld32(tS + 96u, *reinterpret_cast<uint32_t(*)[32]>(sv + 96));
-      tmem_ld_wait();
       const int t0 = (kt_begin + jj) * 128;
       const bool need_mask = t0 + 128 > C;   // warp-uniform
-      if (need_mask) {
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
+      unsigned long long sum = f2_pack(0.f, 0.f);
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        tmem_ld32(tS + (uint32_t)c * 32u, r);
+        tmem_ld_wait();
+        if (need_mask) {
           const uint32_t vw = vis_word(t0 + c * 32 - C, am0, am1, am2, am3);
 #pragma unroll
-          for (int e = 0; e < 32; ++e)
-            sv[c * 32 + e] = ((vw >> e) & 1u) ? sv[c * 32 + e] : __float_as_uint(-INFINITY);
+          for (int e = 0; e < 32; ++e) r[e] = ((vw >> e) & 1u) ? r[e] : __float_as_uint(-INFINITY);
         }
-      }
-      // P = 2^(s * scale * log2e - m) (masked: 2^-inf = 0), bf16 into the first 64 columns
-      // of S_t; returns the row sum and (optionally) the row max of s.
-      auto exp_pass = [&](float m_ref, float& mx_out) -> float {
-        const unsigned long long negm = f2_pack(-m_ref, -m_ref);
-        unsigned long long sum = f2_pack(0.f, 0.f);
-        float a0 = -INFINITY, a1 = -INFINITY;
+        float cm;
+        {
+          float a0 = -INFINITY, a1 = -INFINITY;
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          uint32_t pk[8];
-#pragma unroll
-          for (int e = 0; e < 16; e += 2) {
-            const float s0 = __uint_as_float(sv[c * 16 + e]), s1 = __uint_as_float(sv[c * 16 + e + 1]);
-            if (e & 2)
-              a1 = fmax3(a1, s0, s1);
-            else
-              a0 = fmax3(a0, s0, s1);
-            const unsigned long long x = f2_fma(f2_pack(s0, s1), sl2x2, negm);
-            float x0, x1;
-            f2_unpack(x, x0, x1);
-            const float p0 = ptx_exp2(x0), p1 = ptx_exp2(x1);
-            sum = f2_add(sum, f2_pack(p0, p1));
-            pk[e >> 1] = pack_bf16x2(p0, p1);
+          for (int e = 0; e < 32; e += 4) {
+            a0 = fmax3(a0, __uint_as_float(r[e]), __uint_as_float(r[e + 1]));
+            a1 = fmax3(a1, __uint_as_float(r[e + 2]), __uint_as_float(r[e + 3]));
           }
-          tmem_st8(tS + (uint32_t)c * 8u, pk);
+          cm = fmaxf(a0, a1) * sl2;
         }
-        mx_out = fmaxf(a0, a1);
+        if (cm > m_run + kRescaleLog2) {
+          // raise the reference: rescale everything taken against the old one
+          const float alpha = m_run == -INFINITY ? 0.f : ptx_exp2(m_run - cm);
+          float s0, s1;
+          f2_unpack(sum, s0, s1);
+          sum = f2_pack(s0 * alpha, s1 * alpha);
+          l_run *= alpha;
+          m_run = cm;
+          if (jj > 0) {
+            // O_t is idle here: PV_t of the previous tile completed before S_t of this one
+#pragma unroll 1
+            for (int q = 0; q < 8; ++q) {
+              uint32_t o16[16];
+              tmem_ld16(tO + (uint32_t)q * 16u, o16);
+              tmem_ld_wait();
+#pragma unroll
+              for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
+              tmem_st16(tO + (uint32_t)q * 16u, o16);
+            }
+          }
+          if (c > 0) {
+            tmem_st_wait();
+#pragma unroll 1
+            for (int q = 0; q < c; ++q) {   // bf16 P of the earlier chunks of this tile
+              uint32_t p16[16];
+              tmem_ld16(tS + (uint32_t)q * 16u, p16);
+              tmem_ld_wait();
+#pragma unroll
+              for (int e = 0; e < 16; ++e)
+                p16[e] = pack_bf16x2(__uint_as_float(p16[e] << 16) * alpha,
+                                     __uint_as_float(p16[e] & 0xFFFF0000u) * alpha);
+              tmem_st16(tS + (uint32_t)q * 16u, p16);
+            }
+          }
+        }
+        const float m_use = m_run == -INFINITY ? 0.f : m_run;   // -inf only when nothing is visible yet
+        const unsigned long long negm = f2_pack(-m_use, -m_use);
+        uint32_t pk[16];
+#pragma unroll
+        for (int e = 0; e < 32; e += 2) {
+          const unsigned long long x =
+              f2_fma(f2_pack(__uint_as_float(r[e]), __uint_as_float(r[e + 1])), sl2x2, negm);
+          float x0, x1;
+          f2_unpack(x, x0, x1);
+          const float p0 = ptx_exp2(x0), p1 = ptx_exp2(x1);
+          sum = f2_add(sum, f2_pack(p0, p1));
+          pk[e >> 1] = pack_bf16x2(p0, p1);
+        }
+        tmem_st16(tS + (uint32_t)c * 16u, pk);   // P chunk c: columns [16c, 16c+16) of S_t
+      }
+      {
         float s0, s1;
         f2_unpack(sum, s0, s1);
-        return s0 + s1;
-      };
-      float alpha = 1.f, tile_sum, mx;
-      if (m_run == -INFINITY) {
-        // no reference yet: row max first
-        float b0 = -INFINITY, b1 = -INFINITY, b2 = -INFINITY, b3 = -INFINITY;
-#pragma unroll
-        for (int e = 0; e < 128; e += 8) {
-          b0 = fmax3(b0, __uint_as_float(sv[e + 0]), __uint_as_float(sv[e + 1]));
-          b1 = fmax3(b1, __uint_as_float(sv[e + 2]), __uint_as_float(sv[e + 3]));
-          b2 = fmax3(b2, __uint_as_float(sv[e + 4]), __uint_as_float(sv[e + 5]));
-          b3 = fmax3(b3, __uint_as_float(sv[e + 6]), __uint_as_float(sv[e + 7]));
-        }
-        m_run = fmaxf(fmaxf(b0, b1), fmaxf(b2, b3)) * sl2;   // stays -inf if nothing is visible
-        tile_sum = exp_pass(m_run == -INFINITY ? 0.f : m_run, mx);
-      } else {
-        // exponentials against the running max; redo only if this tile raises it by > 2^8
-        tile_sum = exp_pass(m_run, mx);
-        const float m_tile = mx * sl2;
-        if (m_tile > m_run + kRescaleLog2) {
-          alpha = ptx_exp2(m_run - m_tile);
-          m_run = m_tile;
-          tile_sum = exp_pass(m_run, mx);
-        }
-      }
-      l_run = l_run * alpha + tile_sum;
-      if (alpha != 1.f) {
-        // O_t is idle here: PV_t of the previous tile completed before S_t of this one
-#pragma unroll 1
-        for (int c = 0; c < 8; ++c) {
-          uint32_t o16[16];
-          tmem_ld16(tO + (uint32_t)c * 16u, o16);
-          tmem_ld_wait();
-#pragma unroll
-          for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
-          tmem_st16(tO + (uint32_t)c * 16u, o16);
-        }
+        l_run += s0 + s1;
       }
       tmem_st_wait();
       tc_fence_before();
