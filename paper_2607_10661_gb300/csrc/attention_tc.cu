@@ -12,7 +12,7 @@
 // K/V tile is loaded from HBM once by TMA and used by both M tiles.
 //
 // Warp roles (320 threads):
-//   warp 0      TMA producer: K, V tiles into a 5-slot ring (K_j, V_j, K_j+1, ...).
+//   warp 0      TMA producer: K and V tiles into two stage pairs (K_j, V_j | K_j+1, V_j+1).
 //   warp 1      TMEM allocator and MMA issuer (one thread issues tcgen05.mma):
 //                 S_t = Q_t K_j^T    (Q and K from shared memory, fp32 S in TMEM)
 //                 O_t += P_t V_j     (P from TMEM, where the softmax wrote it over S_t;
@@ -415,14 +415,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           cm = fmaxf(a0, a1) * sl2;
         }
-        if (cm > m_run + kRescaleLog2) {
+        // The TMEM accesses of a rescale are warp-collective, so the whole warp takes the
+        // branch when any of its rows needs it; the other rows rescale by exactly 1.  (Rows
+        // differ when a split starts on a key tile past the committed context: each row
+        // first meets a visible ancestor in whichever chunk holds one.)
+        const bool raise = cm > m_run + kRescaleLog2;
+        if (__any_sync(0xffffffffu, raise)) {
           // raise the reference: rescale everything taken against the old one
-          const float alpha = m_run == -INFINITY ? 0.f : ptx_exp2(m_run - cm);
+          float alpha = 1.f;
+          if (raise) {
+            alpha = m_run == -INFINITY ? 0.f : ptx_exp2(m_run - cm);
+            m_run = cm;
+          }
           float s0, s1;
           f2_unpack(sum, s0, s1);
           sum = f2_pack(s0 * alpha, s1 * alpha);
           l_run *= alpha;
-          m_run = cm;
           if (jj > 0) {
             // O_t is idle here: PV_t of the previous tile completed before S_t of this one
 #pragma unroll 1

@@ -81,6 +81,11 @@ ATTN_CASES = {
     "single-node": ("llama3-8b-gqa", dict(layers=1, ctx=(200, 200), vocab=100, tree="chain", nodes=(1, 1))),
     "mha-g1-t64": ("llama2-7b-layer", dict(hq=4, hkv=4, ctx=(129, 129), vocab=100, tree="chain",
                                            nodes=(64, 64))),
+    # one key tile per split; the last split starts at node 63 of a complete binary tree, so
+    # within one warp nodes 88..94 first see a visible key (themselves) in chunk 0 and node
+    # 95 only in chunk 1: the lazy rescale must still run warp-uniformly
+    "split-on-tree-tile": ("llama3-8b-gqa", dict(layers=1, hq=4, hkv=1, ctx=(961, 961), vocab=100, tree="binary",
+                                                  nodes=(127, 127))),
 }
 
 
