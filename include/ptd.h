@@ -93,9 +93,12 @@ typedef struct {
   int32_t max_pages;           /* paged: entries per block-table row                   */
 } ptd_kv_cache;
 
-/* Bytes of scratch `ptd_tree_attention` wants for these shapes (0 if it needs none).
- * Passing less (even 0 with a NULL pointer) is allowed: the call then uses fewer
- * key splits, down to one split which needs no scratch. */
+/* Bytes of scratch `ptd_tree_attention` wants for these shapes (0 if it needs none):
+ * per-block counters and the fp32 partials of the units that the balanced schedule splits
+ * between neighbouring SMs.  Passing less (even 0 with a NULL pointer) is allowed: the
+ * call then computes each (layer, tree, KV head, 256-row block) in one CTA, which needs no
+ * scratch but leaves SMs idle when such units are few or their count is not a multiple of
+ * the SM count. */
 size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache,
                                     int32_t num_q_heads, int32_t num_layers);
 
@@ -124,13 +127,13 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache,
  * runtime's engine may have no allocator of its own to ask, and a latency-critical decode
  * loop may not tolerate cudaMalloc, whose implicit device synchronisation stalls every
  * stream.  This variant computes exactly what ptd_tree_attention computes, with the same
- * key-split schedule, but takes its split scratch from a fixed array that the library
+ * schedule, but takes its scratch from a fixed array that the library
  * holds in device memory (PTD_STATIC_SCRATCH_BYTES; every GPU that loads the library keeps
  * it until the process exits) instead of from a caller workspace.  The paper has no
  * counterpart of this entry point.
  *   - Arguments are those of ptd_tree_attention without workspace / workspace_bytes.
- *   - If the split schedule for these shapes needs more than PTD_STATIC_SCRATCH_BYTES of
- *     scratch (ptd_attention_workspace_size > PTD_STATIC_SCRATCH_BYTES) the call returns
+ *   - If these shapes need more than PTD_STATIC_SCRATCH_BYTES of scratch
+ *     (ptd_attention_workspace_size > PTD_STATIC_SCRATCH_BYTES) the call returns
  *     PTD_ERR_WORKSPACE and enqueues nothing; use ptd_tree_attention with a workspace then.
  *   - The first call on each device resolves the array's device address on that device
  *     (make that device current); issue that first call before any stream capture.

@@ -20,7 +20,6 @@ namespace {
 
 thread_local int32_t g_last_launches = 0;
 
-constexpr int kMaxSplits = 16;
 constexpr int kMaxDevices = 64;
 
 int num_sms_of_current_device() {
@@ -93,26 +92,21 @@ void tc_geometry(const ptd_tree* t, const ptd_kv_cache* c, int hq, int layers, i
   *n_kt_max = (t->max_ctx + t->max_nodes + 127) / 128;
 }
 
-// Split count: minimise (waves of CTAs) x (key tiles per CTA + fixed cost); one split
-// needs no scratch and no combine pass, so it wins ties.
-int choose_splits(int units, int n_kt, int sms) {
-  int best = 1;
-  double best_cost = 1e300;
-  for (int s = 1; s <= kMaxSplits && s <= n_kt; ++s) {
-    const double waves = std::ceil((double)units * s / sms);
-    const double cost = waves * (std::ceil((double)n_kt / s) + 2.0) + (s > 1 ? 1.0 : 0.0);
-    if (cost < best_cost - 1e-9) {
-      best_cost = cost;
-      best = s;
-    }
-  }
-  return best;
+// Persistent schedule: one CTA per SM (fewer for tiny problems); per-(unit, 32-row block)
+// piece counters and two partial slots per CTA (the pieces at either end of its range).
+int persistent_ctas(int units, int n_kt, int sms) {
+  const long long w = (long long)units * n_kt;
+  return (int)(w < sms ? w : sms);
 }
 
-size_t split_workspace_bytes(int units, int splits, int head_dim) {
-  if (splits <= 1) return 0;
-  return (size_t)units * splits * 256 * ((size_t)head_dim + 2) * sizeof(float);
+size_t counters_bytes(int units) { return (((size_t)units * 8 * sizeof(int32_t)) + 255) / 256 * 256; }
+
+size_t persistent_workspace_bytes(int units, int ctas, int head_dim) {
+  return counters_bytes(units) + (size_t)2 * ctas * 256 * ((size_t)head_dim + 2) * sizeof(float);
 }
+
+// Tile indices of the persistent schedule are 32-bit.
+bool persistent_fits(int units, int n_kt) { return (long long)units * n_kt < (1ll << 30); }
 
 ptd_status cuda_status(cudaError_t e) { return e == cudaSuccess ? PTD_OK : PTD_ERR_CUDA; }
 
@@ -149,8 +143,10 @@ size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* ca
     return 0;
   int pairs, units, n_kt;
   tc_geometry(tree, cache, num_q_heads, num_layers, &pairs, &units, &n_kt);
-  const int s = choose_splits(units, n_kt, num_sms_of_current_device());
-  return split_workspace_bytes(units, s, cache->head_dim);
+  if (units <= 0 || n_kt <= 0) return 0;
+  const int sms = num_sms_of_current_device();
+  if (!persistent_fits(units, n_kt)) return 0;
+  return persistent_workspace_bytes(units, persistent_ctas(units, n_kt, sms), cache->head_dim);
 }
 
 ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
@@ -195,7 +191,6 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
 
   if (cache->dtype == PTD_F32) {
     if (D != 32 && D != 64 && D != 128) return PTD_ERR_UNSUPPORTED;
-    p.splits = 1;
     p.pairs = 1;
     st = cuda_status(ptd::launch_tree_attn_simt(p, s));
     if (st == PTD_OK) g_last_launches = 1;
@@ -205,15 +200,22 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
 
   int pairs, units, n_kt;
   tc_geometry(tree, cache, num_q_heads, num_layers, &pairs, &units, &n_kt);
-  if (units <= 0) return PTD_ERR_INVALID_ARG;
-  int splits = choose_splits(units, n_kt, num_sms_of_current_device());
-  while (splits > 1 && (workspace == nullptr || split_workspace_bytes(units, splits, D) > workspace_bytes)) --splits;
+  if (units <= 0 || n_kt <= 0) return PTD_ERR_INVALID_ARG;
   p.pairs = pairs;
-  p.splits = splits;
-  if (splits > 1) {
-    if (!aligned16(workspace)) return PTD_ERR_WORKSPACE;
-    p.part_o = static_cast<float*>(workspace);
-    p.part_ml = p.part_o + (size_t)units * splits * 256 * D;
+  const int sms = num_sms_of_current_device();
+  const int ctas = persistent_ctas(units, n_kt, sms);
+  const bool persistent = persistent_fits(units, n_kt) && workspace != nullptr && aligned16(workspace) &&
+                          workspace_bytes >= persistent_workspace_bytes(units, ctas, D);
+  dim3 grid;
+  if (persistent) {
+    p.persistent = 1;
+    p.counters = static_cast<int32_t*>(workspace);
+    p.part_o = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + counters_bytes(units));
+    p.part_ml = p.part_o + (size_t)2 * ctas * 256 * D;
+    grid = dim3((unsigned)ctas, 1, 1);
+  } else {
+    p.persistent = 0;   // one CTA per unit, no scratch
+    grid = dim3((unsigned)units, 1, 1);
   }
 
   PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
@@ -234,13 +236,10 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return PTD_ERR_CUDA;
 
-  if ((st = cuda_status(ptd::launch_tree_attn_tc(map_k, map_v, p, units, s))) != PTD_OK) return st;
-  int launches = 1;
-  if (splits > 1) {
-    if ((st = cuda_status(ptd::launch_attn_combine(p, units, s))) != PTD_OK) return st;
-    ++launches;
-  }
-  g_last_launches = launches;
+  if (persistent && cudaMemsetAsync(p.counters, 0, (size_t)units * 8 * sizeof(int32_t), s) != cudaSuccess)
+    return PTD_ERR_CUDA;
+  if ((st = cuda_status(ptd::launch_tree_attn_tc(map_k, map_v, p, grid, s))) != PTD_OK) return st;
+  g_last_launches = 1;   // (the counter clear before it is a memset, not a kernel of this library)
   return PTD_OK;
 }
 

@@ -12,8 +12,9 @@ namespace ptd {
 struct AttnParams {
   const void* q;               // [layers][n_total][hq][D]
   void* out;                   // [layers][n_total][hq][D]
-  float* part_o;               // split partials: [units][splits][256][D] fp32
-  float* part_ml;              // [units][splits][256][2] (running max in log2 units, sum)
+  float* part_o;               // piece partials: [slot][M tile][D][128 rows] fp32 (O unnormalised)
+  float* part_ml;              // [slot][256 rows][2] (running max in log2 units, row sum)
+  int32_t* counters;           // persistent schedule: pieces finished per (unit, 32-row block)
   const int32_t* node_offsets;
   const int32_t* parents;
   const int32_t* ctx_lens;
@@ -25,7 +26,7 @@ struct AttnParams {
   int layer_begin, layers;     // layers of this call
   int n_total, max_nodes;
   int pairs;                   // 256-row M-tile pairs per (tree, KV head)
-  int splits;                  // KV splits
+  int persistent;              // 1: balanced persistent schedule, one CTA per SM
   int page_size, seq_capacity, num_pages, max_pages;
   float scale_log2;            // scale * log2(e)
   float scale;
@@ -33,8 +34,7 @@ struct AttnParams {
 
 size_t tc_smem_bytes();
 cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const AttnParams& p,
-                                int units, cudaStream_t stream);
-cudaError_t launch_attn_combine(const AttnParams& p, int units, cudaStream_t stream);
+                                dim3 grid, cudaStream_t stream);
 cudaError_t launch_tree_attn_simt(const AttnParams& p, cudaStream_t stream);
 
 }  // namespace ptd

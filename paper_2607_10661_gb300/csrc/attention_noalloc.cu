@@ -1,10 +1,11 @@
-// Tree attention without a caller workspace: the key-split scratch is a file-scope device
-// array of PTD_STATIC_SCRATCH_BYTES (declared in include/ptd.h).
+// Tree attention without a caller workspace: the scratch is a file-scope device array of
+// PTD_STATIC_SCRATCH_BYTES (declared in include/ptd.h).
 //
 // In host code the array's name only stands for the symbol; its device address is looked
 // up once per device with cudaGetSymbolAddress (with that device current) and cached.
-// The split partials written by one call are read back only by that same call's combine
-// pass, and each partial row is written before it is read, so no clearing is needed.
+// Each call clears the piece counters at the front of the scratch before its kernel; the
+// partials written by one call are read back only by that same call, and each partial row
+// is written before it is read, so nothing else needs clearing.
 #include <cuda_runtime.h>
 
 #include <cstdint>

@@ -7,9 +7,19 @@
 //
 // Work decomposition.  All G = Hq/Hkv query heads of one KV head and all T_b nodes of a
 // tree form the rows of one dense problem: row r = node * G + g, so M = T_b * G rows share
-// every K/V tile.  A CTA owns two 128-row M tiles (256 rows, e.g. 63 nodes x 4 heads) of
-// one (layer, tree, KV head) and a contiguous range of 128-key tiles (a KV split).  Each
-// K/V tile is loaded from HBM once by TMA and used by both M tiles.
+// every K/V tile.  A unit is one (layer, tree, KV head, pair of 128-row M tiles), e.g. 63
+// nodes x 4 heads = 252 rows, and its keys are cut into 128-key tiles.  Each K/V tile is
+// loaded from HBM once by TMA and used by both M tiles.
+//
+// Schedules.  Persistent (the default when the caller's scratch allows it): the flattened
+// (unit, key tile) space is cut into one equal contiguous range per CTA, one CTA per SM, so
+// every SM gets the same number of key tiles whatever the unit count.  Each warp walks its
+// CTA's range as segments (whole units, or a piece of a unit at either end of the range).
+// Whole units are written directly; a piece writes an fp32 partial (O unnormalised, running
+// max, row sum), and the warp that writes the last piece of a 32-row block merges the
+// pieces of that block once its own range is done.  The softmax warps load the next
+// segment's Q before the epilogue of the current one, so the tensor core does not wait on
+// it.  Grid (fallback without scratch): one CTA per unit.
 //
 // Warp roles (320 threads):
 //   warp 0      TMA producer: K and V tiles into two stage pairs (K_j, V_j | K_j+1, V_j+1).
@@ -22,7 +32,7 @@
 //   warps 2-5   softmax of M tile 0, warps 6-9 of M tile 1 (thread = row = TMEM lane
 //               (warp % 4) * 32 + lane): row max, lazy rescaling of O (only when the
 //               running max grows by more than 2^8), exp2, bf16 P back into TMEM, row sum;
-//               at the end O / l (or a split partial).  Tiles that lie entirely inside the
+//               at the end O / l (or a piece's partial).  Tiles that lie entirely inside the
 //               committed prefix skip the mask arithmetic.
 // TMEM: S_0 | S_1 | O_0 | O_1, 128 fp32 columns each = all 512 columns of the SM; P_t
 // takes the first 64 columns of S_t (two bf16 per column).
@@ -30,6 +40,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <climits>
 #include <cmath>
 #include <cstdint>
 
@@ -46,15 +57,15 @@ constexpr uint32_t kHalfBytes = 16384;   // 128 rows x 64 bf16 (one 128-byte swi
 constexpr uint32_t kStageBytes = 2 * kTileBytes;
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffRing = 2 * kTileBytes;
-constexpr uint32_t kOffScratch = kOffRing + kStageBytes + kTileBytes;   // setup only (V of stage 1)
 constexpr uint32_t kOffBar = kOffRing + kStages * kStageBytes;
-// barriers: full_k[2], full_v[2], empty[2], vzero, s_full[2], p_full[2], o_full[2], drain
-constexpr uint32_t kNumBars = 3 * kStages + 8;
+// barriers: full_k[2], full_v[2], empty_k[2], v_load[2], s_full[2], p_full[2], o_full[2], drain, q_ready[2],
+// empty_v[2]
+constexpr uint32_t kNumBars = 5 * kStages + 9;
 constexpr uint32_t kOffTmemPtr = kOffBar + kNumBars * 8;
 constexpr uint32_t kOffAbort = kOffTmemPtr + 4;
-constexpr uint32_t kSmemUsed = kOffAbort + 4;
-constexpr uint32_t kSmemBytes = kSmemUsed + 1024;   // slack to align the base to 1024 B
-static_assert(kSmemBytes <= 232448, "shared memory budget");
+constexpr uint32_t kOffSched = (kOffAbort + 4 + 15) / 16 * 16;   // schedule constants + one slot per warp
+constexpr uint32_t kSchedBytes = 1024;
+constexpr uint32_t kOffWarp = kOffSched + kSchedBytes;   // one WarpArea per softmax warp (below)
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleLog2 = 8.0f;                // lazy rescale threshold (log2 units)
 
@@ -76,6 +87,196 @@ __device__ __forceinline__ uint32_t vis_word(int a0, uint32_t m0, uint32_t m1, u
   return __funnelshift_r(lo, hi, sh);
 }
 
+// One segment of work: key tiles [kt_begin, kt_end) of one unit.
+struct Seg {
+  int lq, b, hkv, mp;          // layer within the call, tree, KV head, M-tile pair
+  int node0, T, C, N;          // the tree's first node, size, committed context, keys
+  int n_kt, nt;                // key tiles of the unit, M tiles of the pair (1 or 2)
+  int kt_begin, kt_end;
+  int unit;                    // canonical unit id (layer, tree, KV head, pair)
+  int ug0;                     // global index of the unit's key tile 0 (persistent)
+  int slot;                    // partial slot, or -1 when the segment is the whole unit
+  int valid;                   // 0: no more segments
+};
+
+// A segment taken by a softmax warp, with the validity of its tree.
+struct SegRun {
+  Seg s;
+  int invalid;
+  int pad;
+};
+
+// A range holds at most two pieces (its first and its last segment), so a warp leaves at
+// most two merges for the end.
+constexpr int kMaxDefer = 2;
+
+// Shared memory of one softmax warp.
+struct WarpArea {
+  int parents[128];            // parent array of the last tree seen
+  SegRun run[2];               // the segment being computed and the next one
+  SegRun defer[kMaxDefer];     // 32-row blocks to merge at the end of the range
+  int tree_node0, tree_T;      // which tree `parents` holds
+  int tree_invalid;            // that tree failed the parent check
+  int mask_mp;                 // M-tile pair the ancestor masks in registers were built for
+  int ndefer;
+  int pad[3];
+};
+constexpr uint32_t kSmemUsed = kOffWarp + 8 * sizeof(WarpArea);
+constexpr uint32_t kSmemBytes = kSmemUsed + 1024;   // slack to align the base to 1024 B
+static_assert(kSmemBytes <= 232448, "shared memory budget");
+
+// Persistent schedule constants: CTA c owns global key tiles [c*W/P, (c+1)*W/P).
+struct WalkConst {
+  int persistent, W, Wl, P, c, r0, r1, backward;
+};
+
+// Tree b: first node, size, context, key tiles and M-tile pairs; returns the key tiles of all
+// its units in one layer (0 for a malformed entry, which is skipped and reported).
+__device__ __forceinline__ int seq_info(const AttnParams& p, int b, int& node0, int& T, int& C, int& n_kt,
+                                        int& pairs) {
+  node0 = p.node_offsets[b];
+  T = p.node_offsets[b + 1] - node0;
+  C = p.ctx_lens[b];
+  const int N = C + T;
+  const bool bad = T < 1 || T > p.max_nodes || node0 < 0 || node0 + T > p.n_total || C < 0 ||
+                   (p.page_size > 0 ? N > p.max_pages * p.page_size : N > p.seq_capacity);
+  if (bad) {
+    n_kt = 0;
+    pairs = 0;
+    return 0;
+  }
+  n_kt = (N + 127) >> 7;
+  pairs = ((T * p.group + 127) / 128 + 1) / 2;
+  return p.hkv * pairs * n_kt;
+}
+
+__device__ __forceinline__ void fill_seg(const AttnParams& p, Seg& s, int b, int node0, int T, int C, int n_kt) {
+  s.b = b;
+  s.node0 = node0;
+  s.T = T;
+  s.C = C;
+  s.N = C + T;
+  s.n_kt = n_kt;
+  s.nt = min(2, (T * p.group + 127) / 128 - 2 * s.mp);
+  s.unit = ((s.lq * p.batch + b) * p.hkv + s.hkv) * p.pairs + s.mp;
+}
+
+__device__ __forceinline__ int range_start(const WalkConst& wc, int c) {
+  return (int)((long long)c * wc.W / wc.P);
+}
+__device__ __forceinline__ int owner_cta(const WalkConst& wc, int g) {
+  return (int)(((long long)(g + 1) * wc.P - 1) / wc.W);
+}
+
+// Returns false (schedule inconsistent with the tree arrays) if g maps to no tree.
+__device__ __noinline__ bool decode_tile(const AttnParams& p, int Wl, int g, Seg& s) {
+  s.lq = g / Wl;
+  int r = g - s.lq * Wl;
+  for (int b = 0; b < p.batch; ++b) {
+    int node0, T, C, n_kt, pairs;
+    const int wb = seq_info(p, b, node0, T, C, n_kt, pairs);
+    if (r < wb) {
+      const int idx = r / n_kt;
+      const int tile = r - idx * n_kt;
+      s.hkv = idx / pairs;
+      s.mp = idx - s.hkv * pairs;
+      fill_seg(p, s, b, node0, T, C, n_kt);
+      s.ug0 = g - tile;
+      return true;
+    }
+    r -= wb;
+  }
+  return false;
+}
+
+__device__ __noinline__ void make_walk_const(const AttnParams& p, WalkConst& wc) {
+  wc.persistent = p.persistent;
+  if (!p.persistent) return;
+  int wl = 0;
+  for (int b = 0; b < p.batch; ++b) {
+    int node0, T, C, n_kt, pairs;
+    const int w = seq_info(p, b, node0, T, C, n_kt, pairs);
+    if (w == 0 && blockIdx.x == 0) atomicMax(p.dev_status, (int)PTD_ERR_INVALID_TREE);   // malformed sizes
+    wl += w;
+  }
+  wc.Wl = wl;
+  wc.W = wl * p.layers;
+  wc.P = (int)gridDim.x;
+  wc.c = (int)blockIdx.x;
+  wc.r0 = range_start(wc, wc.c);
+  wc.r1 = range_start(wc, wc.c + 1);
+  wc.backward = wc.c & 1;
+}
+
+// A walker's cursor before its first step.  A backward walk ends at g0 - 1 >= -1, so the
+// start value must lie outside [-1, W].
+constexpr int kWalkStart = INT_MIN;
+
+// Next segment of this CTA for one walker (cursor starts at kWalkStart); s.valid = 0 when done.
+__device__ __noinline__ void next_segment(const AttnParams& p, const WalkConst& wc, int& cursor, Seg& s) {
+  s.valid = 0;
+  if (!wc.persistent) {
+    // grid schedule: CTA u computes unit u whole
+    if (cursor != kWalkStart) return;
+    cursor = 0;
+    int u = blockIdx.x;
+    s.mp = u % p.pairs;
+    u /= p.pairs;
+    s.hkv = u % p.hkv;
+    u /= p.hkv;
+    const int b = u % p.batch;
+    s.lq = u / p.batch;
+    int node0, T, C, n_kt, pairs;
+    if (seq_info(p, b, node0, T, C, n_kt, pairs) == 0) {
+      atomicMax(p.dev_status, (int)PTD_ERR_INVALID_TREE);   // malformed sizes
+      return;
+    }
+    if (s.mp >= pairs) return;
+    fill_seg(p, s, b, node0, T, C, n_kt);
+    s.ug0 = 0;
+    s.kt_begin = 0;
+    s.kt_end = n_kt;
+    s.slot = -1;
+    s.valid = 1;
+    return;
+  }
+  if (wc.W <= 0) return;
+  if (cursor == kWalkStart) cursor = wc.backward ? wc.r1 - 1 : wc.r0;
+  // self-check: every step must decode and move the cursor (the walk then always ends)
+  auto fail = [&]() {
+    atomicMax(p.dev_status, (int)PTD_ERR_TIMEOUT);
+    cursor = wc.backward ? wc.r0 - 1 : wc.r1;
+  };
+  int g0, g1;
+  if (!wc.backward) {
+    if (cursor >= wc.r1) return;
+    if (!decode_tile(p, wc.Wl, cursor, s) || s.ug0 + s.n_kt <= cursor || s.ug0 > cursor) return fail();
+    g0 = cursor;
+    g1 = min(s.ug0 + s.n_kt, wc.r1);
+    cursor = g1;
+  } else {
+    if (cursor < wc.r0) return;
+    if (!decode_tile(p, wc.Wl, cursor, s) || s.ug0 + s.n_kt <= cursor || s.ug0 > cursor) return fail();
+    g1 = cursor + 1;
+    g0 = max(s.ug0, wc.r0);
+    cursor = g0 - 1;
+  }
+  s.kt_begin = g0 - s.ug0;
+  s.kt_end = g1 - s.ug0;
+  if (s.kt_begin == 0 && s.kt_end == s.n_kt) {
+    s.slot = -1;
+  } else {
+    s.slot = wc.c * 2 + ((wc.r0 >= s.ug0 && wc.r0 < s.ug0 + s.n_kt) ? 0 : 1);
+  }
+  s.valid = 1;
+}
+
+// Partial slot of CTA c's piece of the unit starting at global tile ug0 (c owns a piece).
+__device__ __forceinline__ int piece_slot(const WalkConst& wc, int c, int ug0, int ug1) {
+  const int rs = range_start(wc, c);
+  return c * 2 + ((rs >= ug0 && rs < ug1) ? 0 : 1);
+}
+
 template <bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
@@ -87,70 +288,46 @@ __global__ void __launch_bounds__(kThreads, 1)
   base += pad;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  // ---- work unit
-  int u = blockIdx.x;
-  const int unit = u;
-  const int mp = u % p.pairs;
-  u /= p.pairs;
-  const int hkv = u % p.hkv;
-  u /= p.hkv;
-  const int b = u % p.batch;
-  const int lq = u / p.batch;
-  const int layer = p.layer_begin + lq;
-  const int split = blockIdx.y;
   const int G = p.group;
-
-  const int node0 = p.node_offsets[b];
-  const int T = p.node_offsets[b + 1] - node0;
-  const int C = p.ctx_lens[b];
-  const int N = C + T;
-  bool bad_shape = T < 1 || T > p.max_nodes || node0 < 0 || node0 + T > p.n_total || C < 0;
-  if (!bad_shape) {
-    if (kPaged)
-      bad_shape = N > p.max_pages * p.page_size;
-    else
-      bad_shape = N > p.seq_capacity;
-  }
-  if (bad_shape) {
-    if (threadIdx.x == 0) atomicMax(p.dev_status, (int)PTD_ERR_INVALID_TREE);
-    return;
-  }
-  const int rows = T * G;
-  const int tiles_b = (rows + 127) >> 7;
-  const int nt = min(2, tiles_b - 2 * mp);
-  if (nt <= 0) return;   // this pair of M tiles is past the tree (uniform over the CTA)
-
-  const int n_kt = (N + 127) >> 7;
-  const int tps = (n_kt + p.splits - 1) / p.splits;
-  const int kt_begin = split * tps;
-  const int n_local = max(0, min(n_kt, kt_begin + tps) - kt_begin);
 
   auto bar = [&](int i) { return base + kOffBar + 8u * (uint32_t)i; };
   auto fullk_bar = [&](int s) { return bar(s); };
   auto fullv_bar = [&](int s) { return bar(kStages + s); };
-  auto empty_bar = [&](int s) { return bar(2 * kStages + s); };
-  const uint32_t vzero_bar = bar(3 * kStages);
-  auto sfull_bar = [&](int t) { return bar(3 * kStages + 1 + t); };
-  auto pfull_bar = [&](int t) { return bar(3 * kStages + 3 + t); };
-  auto ofull_bar = [&](int t) { return bar(3 * kStages + 5 + t); };
-  const uint32_t drain_bar = bar(3 * kStages + 7);
+  // K of a stage is free once both S GEMMs of its tile are done, V only after both PV GEMMs:
+  // separate barriers let the producer refill K about one softmax earlier.
+  auto emptyk_bar = [&](int s) { return bar(2 * kStages + s); };
+  auto emptyv_bar = [&](int s) { return bar(4 * kStages + 9 + s); };
+  // V of a tile that reaches past the sequence lands on v_load (waited on by the producer
+  // only); the producer zeroes the tail rows and then arrives on full_v itself, so the MMA
+  // issuer always waits on full_v, once per use of the stage.
+  auto vload_bar = [&](int s) { return bar(3 * kStages + s); };
+  auto sfull_bar = [&](int t) { return bar(4 * kStages + t); };
+  auto pfull_bar = [&](int t) { return bar(4 * kStages + 2 + t); };
+  auto ofull_bar = [&](int t) { return bar(4 * kStages + 4 + t); };
+  const uint32_t drain_bar = bar(4 * kStages + 6);
+  auto qready_bar = [&](int t) { return bar(4 * kStages + 7 + t); };
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffAbort);
+  WalkConst* wc_s = reinterpret_cast<WalkConst*>(smem + kOffSched);
+  Seg* my_seg = reinterpret_cast<Seg*>(smem + kOffSched + 64) + warp;   // this warp's schedule slot
+  static_assert(64 + (kThreads / 32) * sizeof(Seg) <= kSchedBytes, "schedule area");
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(fullk_bar(s), 1);
       mbar_init(fullv_bar(s), 1);
-      mbar_init(empty_bar(s), 1);
+      mbar_init(emptyk_bar(s), 1);
+      mbar_init(emptyv_bar(s), 1);
+      mbar_init(vload_bar(s), 1);
     }
-    mbar_init(vzero_bar, 1);
     for (int t = 0; t < 2; ++t) {
       mbar_init(sfull_bar(t), 1);
-      mbar_init(pfull_bar(t), 4);   // one arrival per softmax warp
+      mbar_init(pfull_bar(t), 4);    // one arrival per softmax warp
       mbar_init(ofull_bar(t), 1);
+      mbar_init(qready_bar(t), 4);   // one arrival per softmax warp
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
+    make_walk_const(p, *wc_s);
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -158,103 +335,44 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_relinquish();
     tc_fence_before();
   }
-
-  // ---- tree: validate and build ancestor masks (scratch in the last ring slot)
-  int* par_s = reinterpret_cast<int*>(smem + kOffScratch);
-  uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + kOffScratch + 512);
-  bool bad = false;
-  if (threadIdx.x < T) {
-    const int pp = p.parents[node0 + threadIdx.x];
-    par_s[threadIdx.x] = pp;
-    bad = threadIdx.x == 0 ? (pp != -1) : (pp < 0 || pp >= (int)threadIdx.x);
-  }
-  const int invalid = __syncthreads_or(bad);
-  if (!invalid && threadIdx.x < T) {
-    uint32_t m0 = 0, m1 = 0, m2 = 0, m3 = 0;
-    for (int a = threadIdx.x; a >= 0; a = par_s[a]) {   // parents strictly decrease
-      const uint32_t bit = 1u << (a & 31);
-      const int w = a >> 5;
-      m0 |= w == 0 ? bit : 0u;
-      m1 |= w == 1 ? bit : 0u;
-      m2 |= w == 2 ? bit : 0u;
-      m3 |= w == 3 ? bit : 0u;
-    }
-    anc_s[threadIdx.x * 4 + 0] = m0;
-    anc_s[threadIdx.x * 4 + 1] = m1;
-    anc_s[threadIdx.x * 4 + 2] = m2;
-    anc_s[threadIdx.x * 4 + 3] = m3;
-  }
   __syncthreads();
-
-  // ---- softmax-thread identity, ancestor mask and Q row
-  const bool is_sm = warp >= 2;
-  const int t = is_sm ? (warp - 2) >> 2 : 0;
-  const int row = (warp & 3) * 32 + lane;   // = TMEM lane this warp may access
-  const int grow = (2 * mp + t) * 128 + row;
-  const int node = grow / G;
-  const int g = grow - node * G;
-  const bool active_t = is_sm && t < nt;
-  const bool row_valid = active_t && node < T;
-  uint32_t am0 = 0, am1 = 0, am2 = 0, am3 = 0;
-  if (row_valid && !invalid) {
-    am0 = anc_s[node * 4 + 0];
-    am1 = anc_s[node * 4 + 1];
-    am2 = anc_s[node * 4 + 2];
-    am3 = anc_s[node * 4 + 3];
-  }
-  const size_t qo_row = row_valid ? ((((size_t)lq * p.n_total + node0 + node) * p.hq + (size_t)hkv * G + g) * 128)
-                                  : 0;
-  if (active_t && !invalid) {
-    const uint32_t qrow = base + kOffQ + (uint32_t)t * kTileBytes + (uint32_t)row * 128u;
-    const uint4* src = reinterpret_cast<const uint4*>(p.q) + qo_row / 8;
-#pragma unroll
-    for (int c = 0; c < 16; ++c) {
-      uint4 v = make_uint4(0, 0, 0, 0);
-      if (row_valid) v = __ldg(src + c);
-      const int half = c >> 3, j = c & 7;
-      st_shared_v4(qrow + (uint32_t)half * kHalfBytes + (uint32_t)((j ^ (row & 7)) << 4), v.x, v.y, v.z, v.w);
-    }
-  }
-  fence_proxy_async_smem();
-  __syncthreads();   // Q visible to the tensor core; the scratch slot is free again
   tc_fence_after();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffTmemPtr);
+  const WalkConst& wc = *wc_s;
+  int cursor = kWalkStart;   // this warp's position in the schedule (lane 0 walks, the warp reads)
+  volatile Seg* sgv = my_seg;
+  auto advance = [&]() -> bool {
+    __syncwarp();
+    if (lane == 0) next_segment(p, wc, cursor, *my_seg);
+    __syncwarp();
+    return sgv->valid != 0;
+  };
 
-  const size_t part_base = ((size_t)unit * p.splits + split) * 256;   // pair-local row base
-
-  if (invalid) {
-    // A malformed parent array: define the outputs as zero and report it.
-    if (threadIdx.x == 0) atomicMax(p.dev_status, (int)PTD_ERR_INVALID_TREE);
-    if (row_valid) {
-      if (p.splits == 1) {
-        uint4* dst = reinterpret_cast<uint4*>(p.out) + qo_row / 8;
-        for (int c = 0; c < 16; ++c) dst[c] = make_uint4(0, 0, 0, 0);
-      } else {
-        const size_t pr = part_base + (size_t)t * 128 + row;
-        p.part_ml[pr * 2 + 0] = -INFINITY;
-        p.part_ml[pr * 2 + 1] = 0.f;
-      }
-    }
-  } else if (warp == 0) {
+  if (warp == 0) {
     // ================================================================ TMA producer
-    if (n_local > 0) {
-      if (lane == 0) {
-        prefetch_tensormap(&map_k);
-        prefetch_tensormap(&map_v);
-      }
-      bool ok = true;
-      int jj = 0;
-      for (; jj < n_local && ok; ++jj) {
-        const int t0 = (kt_begin + jj) * 128;
-        const int st = jj % kStages;
-        const uint32_t ph = (uint32_t)((jj / kStages) & 1);
+    if (lane == 0) {
+      prefetch_tensormap(&map_k);
+      prefetch_tensormap(&map_v);
+    }
+    bool ok = true;
+    int gt = 0;                    // key tiles issued by this CTA (ring position)
+    int vloads[kStages] = {0, 0};  // v_load completions per stage (waited on here only)
+    while (ok && advance()) {
+      const int layer = p.layer_begin + sgv->lq;
+      const int b = sgv->b, hkv = sgv->hkv, N = sgv->N;
+      const int kt_end = sgv->kt_end;
+      for (int kt = sgv->kt_begin; kt < kt_end && ok; ++kt, ++gt) {
+        const int t0 = kt * 128;
+        const int st = gt % kStages;
+        const uint32_t ph = (uint32_t)((gt / kStages) & 1);
+        const bool zero_tail = t0 + 128 > N;
         if (lane == 0) {
-          ok = mbar_wait(empty_bar(st), ph ^ 1u, abort_flag, p.dev_status);
-          if (ok) {
-            const uint32_t dst = base + kOffRing + (uint32_t)st * kStageBytes;
-            for (int which = 0; which < 2; ++which) {
+          const uint32_t dst = base + kOffRing + (uint32_t)st * kStageBytes;
+          for (int which = 0; which < 2 && ok; ++which) {
+            ok = mbar_wait(which ? emptyv_bar(st) : emptyk_bar(st), ph ^ 1u, abort_flag, p.dev_status);
+            if (ok) {
               const CUtensorMap* map = which ? &map_v : &map_k;
-              const uint32_t fb = which ? fullv_bar(st) : fullk_bar(st);
+              const uint32_t fb = which ? (zero_tail ? vload_bar(st) : fullv_bar(st)) : fullk_bar(st);
               const uint32_t d = dst + (uint32_t)which * kTileBytes;
               if (!kPaged) {
                 const int row0 = (layer * p.batch + b) * p.seq_capacity + t0;
@@ -279,9 +397,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-        if (ok && t0 + 128 > N) {
+        if (ok && zero_tail) {
           // V rows past the sequence: zero them so that P = 0 never meets a non-finite value
-          if ((ok = mbar_wait_warp(fullv_bar(st), ph, abort_flag, p.dev_status))) {
+          ok = mbar_wait_warp(vload_bar(st), (uint32_t)(vloads[st] & 1), abort_flag, p.dev_status);
+          vloads[st] += 1;
+          if (ok) {
             const uint32_t vbase = base + kOffRing + (uint32_t)st * kStageBytes + kTileBytes;
             const int r0 = N - t0;
             for (int c = lane; c < (128 - r0) * 16; c += 32) {
@@ -291,248 +411,490 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(vzero_bar);
+            if (lane == 0) mbar_arrive(fullv_bar(st));
           }
         }
       }
-      if (!ok && lane == 0) {
-        // drain the copies already issued (bounded) before the CTA can exit
-        for (int back = 1; back <= kStages && jj - back >= 0; ++back) {
-          const int j2 = jj - back;
-          mbar_drain(fullk_bar(j2 % kStages), (uint32_t)((j2 / kStages) & 1), 100000000ull);
-          mbar_drain(fullv_bar(j2 % kStages), (uint32_t)((j2 / kStages) & 1), 100000000ull);
-        }
+    }
+    if (!ok && lane == 0) {
+      // drain the copies already issued (bounded) before the CTA can exit
+      for (int back = 1; back <= kStages && gt - back >= 0; ++back) {
+        const int j2 = gt - back;
+        mbar_drain(fullk_bar(j2 % kStages), (uint32_t)((j2 / kStages) & 1), 100000000ull);
+        mbar_drain(fullv_bar(j2 % kStages), (uint32_t)((j2 / kStages) & 1), 100000000ull);
+        mbar_drain(vload_bar(j2 % kStages), (uint32_t)((vloads[j2 % kStages] + 1) & 1), 100000000ull);
       }
     }
   } else if (warp == 1) {
     // ================================================================ MMA issuer (one thread)
-    if (n_local > 0 && lane == 0) {
-      const uint32_t q_base = base + kOffQ, ring = base + kOffRing;
-      auto issue_s = [&](int tt, int st) {
-        const uint32_t d = tmem + (uint32_t)tt * 128u;
+    const uint32_t q_base = base + kOffQ, ring = base + kOffRing;
+    auto issue_s = [&](int tt, int st) {
+      const uint32_t d = tmem + (uint32_t)tt * 128u;
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t koff = (uint32_t)(kk >> 2) * kHalfBytes + (uint32_t)(kk & 3) * 32u;
-          const uint64_t a = smem_desc_sw128(q_base + (uint32_t)tt * kTileBytes + koff, 16, 1024);
-          const uint64_t bd = smem_desc_sw128(ring + (uint32_t)st * kStageBytes + koff, 16, 1024);
-          mma_bf16_ss(d, a, bd, kIdescS, kk > 0 ? 1u : 0u);
-        }
-      };
-      auto issue_pv = [&](int tt, int st, bool acc) {
-        const uint32_t d = tmem + 256u + (uint32_t)tt * 128u;
-        const uint32_t a = tmem + (uint32_t)tt * 128u;   // P: 16 keys = 8 packed columns per step
-        const uint32_t vb = ring + (uint32_t)st * kStageBytes + kTileBytes;
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t koff = (uint32_t)(kk >> 2) * kHalfBytes + (uint32_t)(kk & 3) * 32u;
+        const uint64_t a = smem_desc_sw128(q_base + (uint32_t)tt * kTileBytes + koff, 16, 1024);
+        const uint64_t bd = smem_desc_sw128(ring + (uint32_t)st * kStageBytes + koff, 16, 1024);
+        mma_bf16_ss(d, a, bd, kIdescS, kk > 0 ? 1u : 0u);
+      }
+    };
+    auto issue_pv = [&](int tt, int st, bool acc) {
+      const uint32_t d = tmem + 256u + (uint32_t)tt * 128u;
+      const uint32_t a = tmem + (uint32_t)tt * 128u;   // P: 16 keys = 8 packed columns per step
+      const uint32_t vb = ring + (uint32_t)st * kStageBytes + kTileBytes;
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t bd = smem_desc_sw128(vb + (uint32_t)kk * 2048u, kHalfBytes, 1024);
-          mma_bf16_ts(d, a + (uint32_t)kk * 8u, bd, kIdescPV, (acc || kk > 0) ? 1u : 0u);
-        }
-      };
-      bool ok = mbar_wait(fullk_bar(0), 0, abort_flag, p.dev_status);
-      tc_fence_after();
-      if (ok) {
-        issue_s(0, 0);
-        mma_commit(sfull_bar(0));
-        if (nt == 2) {
-          issue_s(1, 0);
-          mma_commit(sfull_bar(1));
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t bd = smem_desc_sw128(vb + (uint32_t)kk * 2048u, kHalfBytes, 1024);
+        mma_bf16_ts(d, a + (uint32_t)kk * 8u, bd, kIdescPV, (acc || kk > 0) ? 1u : 0u);
+      }
+    };
+    bool ok = true;
+    int gt = 0;
+    int tiles_t[2] = {0, 0}, segs_t[2] = {0, 0};
+    // The whole warp walks the schedule together; lane 0 issues, and its status is
+    // broadcast after every segment so that no lane is left waiting on the others.
+    while (ok && advance()) {
+      if (lane == 0) {
+        const int n = sgv->kt_end - sgv->kt_begin;
+        const int nt = sgv->nt;
+        if (n > 0) {
+          // Q of this segment is in shared memory
+          for (int t = 0; t < nt && ok; ++t)
+            ok = mbar_wait(qready_bar(t), (uint32_t)(segs_t[t] & 1), abort_flag, p.dev_status);
+          if (ok) ok = mbar_wait(fullk_bar(gt % kStages), (uint32_t)((gt / kStages) & 1), abort_flag, p.dev_status);
+          if (ok) {
+            tc_fence_after();
+            issue_s(0, gt % kStages);
+            mma_commit(sfull_bar(0));
+            if (nt == 2) {
+              issue_s(1, gt % kStages);
+              mma_commit(sfull_bar(1));
+            }
+            mma_commit(emptyk_bar(gt % kStages));   // K of this tile is no longer read
+          }
+          for (int jj = 0; jj < n && ok; ++jj, ++gt) {
+            const int st = gt % kStages;
+            const uint32_t ph = (uint32_t)((gt / kStages) & 1);
+            if (!(ok = mbar_wait(fullv_bar(st), ph, abort_flag, p.dev_status))) break;
+            if (!(ok = mbar_wait(pfull_bar(0), (uint32_t)(tiles_t[0] & 1), abort_flag, p.dev_status))) break;
+            tc_fence_after();
+            issue_pv(0, st, jj > 0);
+            const bool more = jj + 1 < n;
+            const int st1 = (gt + 1) % kStages;
+            if (more) {
+              if (!(ok = mbar_wait(fullk_bar(st1), (uint32_t)(((gt + 1) / kStages) & 1), abort_flag,
+                                   p.dev_status)))
+                break;
+              tc_fence_after();
+              issue_s(0, st1);
+              mma_commit(sfull_bar(0));
+              if (nt == 1) mma_commit(emptyk_bar(st1));
+            }
+            if (nt == 2) {
+              if (!(ok = mbar_wait(pfull_bar(1), (uint32_t)(tiles_t[1] & 1), abort_flag, p.dev_status))) break;
+              tc_fence_after();
+              issue_pv(1, st, jj > 0);
+            }
+            mma_commit(emptyv_bar(st));   // V of this stage is no longer read
+            if (more && nt == 2) {
+              issue_s(1, st1);
+              mma_commit(sfull_bar(1));
+              mma_commit(emptyk_bar(st1));
+            }
+            ++tiles_t[0];
+            if (nt == 2) ++tiles_t[1];
+          }
+          if (ok) {
+            mma_commit(ofull_bar(0));
+            ++segs_t[0];
+            if (nt == 2) {
+              mma_commit(ofull_bar(1));
+              ++segs_t[1];
+            }
+          }
         }
       }
-      for (int jj = 0; jj < n_local && ok; ++jj) {
-        const int st = jj % kStages;
-        const uint32_t ph = (uint32_t)((jj / kStages) & 1);
-        const int t0 = (kt_begin + jj) * 128;
-        // V of this tile (zeroed past the sequence by the producer warp on the last tile)
-        if (!(ok = (t0 + 128 > N) ? mbar_wait(vzero_bar, 0, abort_flag, p.dev_status)
-                                  : mbar_wait(fullv_bar(st), ph, abort_flag, p.dev_status)))
-          break;
-        if (!(ok = mbar_wait(pfull_bar(0), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
-        tc_fence_after();
-        issue_pv(0, st, jj > 0);
-        const bool more = jj + 1 < n_local;
-        const int st1 = (jj + 1) % kStages;
-        if (more) {
-          if (!(ok = mbar_wait(fullk_bar(st1), (uint32_t)(((jj + 1) / kStages) & 1), abort_flag, p.dev_status)))
-            break;
-          tc_fence_after();
-          issue_s(0, st1);
-          mma_commit(sfull_bar(0));
-        }
-        if (nt == 2) {
-          if (!(ok = mbar_wait(pfull_bar(1), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
-          tc_fence_after();
-          issue_pv(1, st, jj > 0);
-        }
-        mma_commit(empty_bar(st));   // K and V of this stage are no longer read
-        if (more && nt == 2) {
-          issue_s(1, st1);
-          mma_commit(sfull_bar(1));
-        }
-      }
-      mma_commit(ofull_bar(0));
-      if (nt == 2) mma_commit(ofull_bar(1));
-      if (!ok) {
-        // error path: let the tensor core finish what was issued before TMEM is freed
-        mma_commit(drain_bar);
-        mbar_drain(drain_bar, 0, 100000000ull);
-      }
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
     }
-  } else if (active_t) {
+    if (lane == 0 && !ok) {
+      // error path: let the tensor core finish what was issued before TMEM is freed
+      mma_commit(drain_bar);
+      mbar_drain(drain_bar, 0, 100000000ull);
+    }
+  } else {
     // ================================================================ softmax / epilogue
+    const int t = (warp - 2) >> 2;
+    const int row = (warp & 3) * 32 + lane;   // = TMEM lane this warp may access
     const float sl2 = p.scale_log2;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     const uint32_t tS = tmem + lane_base + (uint32_t)t * 128u;
     const uint32_t tO = tmem + lane_base + 256u + (uint32_t)t * 128u;
     const unsigned long long sl2x2 = f2_pack(sl2, sl2);
-    // Reference max m_run (log2 units) against which P = 2^(s*scale*log2e - m_run) is taken.
-    // It only moves up, and only when a 32-column chunk exceeds it by more than 2^8; then the
-    // row sum, O and the P chunks already written for this tile are rescaled (rare).
-    float m_run = -INFINITY, l_run = 0.f;
+    const uint32_t qrow_smem = base + kOffQ + (uint32_t)t * kTileBytes + (uint32_t)row * 128u;
+    WarpArea* wa = reinterpret_cast<WarpArea*>(smem + kOffWarp) + (warp - 2);
+    volatile WarpArea* wv = wa;
+    if (lane == 0) {
+      wa->tree_node0 = -1;
+      wa->tree_T = -1;
+      wa->mask_mp = -1;
+      wa->ndefer = 0;
+    }
+    __syncwarp();
+    uint32_t am0 = 0, am1 = 0, am2 = 0, am3 = 0;   // ancestor mask of this row's node
+    int tiles = 0, segs = 0;
     bool ok = true;
     uint32_t r[32];
-    for (int jj = 0; jj < n_local; ++jj) {
-      if (!(ok = mbar_wait_warp(sfull_bar(t), (uint32_t)(jj & 1), abort_flag, p.dev_status))) break;
-      tc_fence_after();
-      const int t0 = (kt_begin + jj) * 128;
-      const bool need_mask = t0 + 128 > C;   // warp-uniform
-      unsigned long long sum = f2_pack(0.f, 0.f);
-#pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
-        tmem_ld32(tS + (uint32_t)c * 32u, r);
-        tmem_ld_wait();
-        if (need_mask) {
-          const uint32_t vw = vis_word(t0 + c * 32 - C, am0, am1, am2, am3);
-#pragma unroll
-          for (int e = 0; e < 32; ++e) r[e] = ((vw >> e) & 1u) ? r[e] : __float_as_uint(-INFINITY);
-        }
-        float cm;
-        {
-          float a0 = -INFINITY, a1 = -INFINITY;
-#pragma unroll
-          for (int e = 0; e < 32; e += 4) {
-            a0 = fmax3(a0, __uint_as_float(r[e]), __uint_as_float(r[e + 1]));
-            a1 = fmax3(a1, __uint_as_float(r[e + 2]), __uint_as_float(r[e + 3]));
-          }
-          cm = fmaxf(a0, a1) * sl2;
-        }
-        // The TMEM accesses of a rescale are warp-collective, so the whole warp takes the
-        // branch when any of its rows needs it; the other rows rescale by exactly 1.  (Rows
-        // differ when a split starts on a key tile past the committed context: each row
-        // first meets a visible ancestor in whichever chunk holds one.)
-        const bool raise = cm > m_run + kRescaleLog2;
-        if (__any_sync(0xffffffffu, raise)) {
-          // raise the reference: rescale everything taken against the old one
-          float alpha = 1.f;
-          if (raise) {
-            alpha = m_run == -INFINITY ? 0.f : ptx_exp2(m_run - cm);
-            m_run = cm;
-          }
-          float s0, s1;
-          f2_unpack(sum, s0, s1);
-          sum = f2_pack(s0 * alpha, s1 * alpha);
-          l_run *= alpha;
-          if (jj > 0) {
-            // O_t is idle here: PV_t of the previous tile completed before S_t of this one
-#pragma unroll 1
-            for (int q = 0; q < 8; ++q) {
-              uint32_t o16[16];
-              tmem_ld16(tO + (uint32_t)q * 16u, o16);
-              tmem_ld_wait();
-#pragma unroll
-              for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
-              tmem_st16(tO + (uint32_t)q * 16u, o16);
-            }
-          }
-          if (c > 0) {
-            tmem_st_wait();
-#pragma unroll 1
-            for (int q = 0; q < c; ++q) {   // bf16 P of the earlier chunks of this tile
-              uint32_t p16[16];
-              tmem_ld16(tS + (uint32_t)q * 16u, p16);
-              tmem_ld_wait();
-#pragma unroll
-              for (int e = 0; e < 16; ++e)
-                p16[e] = pack_bf16x2(__uint_as_float(p16[e] << 16) * alpha,
-                                     __uint_as_float(p16[e] & 0xFFFF0000u) * alpha);
-              tmem_st16(tS + (uint32_t)q * 16u, p16);
-            }
-          }
-        }
-        const float m_use = m_run == -INFINITY ? 0.f : m_run;   // -inf only when nothing is visible yet
-        const unsigned long long negm = f2_pack(-m_use, -m_use);
-        uint32_t pk[16];
-#pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          const unsigned long long x =
-              f2_fma(f2_pack(__uint_as_float(r[e]), __uint_as_float(r[e + 1])), sl2x2, negm);
-          float x0, x1;
-          f2_unpack(x, x0, x1);
-          const float p0 = ptx_exp2(x0), p1 = ptx_exp2(x1);
-          sum = f2_add(sum, f2_pack(p0, p1));
-          pk[e >> 1] = pack_bf16x2(p0, p1);
-        }
-        tmem_st16(tS + (uint32_t)c * 16u, pk);   // P chunk c: columns [16c, 16c+16) of S_t
-      }
+
+    // Next segment of the range that has rows in this warp's M tile.
+    auto next_mine = [&]() -> bool {
+      while (advance())
+        if (t < sgv->nt) return true;
+      return false;
+    };
+    // Takes the segment just walked to as run slot k: tree check and ancestor masks (the
+    // parents of the last tree seen are kept in shared memory), Q rows, q_ready.
+    auto prepare = [&](int k) {
+      const int T = sgv->T, node0 = sgv->node0, mp = sgv->mp;
+      const int grow = (2 * mp + t) * 128 + row;
+      const int node = grow / G, g = grow - node * G;
+      const bool row_valid = node < T;
+      const bool has_keys = sgv->kt_end > sgv->kt_begin;
+      // Q rows first: their loads overlap the tree work below
+      uint4 v[16];
       {
-        float s0, s1;
-        f2_unpack(sum, s0, s1);
-        l_run += s0 + s1;
-      }
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(pfull_bar(t));
-    }
-    // ---- epilogue
-    ok = __all_sync(0xffffffffu, ok);
-    if (ok && n_local > 0) ok = mbar_wait_warp(ofull_bar(t), 0, abort_flag, p.dev_status);
-    tc_fence_after();
-    const bool have_o = ok && n_local > 0;
-    if (p.splits == 1) {
-      const float inv = (have_o && l_run > 0.f) ? 1.f / l_run : 0.f;
-      uint4* dst = reinterpret_cast<uint4*>(p.out) + qo_row / 8;
+        const size_t orow = (((size_t)sgv->lq * p.n_total + node0 + node) * p.hq + (size_t)sgv->hkv * G + g) * 128;
+        const uint4* srcq = reinterpret_cast<const uint4*>(p.q) + (row_valid ? orow : 0) / 8;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        if (have_o) {
-          tmem_ld32(tO + (uint32_t)c * 32u, r);
-          tmem_ld_wait();
+        for (int c = 0; c < 16; ++c) v[c] = (row_valid && has_keys) ? __ldg(srcq + c) : make_uint4(0, 0, 0, 0);
+      }
+      if (node0 != wv->tree_node0 || T != wv->tree_T) {
+        // tree validity (parents[0] = -1, 0 <= parents[i] < i), checked by every warp on its own
+        bool bad = false;
+        for (int i = lane; i < T; i += 32) {
+          const int pp = __ldg(p.parents + node0 + i);
+          wv->parents[i] = pp;
+          bad = bad || (i == 0 ? (pp != -1) : (pp < 0 || pp >= i));
+        }
+        const bool invalid = __any_sync(0xffffffffu, bad);
+        __syncwarp();
+        if (lane == 0) {
+          wa->tree_node0 = node0;
+          wa->tree_T = T;
+          wa->tree_invalid = invalid ? 1 : 0;
+          wa->mask_mp = -1;
+        }
+        __syncwarp();
+      }
+      const bool invalid = wv->tree_invalid != 0;
+      if (mp != wv->mask_mp) {
+        // ancestor bitmask of this row's node (walk up the parent pointers, strictly decreasing)
+        am0 = am1 = am2 = am3 = 0;
+        if (row_valid && !invalid) {
+          for (int q = node; q >= 0; q = wv->parents[q]) {
+            const uint32_t bit = 1u << (q & 31);
+            const int w = q >> 5;
+            am0 |= w == 0 ? bit : 0u;
+            am1 |= w == 1 ? bit : 0u;
+            am2 |= w == 2 ? bit : 0u;
+            am3 |= w == 3 ? bit : 0u;
+          }
+        }
+        __syncwarp();
+        if (lane == 0) wa->mask_mp = mp;
+      }
+      // keep the segment for the epilogue (the walker's slot moves on before it runs)
+      constexpr int kSegWords = (int)(sizeof(Seg) / 4);
+      if (lane < kSegWords)
+        reinterpret_cast<volatile int*>(&wa->run[k].s)[lane] = reinterpret_cast<const volatile int*>(sgv)[lane];
+      if (lane == 0) wa->run[k].invalid = invalid ? 1 : 0;
+      if (has_keys) {
+        // Q rows of this segment (every S_t GEMM of the previous segment has completed)
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+          const int half = c >> 3, j = c & 7;
+          const uint4 q4 = invalid ? make_uint4(0, 0, 0, 0) : v[c];
+          st_shared_v4(qrow_smem + (uint32_t)half * kHalfBytes + (uint32_t)((j ^ (row & 7)) << 4), q4.x, q4.y,
+                       q4.z, q4.w);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(qready_bar(t));
+      }
+      __syncwarp();
+    };
+
+    // Output rows of one 32-row block from the partials of all pieces of its unit:
+    // O = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c (pieces with l_c = 0 saw no key).
+    auto merge = [&](const volatile SegRun* rec) {
+      const int ug0 = rec->s.ug0, ug1 = ug0 + rec->s.n_kt;
+      const int T = rec->s.T, mp = rec->s.mp;
+      const bool invalid = rec->invalid != 0;
+      const int grow = (2 * mp + t) * 128 + row;
+      const int node = grow / G, g = grow - node * G;
+      const bool row_valid = node < T;
+      const int first = owner_cta(wc, ug0), last = owner_cta(wc, ug1 - 1);
+      const float2* pml = reinterpret_cast<const float2*>(p.part_ml) + (size_t)t * 128 + row;
+      auto owns = [&](int c) { return c <= last && range_start(wc, c + 1) > range_start(wc, c); };
+      float M = -INFINITY, L = 0.f;
+      auto fold = [&](float2 ml) {
+        if (ml.y > 0.f) {
+          if (ml.x > M) {
+            L = L * ptx_exp2(M - ml.x) + ml.y;
+            M = ml.x;
+          } else {
+            L += ml.y * ptx_exp2(ml.x - M);
+          }
+        }
+      };
+      for (int c = first; c <= last; c += 2) {   // two pieces' (m, l) loads at a time
+        const bool h0 = owns(c), h1 = owns(c + 1);
+        const float2 a0 = h0 ? __ldcg(pml + (size_t)piece_slot(wc, c, ug0, ug1) * 256) : make_float2(-INFINITY, 0.f);
+        const float2 a1 = h1 ? __ldcg(pml + (size_t)piece_slot(wc, c + 1, ug0, ug1) * 256) : make_float2(-INFINITY, 0.f);
+        fold(a0);
+        fold(a1);
+      }
+      const float inv = (L > 0.f && !invalid) ? 1.f / L : 0.f;
+      const size_t orow = (((size_t)rec->s.lq * p.n_total + rec->s.node0 + node) * p.hq + (size_t)rec->s.hkv * G + g) * 128;
+      uint4* dst = reinterpret_cast<uint4*>(p.out) + (row_valid ? orow : 0) / 8;
+#pragma unroll 1
+      for (int h = 0; h < 4; ++h) {   // 32 output columns at a time
+        float acc[32];
+#pragma unroll
+        for (int d = 0; d < 32; ++d) acc[d] = 0.f;
+        for (int c = first; c <= last; ++c) {
+          if (!owns(c)) continue;
+          const size_t q = (size_t)piece_slot(wc, c, ug0, ug1);
+          const float2 ml = __ldcg(pml + q * 256);
+          const float* po = p.part_o + (q * 2 + t) * (128 * 128) + (size_t)(h * 32) * 128 + row;
+          float o[32];
+#pragma unroll
+          for (int d = 0; d < 32; ++d) o[d] = __ldcg(po + (size_t)d * 128);
+          // rows of a piece that saw no key were not written: weight 0 and never read into acc
+          const float wgt = ml.y > 0.f ? ptx_exp2(ml.x - M) : 0.f;
+#pragma unroll
+          for (int d = 0; d < 32; ++d) acc[d] = wgt > 0.f ? fmaf(wgt, o[d], acc[d]) : acc[d];
         }
         if (row_valid) {
 #pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4) {
+          for (int c8 = 0; c8 < 4; ++c8) {
             uint32_t w[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float a0 = have_o ? __uint_as_float(r[q4 * 8 + 2 * e]) * inv : 0.f;
-              const float a1 = have_o ? __uint_as_float(r[q4 * 8 + 2 * e + 1]) * inv : 0.f;
-              w[e] = pack_bf16x2(a0, a1);
-            }
-            dst[c * 4 + q4] = make_uint4(w[0], w[1], w[2], w[3]);
+            for (int e = 0; e < 4; ++e) w[e] = pack_bf16x2(acc[c8 * 8 + 2 * e] * inv, acc[c8 * 8 + 2 * e + 1] * inv);
+            dst[h * 4 + c8] = make_uint4(w[0], w[1], w[2], w[3]);
           }
         }
       }
-    } else {
-      const size_t pr = part_base + (size_t)t * 128 + row;
-      float4* po = reinterpret_cast<float4*>(p.part_o + pr * 128);
+    };
+
+    bool have = next_mine();
+    int k = 0;   // run slot of the current segment
+    if (have) prepare(0);
+    while (have) {
+      const volatile SegRun* cur = &wv->run[k];
+      const int kt_begin = cur->s.kt_begin;
+      const int C = cur->s.C;
+      const int n = cur->s.kt_end - kt_begin;
+      // Reference max m_run (log2 units) against which P = 2^(s*scale*log2e - m_run) is
+      // taken.  It only moves up, and only when a 32-column chunk exceeds it by more than
+      // 2^8; then the row sum, O and the P chunks already written for this tile are rescaled.
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int jj = 0; jj < n; ++jj, ++tiles) {
+        if (!(ok = mbar_wait_warp(sfull_bar(t), (uint32_t)(tiles & 1), abort_flag, p.dev_status))) break;
+        tc_fence_after();
+        const int t0 = (kt_begin + jj) * 128;
+        const bool need_mask = t0 + 128 > C;   // warp-uniform
+        unsigned long long sum = f2_pack(0.f, 0.f);
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          tmem_ld32(tS + (uint32_t)c * 32u, r);
+          tmem_ld_wait();
+          if (need_mask) {
+            const uint32_t vw = vis_word(t0 + c * 32 - C, am0, am1, am2, am3);
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        if (have_o) {
+            for (int e = 0; e < 32; ++e) r[e] = ((vw >> e) & 1u) ? r[e] : __float_as_uint(-INFINITY);
+          }
+          float cm;
+          {
+            float a0 = -INFINITY, a1 = -INFINITY;
+#pragma unroll
+            for (int e = 0; e < 32; e += 4) {
+              a0 = fmax3(a0, __uint_as_float(r[e]), __uint_as_float(r[e + 1]));
+              a1 = fmax3(a1, __uint_as_float(r[e + 2]), __uint_as_float(r[e + 3]));
+            }
+            cm = fmaxf(a0, a1) * sl2;
+          }
+          // The TMEM accesses of a rescale are warp-collective, so the whole warp takes the
+          // branch when any of its rows needs it; the other rows rescale by exactly 1.  (Rows
+          // differ when a piece starts on a key tile past the committed context: each row
+          // first meets a visible ancestor in whichever chunk holds one.)
+          const bool raise = cm > m_run + kRescaleLog2;
+          if (__any_sync(0xffffffffu, raise)) {
+            // raise the reference: rescale everything taken against the old one
+            float alpha = 1.f;
+            if (raise) {
+              alpha = m_run == -INFINITY ? 0.f : ptx_exp2(m_run - cm);
+              m_run = cm;
+            }
+            float s0, s1;
+            f2_unpack(sum, s0, s1);
+            sum = f2_pack(s0 * alpha, s1 * alpha);
+            l_run *= alpha;
+            if (jj > 0) {
+              // O_t is idle here: PV_t of the previous tile completed before S_t of this one
+#pragma unroll 1
+              for (int q = 0; q < 8; ++q) {
+                uint32_t o16[16];
+                tmem_ld16(tO + (uint32_t)q * 16u, o16);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
+                tmem_st16(tO + (uint32_t)q * 16u, o16);
+              }
+            }
+            if (c > 0) {
+              tmem_st_wait();
+#pragma unroll 1
+              for (int q = 0; q < c; ++q) {   // bf16 P of the earlier chunks of this tile
+                uint32_t p16[16];
+                tmem_ld16(tS + (uint32_t)q * 16u, p16);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                  p16[e] = pack_bf16x2(__uint_as_float(p16[e] << 16) * alpha,
+                                       __uint_as_float(p16[e] & 0xFFFF0000u) * alpha);
+                tmem_st16(tS + (uint32_t)q * 16u, p16);
+              }
+            }
+          }
+          const float m_use = m_run == -INFINITY ? 0.f : m_run;   // -inf only while nothing is visible
+          const unsigned long long negm = f2_pack(-m_use, -m_use);
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            const unsigned long long x =
+                f2_fma(f2_pack(__uint_as_float(r[e]), __uint_as_float(r[e + 1])), sl2x2, negm);
+            float x0, x1;
+            f2_unpack(x, x0, x1);
+            const float p0 = ptx_exp2(x0), p1 = ptx_exp2(x1);
+            sum = f2_add(sum, f2_pack(p0, p1));
+            pk[e >> 1] = pack_bf16x2(p0, p1);
+          }
+          tmem_st16(tS + (uint32_t)c * 16u, pk);   // P chunk c: columns [16c, 16c+16) of S_t
+        }
+        {
+          float s0, s1;
+          f2_unpack(sum, s0, s1);
+          l_run += s0 + s1;
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pfull_bar(t));
+      }
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      // Every S_t GEMM of this segment has completed (its last s_full was seen), so the next
+      // segment's Q can go in now: the tensor core starts on it while this epilogue runs.
+      const bool have_next = next_mine();
+      if (have_next) prepare(k ^ 1);
+      // ---- epilogue of the segment
+      if (n > 0) {
+        if (!(ok = mbar_wait_warp(ofull_bar(t), (uint32_t)(segs & 1), abort_flag, p.dev_status))) break;
+        ++segs;
+        tc_fence_after();
+      }
+      const bool invalid = cur->invalid != 0;
+      const bool have_o = n > 0 && !invalid;
+      if (invalid && lane == 0) atomicMax(p.dev_status, (int)PTD_ERR_INVALID_TREE);
+      const int slot = cur->s.slot;
+      if (slot < 0) {
+        // the whole unit: normalised bf16 output
+        const int T = cur->s.T;
+        const int grow = (2 * cur->s.mp + t) * 128 + row;
+        const int node = grow / G, g = grow - node * G;
+        const bool row_valid = node < T;
+        const size_t orow =
+            (((size_t)cur->s.lq * p.n_total + cur->s.node0 + node) * p.hq + (size_t)cur->s.hkv * G + g) * 128;
+        const float inv = (have_o && l_run > 0.f) ? 1.f / l_run : 0.f;
+        uint4* dst = reinterpret_cast<uint4*>(p.out) + (row_valid ? orow : 0) / 8;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          if (n > 0) {
+            tmem_ld32(tO + (uint32_t)c * 32u, r);
+            tmem_ld_wait();
+          }
+          if (row_valid) {
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+              uint32_t w[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float a0 = have_o ? __uint_as_float(r[q4 * 8 + 2 * e]) * inv : 0.f;
+                const float a1 = have_o ? __uint_as_float(r[q4 * 8 + 2 * e + 1]) * inv : 0.f;
+                w[e] = pack_bf16x2(a0, a1);
+              }
+              dst[c * 4 + q4] = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+          }
+        }
+      } else {
+        // A piece: O unnormalised, running max (log2 units) and row sum.  The partial of an
+        // M tile is column-major ([column][128 rows]), so each store of the warp is one
+        // contiguous 128-byte line.
+        float* po = p.part_o + ((size_t)slot * 2 + t) * (128 * 128) + row;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
           tmem_ld32(tO + (uint32_t)c * 32u, r);
           tmem_ld_wait();
-        }
-        if (row_valid && have_o) {
+          if (have_o) {
 #pragma unroll
-          for (int q4 = 0; q4 < 8; ++q4)
-            po[c * 8 + q4] = make_float4(__uint_as_float(r[q4 * 4 + 0]), __uint_as_float(r[q4 * 4 + 1]),
-                                         __uint_as_float(r[q4 * 4 + 2]), __uint_as_float(r[q4 * 4 + 3]));
+            for (int e = 0; e < 32; ++e) po[(size_t)(c * 32 + e) * 128] = __uint_as_float(r[e]);
+          }
+        }
+        reinterpret_cast<float2*>(p.part_ml)[(size_t)slot * 256 + (size_t)t * 128 + row] =
+            have_o ? make_float2(m_run, l_run) : make_float2(-INFINITY, 0.f);
+        // The warp that writes the last piece of this 32-row block merges the block (CTAs
+        // with an empty range own no piece), after the rest of its range: a merge waits on
+        // loads from other SMs and would stall this CTA's pipeline here.
+        const int ug0 = cur->s.ug0;
+        const int ug1 = ug0 + cur->s.n_kt;
+        const int first = owner_cta(wc, ug0);
+        const int last = owner_cta(wc, ug1 - 1);
+        __threadfence();
+        __syncwarp();
+        int is_last = 0;
+        if (lane == 0) {
+          int pieces = 0;
+          for (int c = first; c <= last; ++c) pieces += range_start(wc, c + 1) > range_start(wc, c) ? 1 : 0;
+          const int old = atomicAdd(p.counters + (size_t)cur->s.unit * 8 + t * 4 + (warp & 3), 1);
+          is_last = old == pieces - 1;
+        }
+        is_last = __shfl_sync(0xffffffffu, is_last, 0);
+        if (is_last) {
+          const int nd = wv->ndefer;
+          if (nd < kMaxDefer) {
+            constexpr int kRunWords = (int)(sizeof(SegRun) / 4);
+            if (lane < kRunWords)
+              reinterpret_cast<volatile int*>(&wa->defer[nd])[lane] = reinterpret_cast<const volatile int*>(cur)[lane];
+            __syncwarp();
+            if (lane == 0) wa->ndefer = nd + 1;
+            __syncwarp();
+          } else {
+            __threadfence();
+            merge(cur);   // not reached: a range holds at most two pieces
+          }
         }
       }
-      if (row_valid) {
-        p.part_ml[pr * 2 + 0] = have_o ? m_run : -INFINITY;
-        p.part_ml[pr * 2 + 1] = have_o ? l_run : 0.f;
-      }
+      tc_fence_before();
+      k ^= 1;
+      have = have_next;
     }
-    tc_fence_before();
+    // merges left for the end of the range
+    if (ok) {
+      const int nd = wv->ndefer;
+      if (nd > 0) __threadfence();
+      for (int d = 0; d < nd; ++d) merge(&wv->defer[d]);
+    }
   }
 
   __syncthreads();
@@ -542,61 +904,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Merge the per-split partials (O unnormalised, running max m in log2 units, sum l) of
-// every row: O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.  One warp per row.
-__global__ void __launch_bounds__(256) attn_combine_kernel(const AttnParams p) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int u = blockIdx.x;
-  const int unit = u;
-  const int mp = u % p.pairs;
-  u /= p.pairs;
-  const int hkv = u % p.hkv;
-  u /= p.hkv;
-  const int b = u % p.batch;
-  const int lq = u / p.batch;
-  const int G = p.group;
-  const int node0 = p.node_offsets[b];
-  const int T = p.node_offsets[b + 1] - node0;
-  if (T < 1 || T > p.max_nodes || node0 < 0 || node0 + T > p.n_total) return;
-  const int prow = blockIdx.y * 8 + warp;   // 0..255
-  const int grow = mp * 256 + prow;
-  const int node = grow / G, g = grow - node * G;
-  if (node >= T) return;
-  float M = -INFINITY;
-  for (int s = 0; s < p.splits; ++s) {
-    const size_t pr = ((size_t)unit * p.splits + s) * 256 + prow;
-    if (p.part_ml[pr * 2 + 1] > 0.f) M = fmaxf(M, p.part_ml[pr * 2 + 0]);
-  }
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  float L = 0.f;
-  for (int s = 0; s < p.splits; ++s) {
-    const size_t pr = ((size_t)unit * p.splits + s) * 256 + prow;
-    const float l = p.part_ml[pr * 2 + 1];
-    if (!(l > 0.f)) continue;
-    const float w = ptx_exp2(p.part_ml[pr * 2 + 0] - M);
-    L += w * l;
-    const float4 o = reinterpret_cast<const float4*>(p.part_o + pr * 128)[lane];
-    acc.x = fmaf(w, o.x, acc.x);
-    acc.y = fmaf(w, o.y, acc.y);
-    acc.z = fmaf(w, o.z, acc.z);
-    acc.w = fmaf(w, o.w, acc.w);
-  }
-  const float inv = L > 0.f ? 1.f / L : 0.f;
-  const size_t orow = (((size_t)lq * p.n_total + node0 + node) * p.hq + (size_t)hkv * G + g) * 128;
-  uint2 w2;
-  w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-  w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-  reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(p.out) + orow)[lane] = w2;
-}
-
 }  // namespace tc
 
 // ------------------------------------------------------------------- host launchers
 size_t tc_smem_bytes() { return tc::kSmemBytes; }
 
 cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const AttnParams& p,
-                                int units, cudaStream_t stream) {
-  const dim3 grid((unsigned)units, (unsigned)p.splits);
+                                dim3 grid, cudaStream_t stream) {
   if (p.page_size > 0) {
     cudaError_t e = cudaFuncSetAttribute(tc::tree_attn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)tc::kSmemBytes);
@@ -611,9 +925,5 @@ cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map
   return cudaGetLastError();
 }
 
-cudaError_t launch_attn_combine(const AttnParams& p, int units, cudaStream_t stream) {
-  tc::attn_combine_kernel<<<dim3((unsigned)units, 32), 256, 0, stream>>>(p);
-  return cudaGetLastError();
-}
 
 }  // namespace ptd

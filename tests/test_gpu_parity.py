@@ -65,7 +65,8 @@ def _run_attention(w):
 
 ATTN_CASES = {
     # name: (base config, overrides) -- sizes the oracle finishes in seconds, spanning several
-    # 128-key tiles, a ragged tail, one and two M tiles, splits and the paged layout
+    # 128-key tiles, a ragged tail, one and two M tiles, units split between CTAs, fewer key
+    # tiles than SMs, and the paged layout
     "tiny-fp32": ("tiny-fp32", {}),
     "fp32-d128-gqa": ("tiny-fp32", dict(hq=8, hkv=2, d=128, ctx=(300, 300))),
     "llama2-layer-short": ("llama2-7b-layer", dict(hq=8, hkv=8, ctx=(333, 333), vocab=100)),
@@ -81,9 +82,9 @@ ATTN_CASES = {
     "single-node": ("llama3-8b-gqa", dict(layers=1, ctx=(200, 200), vocab=100, tree="chain", nodes=(1, 1))),
     "mha-g1-t64": ("llama2-7b-layer", dict(hq=4, hkv=4, ctx=(129, 129), vocab=100, tree="chain",
                                            nodes=(64, 64))),
-    # one key tile per split; the last split starts at node 63 of a complete binary tree, so
-    # within one warp nodes 88..94 first see a visible key (themselves) in chunk 0 and node
-    # 95 only in chunk 1: the lazy rescale must still run warp-uniformly
+    # 18 key tiles on 18 CTAs, one each; the last tile starts at node 63 of a complete binary
+    # tree, so within one warp nodes 88..94 first see a visible key (themselves) in chunk 0
+    # and node 95 only in chunk 1: the lazy rescale must still run warp-uniformly
     "split-on-tree-tile": ("llama3-8b-gqa", dict(layers=1, hq=4, hkv=1, ctx=(961, 961), vocab=100, tree="binary",
                                                   nodes=(127, 127))),
 }
@@ -98,6 +99,22 @@ def test_attention_matches_oracle(case):
         for b in range(w.cfg.batch):
             ref = _attn_ref(w, l, b)
             _check_attn(got[l][w.nodes_of(b)], ref, w.cfg.dtype, f"{case} l{l} b{b}")
+
+
+@pytest.mark.parametrize("case", ["llama3-gqa-2layers", "batched-paged-short", "split-on-tree-tile"])
+def test_attention_without_workspace_matches_oracle(case):
+    """No scratch: each (layer, tree, KV head, 256-row block) in one CTA, same results."""
+    base, over = ATTN_CASES[case]
+    w = syn.Workload(syn.shrink(syn.CONFIGS[base], **over), 11)
+    dw = DeviceWorkload(w, with_step_buffers=False)
+    dw.workspace = None
+    dw.attention()
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == 0
+    got = dw.attn_out.float().cpu().numpy()
+    for l in range(w.cfg.layers):
+        for b in range(w.cfg.batch):
+            _check_attn(got[l][w.nodes_of(b)], _attn_ref(w, l, b), w.cfg.dtype, f"{case} l{l} b{b}")
 
 
 def test_attention_peaked_context_exposes_mask():

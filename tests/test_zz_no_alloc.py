@@ -47,7 +47,7 @@ def _case(cfg_name, seed, **over):
 def test_noalloc_matches_workspace_entry_on_consecutive_calls():
     cases = [
         _case("llama2-7b-layer", 71, hq=8, hkv=8, ctx=(333, 333), vocab=100),
-        _case("batched-paged", 72, batch=2, ctx=(300, 900), vocab=100, hq=8, hkv=2),
+        _case("batched-paged", 72, batch=2, ctx=(300, 600), vocab=100, hq=8, hkv=2),
     ]
     for dw, need in cases:
         assert 0 < need <= STATIC_SCRATCH_BYTES, need     # the split path (scratch) is exercised
