@@ -15,11 +15,11 @@
 // (unit, key tile) space is cut into one equal contiguous range per CTA, one CTA per SM, so
 // every SM gets the same number of key tiles whatever the unit count.  Each warp walks its
 // CTA's range as segments (whole units, or a piece of a unit at either end of the range).
-// Whole units are written directly; a piece writes an fp32 partial (O unnormalised, running
-// max, row sum), and the warp that writes the last piece of a 32-row block merges the
-// pieces of that block once its own range is done.  The softmax warps load the next
-// segment's Q before the epilogue of the current one, so the tensor core does not wait on
-// it.  Grid (fallback without scratch): one CTA per unit.
+// Whole units are written directly.  Of the pieces of a unit cut by range ends, all but the
+// last leave an fp32 partial (O unnormalised, running max, row sum); the warp that finishes
+// the last one merges those partials with its own O, still in TMEM.  The softmax warps load
+// the next segment's Q before the epilogue of the current one, so the tensor core does not
+// wait on it.  Grid (fallback without scratch): one CTA per unit.
 //
 // Warp roles (320 threads):
 //   warp 0      TMA producer: K and V tiles into two stage pairs (K_j, V_j | K_j+1, V_j+1).
@@ -106,20 +106,13 @@ struct SegRun {
   int pad;
 };
 
-// A range holds at most two pieces (its first and its last segment), so a warp leaves at
-// most two merges for the end.
-constexpr int kMaxDefer = 2;
-
 // Shared memory of one softmax warp.
 struct WarpArea {
   int parents[128];            // parent array of the last tree seen
   SegRun run[2];               // the segment being computed and the next one
-  SegRun defer[kMaxDefer];     // 32-row blocks to merge at the end of the range
   int tree_node0, tree_T;      // which tree `parents` holds
   int tree_invalid;            // that tree failed the parent check
   int mask_mp;                 // M-tile pair the ancestor masks in registers were built for
-  int ndefer;
-  int pad[3];
 };
 constexpr uint32_t kSmemUsed = kOffWarp + 8 * sizeof(WarpArea);
 constexpr uint32_t kSmemBytes = kSmemUsed + 1024;   // slack to align the base to 1024 B
@@ -127,7 +120,7 @@ static_assert(kSmemBytes <= 232448, "shared memory budget");
 
 // Persistent schedule constants: CTA c owns global key tiles [c*W/P, (c+1)*W/P).
 struct WalkConst {
-  int persistent, W, Wl, P, c, r0, r1, backward;
+  int persistent, W, Wl, P, c, r0, r1;
 };
 
 // Tree b: first node, size, context, key tiles and M-tile pairs; returns the key tiles of all
@@ -205,11 +198,9 @@ __device__ __noinline__ void make_walk_const(const AttnParams& p, WalkConst& wc)
   wc.c = (int)blockIdx.x;
   wc.r0 = range_start(wc, wc.c);
   wc.r1 = range_start(wc, wc.c + 1);
-  wc.backward = wc.c & 1;
 }
 
-// A walker's cursor before its first step.  A backward walk ends at g0 - 1 >= -1, so the
-// start value must lie outside [-1, W].
+// A walker's cursor before its first step (a walk's cursors lie in [0, W]).
 constexpr int kWalkStart = INT_MIN;
 
 // Next segment of this CTA for one walker (cursor starts at kWalkStart); s.valid = 0 when done.
@@ -241,26 +232,17 @@ __device__ __noinline__ void next_segment(const AttnParams& p, const WalkConst& 
     return;
   }
   if (wc.W <= 0) return;
-  if (cursor == kWalkStart) cursor = wc.backward ? wc.r1 - 1 : wc.r0;
-  // self-check: every step must decode and move the cursor (the walk then always ends)
-  auto fail = [&]() {
+  if (cursor == kWalkStart) cursor = wc.r0;
+  if (cursor >= wc.r1) return;
+  // self-check: every step must decode and move the cursor forward (the walk then ends)
+  if (!decode_tile(p, wc.Wl, cursor, s) || s.ug0 + s.n_kt <= cursor || s.ug0 > cursor) {
     atomicMax(p.dev_status, (int)PTD_ERR_TIMEOUT);
-    cursor = wc.backward ? wc.r0 - 1 : wc.r1;
-  };
-  int g0, g1;
-  if (!wc.backward) {
-    if (cursor >= wc.r1) return;
-    if (!decode_tile(p, wc.Wl, cursor, s) || s.ug0 + s.n_kt <= cursor || s.ug0 > cursor) return fail();
-    g0 = cursor;
-    g1 = min(s.ug0 + s.n_kt, wc.r1);
-    cursor = g1;
-  } else {
-    if (cursor < wc.r0) return;
-    if (!decode_tile(p, wc.Wl, cursor, s) || s.ug0 + s.n_kt <= cursor || s.ug0 > cursor) return fail();
-    g1 = cursor + 1;
-    g0 = max(s.ug0, wc.r0);
-    cursor = g0 - 1;
+    cursor = wc.r1;
+    return;
   }
+  const int g0 = cursor;
+  const int g1 = min(s.ug0 + s.n_kt, wc.r1);
+  cursor = g1;
   s.kt_begin = g0 - s.ug0;
   s.kt_end = g1 - s.ug0;
   if (s.kt_begin == 0 && s.kt_end == s.n_kt) {
@@ -537,7 +519,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       wa->tree_node0 = -1;
       wa->tree_T = -1;
       wa->mask_mp = -1;
-      wa->ndefer = 0;
     }
     __syncwarp();
     uint32_t am0 = 0, am1 = 0, am2 = 0, am3 = 0;   // ancestor mask of this row's node
@@ -623,9 +604,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
     };
 
-    // Output rows of one 32-row block from the partials of all pieces of its unit:
+    // Output rows of one 32-row block from all pieces of its unit:
     // O = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c (pieces with l_c = 0 saw no key).
-    auto merge = [&](const volatile SegRun* rec) {
+    // With `own`, this warp's piece is still in TMEM (O_t, m_own, l_own) rather than a partial.
+    auto merge = [&](const volatile SegRun* rec, bool own, float m_own, float l_own) {
       const int ug0 = rec->s.ug0, ug1 = ug0 + rec->s.n_kt;
       const int T = rec->s.T, mp = rec->s.mp;
       const bool invalid = rec->invalid != 0;
@@ -634,7 +616,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool row_valid = node < T;
       const int first = owner_cta(wc, ug0), last = owner_cta(wc, ug1 - 1);
       const float2* pml = reinterpret_cast<const float2*>(p.part_ml) + (size_t)t * 128 + row;
-      auto owns = [&](int c) { return c <= last && range_start(wc, c + 1) > range_start(wc, c); };
+      // CTAs whose partial is read (an empty range owns no piece; with `own`, skip this CTA)
+      auto partial_of = [&](int c) {
+        return c <= last && range_start(wc, c + 1) > range_start(wc, c) && !(own && c == wc.c);
+      };
       float M = -INFINITY, L = 0.f;
       auto fold = [&](float2 ml) {
         if (ml.y > 0.f) {
@@ -646,23 +631,32 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       };
+      if (own) fold(make_float2(m_own, l_own));
       for (int c = first; c <= last; c += 2) {   // two pieces' (m, l) loads at a time
-        const bool h0 = owns(c), h1 = owns(c + 1);
+        const bool h0 = partial_of(c), h1 = partial_of(c + 1);
         const float2 a0 = h0 ? __ldcg(pml + (size_t)piece_slot(wc, c, ug0, ug1) * 256) : make_float2(-INFINITY, 0.f);
         const float2 a1 = h1 ? __ldcg(pml + (size_t)piece_slot(wc, c + 1, ug0, ug1) * 256) : make_float2(-INFINITY, 0.f);
         fold(a0);
         fold(a1);
       }
       const float inv = (L > 0.f && !invalid) ? 1.f / L : 0.f;
+      const float w_own = (own && l_own > 0.f) ? ptx_exp2(m_own - M) : 0.f;
       const size_t orow = (((size_t)rec->s.lq * p.n_total + rec->s.node0 + node) * p.hq + (size_t)rec->s.hkv * G + g) * 128;
       uint4* dst = reinterpret_cast<uint4*>(p.out) + (row_valid ? orow : 0) / 8;
 #pragma unroll 1
       for (int h = 0; h < 4; ++h) {   // 32 output columns at a time
         float acc[32];
+        if (own) {   // warp-uniform
+          tmem_ld32(tO + (uint32_t)h * 32u, r);
+          tmem_ld_wait();
 #pragma unroll
-        for (int d = 0; d < 32; ++d) acc[d] = 0.f;
+          for (int d = 0; d < 32; ++d) acc[d] = w_own > 0.f ? __uint_as_float(r[d]) * w_own : 0.f;
+        } else {
+#pragma unroll
+          for (int d = 0; d < 32; ++d) acc[d] = 0.f;
+        }
         for (int c = first; c <= last; ++c) {
-          if (!owns(c)) continue;
+          if (!partial_of(c)) continue;
           const size_t q = (size_t)piece_slot(wc, c, ug0, ug1);
           const float2 ml = __ldcg(pml + q * 256);
           const float* po = p.part_o + (q * 2 + t) * (128 * 128) + (size_t)(h * 32) * 128 + row;
@@ -838,62 +832,53 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       } else {
-        // A piece: O unnormalised, running max (log2 units) and row sum.  The partial of an
-        // M tile is column-major ([column][128 rows]), so each store of the warp is one
-        // contiguous 128-byte line.
-        float* po = p.part_o + ((size_t)slot * 2 + t) * (128 * 128) + row;
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          tmem_ld32(tO + (uint32_t)c * 32u, r);
-          tmem_ld_wait();
-          if (have_o) {
-#pragma unroll
-            for (int e = 0; e < 32; ++e) po[(size_t)(c * 32 + e) * 128] = __uint_as_float(r[e]);
-          }
-        }
-        reinterpret_cast<float2*>(p.part_ml)[(size_t)slot * 256 + (size_t)t * 128 + row] =
-            have_o ? make_float2(m_run, l_run) : make_float2(-INFINITY, 0.f);
-        // The warp that writes the last piece of this 32-row block merges the block (CTAs
-        // with an empty range own no piece), after the rest of its range: a merge waits on
-        // loads from other SMs and would stall this CTA's pipeline here.
+        // A piece.  If every other piece of this 32-row block has left its partial, this warp
+        // finishes the block from its own O in TMEM.  Otherwise it leaves a partial (O
+        // unnormalised, running max in log2 units, row sum; column-major per M tile, so each
+        // store of the warp is one 128-byte line) and counts itself in; if that makes it the
+        // last, it merges the partials.  (Ranges are walked forward, so the piece at the start
+        // of a range is normally done long before the piece that ends the previous range.)
         const int ug0 = cur->s.ug0;
         const int ug1 = ug0 + cur->s.n_kt;
         const int first = owner_cta(wc, ug0);
         const int last = owner_cta(wc, ug1 - 1);
-        __threadfence();
-        __syncwarp();
-        int is_last = 0;
+        int* counter = p.counters + (size_t)cur->s.unit * 8 + t * 4 + (warp & 3);
+        int pieces = 0, done = 0;
         if (lane == 0) {
-          int pieces = 0;
           for (int c = first; c <= last; ++c) pieces += range_start(wc, c + 1) > range_start(wc, c) ? 1 : 0;
-          const int old = atomicAdd(p.counters + (size_t)cur->s.unit * 8 + t * 4 + (warp & 3), 1);
-          is_last = old == pieces - 1;
+          done = atomicAdd(counter, 0) == pieces - 1;
         }
-        is_last = __shfl_sync(0xffffffffu, is_last, 0);
-        if (is_last) {
-          const int nd = wv->ndefer;
-          if (nd < kMaxDefer) {
-            constexpr int kRunWords = (int)(sizeof(SegRun) / 4);
-            if (lane < kRunWords)
-              reinterpret_cast<volatile int*>(&wa->defer[nd])[lane] = reinterpret_cast<const volatile int*>(cur)[lane];
-            __syncwarp();
-            if (lane == 0) wa->ndefer = nd + 1;
-            __syncwarp();
-          } else {
+        done = __shfl_sync(0xffffffffu, done, 0);
+        if (done) {
+          __threadfence();
+          merge(cur, true, have_o ? m_run : -INFINITY, have_o ? l_run : 0.f);
+        } else {
+          float* po = p.part_o + ((size_t)slot * 2 + t) * (128 * 128) + row;
+#pragma unroll 1
+          for (int c = 0; c < 4; ++c) {
+            tmem_ld32(tO + (uint32_t)c * 32u, r);
+            tmem_ld_wait();
+            if (have_o) {
+#pragma unroll
+              for (int e = 0; e < 32; ++e) po[(size_t)(c * 32 + e) * 128] = __uint_as_float(r[e]);
+            }
+          }
+          reinterpret_cast<float2*>(p.part_ml)[(size_t)slot * 256 + (size_t)t * 128 + row] =
+              have_o ? make_float2(m_run, l_run) : make_float2(-INFINITY, 0.f);
+          __threadfence();
+          __syncwarp();
+          int is_last = 0;
+          if (lane == 0) is_last = atomicAdd(counter, 1) == pieces - 1;
+          is_last = __shfl_sync(0xffffffffu, is_last, 0);
+          if (is_last) {
             __threadfence();
-            merge(cur);   // not reached: a range holds at most two pieces
+            merge(cur, false, 0.f, 0.f);
           }
         }
       }
       tc_fence_before();
       k ^= 1;
       have = have_next;
-    }
-    // merges left for the end of the range
-    if (ok) {
-      const int nd = wv->ndefer;
-      if (nd > 0) __threadfence();
-      for (int d = 0; d < nd; ++d) merge(&wv->defer[d]);
     }
   }
 
