@@ -259,6 +259,29 @@ __device__ __forceinline__ int piece_slot(const WalkConst& wc, int c, int ug0, i
   return c * 2 + ((rs >= ug0 && rs < ug1) ? 0 : 1);
 }
 
+// Rare path of the softmax, kept out of the hot loop: O_t (n_o 16-column groups) and the
+// bf16 P chunks [0, c) of S_t scaled by alpha.  Warp-collective.
+__device__ __noinline__ void rescale_tmem(uint32_t tO, uint32_t tS, int n_o, int c, float alpha) {
+  for (int q = 0; q < n_o; ++q) {
+    uint32_t o16[16];
+    tmem_ld16(tO + (uint32_t)q * 16u, o16);
+    tmem_ld_wait();
+#pragma unroll
+    for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
+    tmem_st16(tO + (uint32_t)q * 16u, o16);
+  }
+  if (c > 0) tmem_st_wait();
+  for (int q = 0; q < c; ++q) {
+    uint32_t p16[16];
+    tmem_ld16(tS + (uint32_t)q * 16u, p16);
+    tmem_ld_wait();
+#pragma unroll
+    for (int e = 0; e < 16; ++e)
+      p16[e] = pack_bf16x2(__uint_as_float(p16[e] << 16) * alpha, __uint_as_float(p16[e] & 0xFFFF0000u) * alpha);
+    tmem_st16(tS + (uint32_t)q * 16u, p16);
+  }
+}
+
 template <bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
@@ -733,32 +756,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             f2_unpack(sum, s0, s1);
             sum = f2_pack(s0 * alpha, s1 * alpha);
             l_run *= alpha;
-            if (jj > 0) {
-              // O_t is idle here: PV_t of the previous tile completed before S_t of this one
-#pragma unroll 1
-              for (int q = 0; q < 8; ++q) {
-                uint32_t o16[16];
-                tmem_ld16(tO + (uint32_t)q * 16u, o16);
-                tmem_ld_wait();
-#pragma unroll
-                for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
-                tmem_st16(tO + (uint32_t)q * 16u, o16);
-              }
-            }
-            if (c > 0) {
-              tmem_st_wait();
-#pragma unroll 1
-              for (int q = 0; q < c; ++q) {   // bf16 P of the earlier chunks of this tile
-                uint32_t p16[16];
-                tmem_ld16(tS + (uint32_t)q * 16u, p16);
-                tmem_ld_wait();
-#pragma unroll
-                for (int e = 0; e < 16; ++e)
-                  p16[e] = pack_bf16x2(__uint_as_float(p16[e] << 16) * alpha,
-                                       __uint_as_float(p16[e] & 0xFFFF0000u) * alpha);
-                tmem_st16(tS + (uint32_t)q * 16u, p16);
-              }
-            }
+            rescale_tmem(tO, tS, jj > 0 ? 8 : 0, c, alpha);
           }
           const float m_use = m_run == -INFINITY ? 0.f : m_run;   // -inf only while nothing is visible
           const unsigned long long negm = f2_pack(-m_use, -m_use);
