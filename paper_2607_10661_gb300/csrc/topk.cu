@@ -236,10 +236,11 @@ __global__ void __launch_bounds__(kThreads) topk_cluster_kernel(const T* __restr
 // Each CTA stages its contiguous slice of the row (up to kSliceVec 16-byte vectors) into
 // shared memory with bulk asynchronous copies, so the row is read from HBM exactly once,
 // then makes three passes over shared memory:
-//   1. every thread's maximum;
-//   2. T = the k-th largest thread maximum.  The k threads holding those maxima own k
-//      distinct elements >= T, so every element of the CTA's top-k is >= T;
-//   3. elements >= T become candidates (exact 64-bit keys); the CTA's top-k is selected
+//   1. every thread's maximum (four vectors in flight per thread);
+//   2. T = the k-th largest warp maximum (k <= 8 warps), else the k-th largest thread
+//      maximum.  The k warps (threads) holding those maxima own k distinct elements >= T,
+//      so every element of the CTA's top-k is >= T;
+//   3. elements >= T become candidates (exact 64-bit keys); warp 0 selects the CTA's top-k
 //      among them.
 // A slice with more than kCandCap candidates (many ties at the threshold, e.g. a constant
 // row) is selected exactly with per-thread sorted lists instead.
@@ -272,6 +273,7 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
   __shared__ uint64_t cand[kCandCap];
   __shared__ int ncand;
   __shared__ float thr_s;
+  __shared__ float wmax_s[kWarps];
   __shared__ __align__(8) uint64_t bar_s;
   __shared__ int abort_s;
 
@@ -320,18 +322,56 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
       for (int i = a1; i < vocab; ++i) tmax = fmaxf(tmax, Vec<__nv_bfloat16>::scalar(row + i));
     mbar_wait(bar, phase, &abort_s, dev_status);   // bounded: a lost copy only flags PTD_ERR_TIMEOUT
 
-    // pass 1: thread maximum
-    for (int v = tid; v < nv; v += kThreads) {
-      const uint4 x = slice[v];
-      tmax = fmax3(tmax, bf16_lo(x.x), bf16_hi(x.x));
-      tmax = fmax3(tmax, bf16_lo(x.y), bf16_hi(x.y));
-      tmax = fmax3(tmax, bf16_lo(x.z), bf16_hi(x.z));
-      tmax = fmax3(tmax, bf16_lo(x.w), bf16_hi(x.w));
+    // pass 1: thread maximum (four vectors in flight, two chains)
+    {
+      float t1 = -INFINITY;
+      int v = tid;
+      for (; v + 3 * kThreads < nv; v += 4 * kThreads) {
+        uint4 x[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) x[u] = slice[v + u * kThreads];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          tmax = fmax3(tmax, bf16_lo(x[u].x), bf16_hi(x[u].x));
+          t1 = fmax3(t1, bf16_lo(x[u].y), bf16_hi(x[u].y));
+          tmax = fmax3(tmax, bf16_lo(x[u].z), bf16_hi(x[u].z));
+          t1 = fmax3(t1, bf16_lo(x[u].w), bf16_hi(x[u].w));
+        }
+      }
+      for (; v < nv; v += kThreads) {
+        const uint4 x = slice[v];
+        tmax = fmax3(tmax, bf16_lo(x.x), bf16_hi(x.x));
+        t1 = fmax3(t1, bf16_lo(x.y), bf16_hi(x.y));
+        tmax = fmax3(tmax, bf16_lo(x.z), bf16_hi(x.z));
+        t1 = fmax3(t1, bf16_lo(x.w), bf16_hi(x.w));
+      }
+      tmax = fmaxf(tmax, t1);
     }
     const bool has_elems = tid < nv || (own_head && a0 > 0) || (own_tail && a1 < vocab);
 
-    // pass 2: T = k-th largest thread maximum (over threads that own elements)
-    {
+    // pass 2: T = k-th largest warp maximum (k <= kWarps: the k warps holding those maxima
+    // own k distinct elements >= T), else the k-th largest thread maximum
+    if (k <= kWarps) {
+      float wm = has_elems ? tmax : -INFINITY;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
+      if (lane == 0) wmax_s[warp] = wm;
+      if (tid == 0) ncand = 0;
+      __syncthreads();
+      float t_k = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < kWarps; ++i) {
+        const float wi = wmax_s[i];
+        int above = 0;
+#pragma unroll
+        for (int j = 0; j < kWarps; ++j) {
+          const float wj = wmax_s[j];
+          above += (wj > wi || (wj == wi && j < i)) ? 1 : 0;
+        }
+        if (above == k - 1) t_k = wi;
+      }
+      if (tid == 0) thr_s = t_k;
+    } else {
       const uint64_t key = has_elems ? make_key(ordered_bits(tmax), (uint32_t)tid) : 0ull;
       const uint64_t wk = warp_topk_of_one(key, k, lane);
       if (lane < k) warp_keys[warp][lane] = wk;
@@ -348,8 +388,8 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
         }
         if (lane == 0) thr_s = kth != 0ull ? from_ordered((uint32_t)(kth >> 32)) : -INFINITY;
       }
-      __syncthreads();
     }
+    __syncthreads();
     const float thr = thr_s;
 
     // pass 3: candidates >= T
@@ -359,8 +399,7 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
         if (pos < kCandCap) cand[pos] = make_key(ordered_bits(f), gidx);
       }
     };
-    for (int v = tid; v < nv; v += kThreads) {
-      const uint4 x = slice[v];
+    auto scan = [&](const uint4& x, int v) {
       float vm = fmax3(bf16_lo(x.x), bf16_hi(x.x), bf16_lo(x.y));
       vm = fmax3(vm, bf16_hi(x.y), bf16_lo(x.z));
       vm = fmax3(vm, bf16_hi(x.z), bf16_lo(x.w));
@@ -374,6 +413,17 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
           offer(bf16_hi(w[q]), gi + 2 * q + 1);
         }
       }
+    };
+    {
+      int v = tid;
+      for (; v + 3 * kThreads < nv; v += 4 * kThreads) {   // four vectors in flight
+        uint4 x[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) x[u] = slice[v + u * kThreads];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) scan(x[u], v + u * kThreads);
+      }
+      for (; v < nv; v += kThreads) scan(slice[v], v);
     }
     if (own_head)
       for (int i = 0; i < a0; ++i) offer(Vec<__nv_bfloat16>::scalar(row + i), (uint32_t)i);
@@ -386,7 +436,17 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
     ThreadList<KM> list;
     list.init();
     if (nc <= kCandCap) {
-      for (int i = tid; i < nc; i += kThreads) list.push_key(cand[i]);
+      // few candidates: warp 0 selects the CTA's top-k by itself (no cross-warp merge)
+      if (warp == 0) {
+        for (int i = lane; i < nc; i += 32) list.push_key(cand[i]);
+        for (int s = 0; s < k; ++s) {
+          const uint64_t mine = list.head();
+          const uint64_t best = warp_max_u64(mine);
+          if (mine == best) list.pop();
+          if (lane == 0) cta_keys[s] = best;
+        }
+      }
+      __syncthreads();   // every thread is done reading the slice
     } else {
       if (own_head)
         for (int i = 0; i < a0; ++i) list.push(ordered_bits(Vec<__nv_bfloat16>::scalar(row + i)), (uint32_t)i);
@@ -398,21 +458,21 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
       }
       if (own_tail)
         for (int i = a1; i < vocab; ++i) list.push(ordered_bits(Vec<__nv_bfloat16>::scalar(row + i)), (uint32_t)i);
-    }
-    for (int s = 0; s < k; ++s) {
-      const uint64_t mine = list.head();
-      const uint64_t best = warp_max_u64(mine);
-      if (mine == best) list.pop();
-      if (lane == 0) warp_keys[warp][s] = best;
-    }
-    __syncthreads();   // also: every thread is done reading the slice
-    if (warp == 0) {
-      int cur = 0;
       for (int s = 0; s < k; ++s) {
-        const uint64_t mine = (lane < kWarps && cur < k) ? warp_keys[lane][cur] : 0ull;
+        const uint64_t mine = list.head();
         const uint64_t best = warp_max_u64(mine);
-        if (lane < kWarps && mine == best && best != 0ull) ++cur;
-        if (lane == 0) cta_keys[s] = best;
+        if (mine == best) list.pop();
+        if (lane == 0) warp_keys[warp][s] = best;
+      }
+      __syncthreads();   // also: every thread is done reading the slice
+      if (warp == 0) {
+        int cur = 0;
+        for (int s = 0; s < k; ++s) {
+          const uint64_t mine = (lane < kWarps && cur < k) ? warp_keys[lane][cur] : 0ull;
+          const uint64_t best = warp_max_u64(mine);
+          if (lane < kWarps && mine == best && best != 0ull) ++cur;
+          if (lane == 0) cta_keys[s] = best;
+        }
       }
     }
     cluster.sync();
