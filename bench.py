@@ -176,8 +176,7 @@ def run_gpu(args, rank: int, world: int, dist):
         if ev is not None:
             ev[1].record(stream)
         n += dw.topk()
-        n += dw.verify()
-        n += dw.compact()
+        n += dw.verify_and_compact()
         return n
 
     dw.dev_status.zero_()              # sticky status word: cleared once, read after the run

@@ -14,6 +14,9 @@
  *   ptd_verify_greedy    eligible edges I and accepted sequence X' (Sec. 3.2)
  *   ptd_kv_compact       move the accepted nodes' K/V behind the prefix (Alg. 1 step 6)
  *
+ * plus ptd_verify_and_compact (the last two as one launch) and ptd_tree_verify_step (the
+ * whole step: attention, top-k, verification and compaction on one stream)
+ *
  * Conventions shared by every call
  *   - Pointers are DEVICE pointers unless a comment says "host".  The caller owns
  *     all memory; the library never allocates, frees or synchronises.  Scratch
@@ -182,9 +185,20 @@ ptd_status ptd_kv_compact(const ptd_tree* tree, const ptd_kv_cache* cache,
                           const int32_t* accepted_nodes, const int32_t* accept_len,
                           int32_t* new_ctx_lens, void* stream);
 
+/* ptd_verify_greedy followed by ptd_kv_compact, in one launch: the same outputs (accepted
+ * path, accept length, bonus token, status, compacted cache, new context lengths) with the
+ * same arguments and rules, computed by one kernel in which every CTA of the compaction
+ * grid verifies its tree first.  This is what ptd_tree_verify_step uses.  The paper has no
+ * separate counterpart: it is Alg. 1 steps 5-6 as one call. */
+ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
+                                  const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
+                                  int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
+                                  int32_t* dev_status, void* stream);
+
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.
- * Equivalent to the four calls above in that order on `stream`. */
+ * Equivalent to ptd_tree_attention, ptd_topk_draft and ptd_verify_and_compact in that
+ * order on `stream` (three launches). */
 typedef struct {
   const void* q;               /* [L][N_tot][Hq][D]                                    */
   int32_t num_q_heads;

@@ -289,6 +289,28 @@ ptd_status ptd_kv_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const
   return st;
 }
 
+ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
+                                  const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
+                                  int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
+                                  int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  ptd_status st = check_tree(tree);
+  if (st != PTD_OK) return st;
+  if ((st = check_cache(cache)) != PTD_OK) return st;
+  if (!tokens || !target || target_stride < 1 || !accepted_nodes || !accept_len || !bonus_token || !dev_status ||
+      !new_ctx_lens)
+    return PTD_ERR_INVALID_ARG;
+  if (new_ctx_lens == tree->ctx_lens) return PTD_ERR_INVALID_ARG;   // other CTAs still read ctx_lens
+  const int row_bytes = cache->num_kv_heads * cache->head_dim * (int)dtype_size(cache->dtype);
+  st = cuda_status(ptd::launch_verify_compact(
+      tree->node_offsets, tree->parents, tokens, target, target_stride, tree->total_nodes, tree->max_nodes,
+      accepted_nodes, accept_len, bonus_token, dev_status, cache->k, cache->v, row_bytes, cache->num_layers,
+      tree->batch, cache->page_size, cache->seq_capacity, cache->num_pages, cache->block_table, cache->max_pages,
+      tree->ctx_lens, new_ctx_lens, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
 ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a,
                                 void* stream) {
   if (!a) return PTD_ERR_INVALID_ARG;
@@ -301,11 +323,8 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
                       a->topk_val, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
-  st = ptd_verify_greedy(tree, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len, a->bonus_token,
-                         a->dev_status, stream);
-  if (st != PTD_OK) return st;
-  total += g_last_launches;
-  st = ptd_kv_compact(tree, cache, a->accepted_nodes, a->accept_len, a->new_ctx_lens, stream);
+  st = ptd_verify_and_compact(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len,
+                              a->bonus_token, a->new_ctx_lens, a->dev_status, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
   g_last_launches = total;

@@ -176,6 +176,193 @@ __global__ void __launch_bounds__(kCompactThreads)
   }
 }
 
+// ------------------------------------------------------------------ fused (whole step)
+// Verification and compaction in one launch for the whole step: every CTA of the compaction
+// grid (layer, tree, K or V) verifies its tree on warp 0 (a tree is at most 128 nodes: 4 per
+// lane, pointer jumping with warp barriers only), so the path is in shared memory before
+// the copy; CTA (0, b, K) writes the verification outputs.  The computation is that of
+// verify_greedy_kernel followed by kv_compact_kernel.
+struct TreeVerdict {
+  int path[kVerifyThreads];
+  int len;      // accepted length (0: the tree failed the checks)
+  int bonus;
+  int invalid;
+};
+
+__device__ void verify_tree_warp(const int32_t* __restrict__ node_offsets, const int32_t* __restrict__ parents,
+                                 const int32_t* __restrict__ tokens, const int32_t* __restrict__ target,
+                                 int target_stride, int n_total, int max_nodes, int b, int* par_s, int* jump_s,
+                                 int* reach_s, int* depth_s, int* onpath_s, TreeVerdict* out) {
+  const int lane = threadIdx.x & 31;
+  const int node0 = node_offsets[b];
+  const int T = node_offsets[b + 1] - node0;
+  const bool bad_shape = T < 1 || T > max_nodes || T > kVerifyThreads || node0 < 0 || node0 + T > n_total;
+  bool bad = false;
+  int par[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = lane + 32 * q;
+    par[q] = -1;
+    if (!bad_shape && i < T) {
+      par[q] = parents[node0 + i];
+      bad = bad || (i == 0 ? (par[q] != -1) : (par[q] < 0 || par[q] >= i));
+    }
+  }
+  if (__any_sync(0xffffffffu, bad) || bad_shape) {
+    if (lane == 0) {
+      out->len = 0;
+      out->bonus = -1;
+      out->invalid = 1;
+    }
+    return;
+  }
+  // eligible edge into node i: tokens[i] == V_{parent}
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = lane + 32 * q;
+    if (i < T) {
+      const int elig = i == 0 ? 1 : (tokens[node0 + i] == target[(size_t)(node0 + par[q]) * target_stride]);
+      par_s[i] = par[q];
+      jump_s[i] = i == 0 ? 0 : par[q];
+      reach_s[i] = elig;
+      depth_s[i] = i == 0 ? 0 : 1;
+      onpath_s[i] = 0;
+    }
+  }
+  __syncwarp();
+  // pointer jumping: after round r, jump[i] is the 2^r-th ancestor (clamped at the root)
+  for (int r = 0; (1 << r) < T; ++r) {
+    int j[4], rj[4], dj[4], jj[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = lane + 32 * q;
+      j[q] = 0;
+      if (i < T) {
+        j[q] = jump_s[i];
+        rj[q] = reach_s[j[q]];
+        dj[q] = depth_s[j[q]];
+        jj[q] = jump_s[j[q]];
+      }
+    }
+    __syncwarp();
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = lane + 32 * q;
+      if (i < T && j[q] != 0) {
+        reach_s[i] &= rj[q];
+        depth_s[i] += dj[q];
+        jump_s[i] = jj[q];
+      }
+    }
+    __syncwarp();
+  }
+  int dmax = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = lane + 32 * q;
+    if (i < T && reach_s[i]) dmax = max(dmax, depth_s[i]);
+  }
+  const int D = __reduce_max_sync(0xffffffffu, dmax);
+  // mark every node on a root path that reaches depth D through eligible edges
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = lane + 32 * q;
+    if (i < T && reach_s[i] && depth_s[i] == D)
+      for (int a = i; a >= 0 && !onpath_s[a]; a = par_s[a]) onpath_s[a] = 1;
+  }
+  __syncwarp();
+  // the lexicographically smallest longest path, one level per step
+  int cur = 0;
+  if (lane == 0) out->path[0] = 0;
+  for (int d = 1; d <= D; ++d) {
+    int best = 0x7FFFFFFF;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = lane + 32 * q;
+      if (i < T && par_s[i] == cur && onpath_s[i]) best = min(best, i);
+    }
+    cur = __reduce_min_sync(0xffffffffu, best);
+    if (lane == 0) out->path[d] = cur;
+  }
+  if (lane == 0) {
+    out->len = D + 1;
+    out->bonus = target[(size_t)(node0 + cur) * target_stride];
+    out->invalid = 0;
+  }
+}
+
+__global__ void __launch_bounds__(kCompactThreads)
+    verify_compact_kernel(const int32_t* __restrict__ node_offsets, const int32_t* __restrict__ parents,
+                          const int32_t* __restrict__ tokens, const int32_t* __restrict__ target, int target_stride,
+                          int n_total, int max_nodes, int32_t* __restrict__ accepted, int32_t* __restrict__ accept_len,
+                          int32_t* __restrict__ bonus, int32_t* __restrict__ dev_status, uint8_t* __restrict__ k_cache,
+                          uint8_t* __restrict__ v_cache, int row_bytes, int batch, int page_size, int seq_capacity,
+                          int num_pages, const int32_t* __restrict__ block_table, int max_pages,
+                          const int32_t* __restrict__ ctx_lens, int32_t* __restrict__ new_ctx) {
+  __shared__ int par_s[kVerifyThreads], jump_s[kVerifyThreads], reach_s[kVerifyThreads];
+  __shared__ int depth_s[kVerifyThreads], onpath_s[kVerifyThreads];
+  __shared__ TreeVerdict verdict;
+  const int layer = blockIdx.x, b = blockIdx.y;
+  if (threadIdx.x < 32)
+    verify_tree_warp(node_offsets, parents, tokens, target, target_stride, n_total, max_nodes, b, par_s, jump_s,
+                     reach_s, depth_s, onpath_s, &verdict);
+  __syncthreads();
+  int len = verdict.len;
+  if (len > max_nodes) len = max_nodes;
+  const int C = ctx_lens[b];
+  if (layer == 0 && blockIdx.z == 0) {
+    int32_t* acc_row = accepted + (size_t)b * max_nodes;
+    for (int j = threadIdx.x; j < max_nodes; j += kCompactThreads) acc_row[j] = j < len ? verdict.path[j] : -1;
+    if (threadIdx.x == 0) {
+      accept_len[b] = len;
+      bonus[b] = verdict.bonus;
+      if (verdict.invalid) atomicMax(dev_status, (int)PTD_ERR_INVALID_TREE);
+      new_ctx[b] = C + len;
+    }
+  }
+  if (len <= 1 || C < 0) return;   // the root already sits at slot C
+  uint8_t* base = blockIdx.z == 0 ? k_cache : v_cache;
+  const int cap = page_size > 0 ? max_pages * page_size : seq_capacity;
+  auto row_ptr = [&](int slot) -> uint8_t* {
+    size_t r;
+    if (page_size > 0) {
+      const int pg = block_table[(size_t)b * max_pages + slot / page_size];
+      if (pg < 0 || pg >= num_pages) return nullptr;
+      r = ((size_t)layer * num_pages + pg) * page_size + slot % page_size;
+    } else {
+      r = ((size_t)layer * batch + b) * seq_capacity + slot;
+    }
+    return base + r * (size_t)row_bytes;
+  };
+  const int nchunk = row_bytes / 16;
+  for (int c = threadIdx.x; c < nchunk; c += kCompactThreads) {
+    for (int j0 = 1; j0 < len; j0 += kGroup) {
+      uint4 v[kGroup];
+      bool ok[kGroup];
+#pragma unroll
+      for (int q = 0; q < kGroup; ++q) {
+        const int j = j0 + q;
+        v[q] = make_uint4(0, 0, 0, 0);
+        ok[q] = false;
+        if (j < len) {
+          const int pj = verdict.path[j];
+          const int src = C + pj;
+          const uint8_t* sp = (pj > j && src < cap) ? row_ptr(src) : nullptr;
+          if (sp) {
+            v[q] = reinterpret_cast<const uint4*>(sp)[c];
+            ok[q] = true;
+          }
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < kGroup; ++q) {
+        uint8_t* dp = ok[q] ? row_ptr(C + j0 + q) : nullptr;
+        if (dp) reinterpret_cast<uint4*>(dp)[c] = v[q];
+      }
+    }
+  }
+}
+
 }  // namespace vc
 
 cudaError_t launch_verify(const int32_t* node_offsets, const int32_t* parents, const int32_t* tokens,
@@ -185,6 +372,19 @@ cudaError_t launch_verify(const int32_t* node_offsets, const int32_t* parents, c
   vc::verify_greedy_kernel<<<batch, vc::kVerifyThreads, 0, stream>>>(node_offsets, parents, tokens, target,
                                                                      target_stride, n_total, max_nodes, accepted,
                                                                      accept_len, bonus, dev_status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_verify_compact(const int32_t* node_offsets, const int32_t* parents, const int32_t* tokens,
+                                  const int32_t* target, int target_stride, int n_total, int max_nodes,
+                                  int32_t* accepted, int32_t* accept_len, int32_t* bonus, int32_t* dev_status, void* k,
+                                  void* v, int row_bytes, int layers, int batch, int page_size, int seq_capacity,
+                                  int num_pages, const int32_t* block_table, int max_pages, const int32_t* ctx_lens,
+                                  int32_t* new_ctx, cudaStream_t stream) {
+  vc::verify_compact_kernel<<<dim3(layers, batch, 2), vc::kCompactThreads, 0, stream>>>(
+      node_offsets, parents, tokens, target, target_stride, n_total, max_nodes, accepted, accept_len, bonus,
+      dev_status, static_cast<uint8_t*>(k), static_cast<uint8_t*>(v), row_bytes, batch, page_size, seq_capacity,
+      num_pages, block_table, max_pages, ctx_lens, new_ctx);
   return cudaGetLastError();
 }
 

@@ -75,5 +75,9 @@ class DeviceWorkload:
         return ptd.verify_greedy(self.tree, self.tokens, self.topk_idx, self.w.cfg.k, self.accepted,
                                  self.accept_len, self.bonus, self.dev_status, stream=stream)
 
+    def verify_and_compact(self, stream=None) -> int:
+        return ptd.verify_and_compact(self.tree, self.cache, self.tokens, self.topk_idx, self.w.cfg.k, self.accepted,
+                                      self.accept_len, self.bonus, self.new_ctx, self.dev_status, stream=stream)
+
     def compact(self, stream=None) -> int:
         return ptd.kv_compact(self.tree, self.cache, self.accepted, self.accept_len, self.new_ctx, stream=stream)

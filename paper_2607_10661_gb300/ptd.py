@@ -25,7 +25,7 @@ MAX_TOPK = 16
 EXPORTED = (
     "ptd_attention_workspace_size", "ptd_tree_attention", "ptd_topk_draft", "ptd_verify_greedy",
     "ptd_kv_compact", "ptd_tree_verify_step", "ptd_tree_verify_step_host", "ptd_last_launch_count",
-    "ptd_status_string", "ptd_tree_attention_noalloc",
+    "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact",
 )
 
 
@@ -92,6 +92,8 @@ def lib() -> ctypes.CDLL:
         L.ptd_verify_greedy.argtypes = [P(_Tree), vp, vp, i32, vp, vp, vp, vp, vp]
         L.ptd_kv_compact.restype = ctypes.c_int
         L.ptd_kv_compact.argtypes = [P(_Tree), P(_Cache), vp, vp, vp, vp]
+        L.ptd_verify_and_compact.restype = ctypes.c_int
+        L.ptd_verify_and_compact.argtypes = [P(_Tree), P(_Cache), vp, vp, i32, vp, vp, vp, vp, vp, vp]
         L.ptd_tree_verify_step.restype = ctypes.c_int
         L.ptd_tree_verify_step.argtypes = [P(_Tree), P(_Cache), P(_StepArgs), vp]
         L.ptd_tree_verify_step_host.restype = ctypes.c_int
@@ -231,6 +233,19 @@ def kv_compact(tree: Tree, cache: KVCache, accepted: torch.Tensor, accept_len: t
                               _dev(accept_len, "accept_len", torch.int32), _dev(new_ctx, "new_ctx", torch.int32),
                               _stream(stream))
     _check(st, "ptd_kv_compact")
+    return last_launch_count()
+
+
+def verify_and_compact(tree: Tree, cache: KVCache, tokens: torch.Tensor, target: torch.Tensor, target_stride: int,
+                       accepted: torch.Tensor, accept_len: torch.Tensor, bonus: torch.Tensor, new_ctx: torch.Tensor,
+                       dev_status: torch.Tensor, stream=None) -> int:
+    st = lib().ptd_verify_and_compact(ctypes.byref(tree.c), ctypes.byref(cache.c), _dev(tokens, "tokens", torch.int32),
+                                      _dev(target, "target", torch.int32), target_stride,
+                                      _dev(accepted, "accepted", torch.int32),
+                                      _dev(accept_len, "accept_len", torch.int32), _dev(bonus, "bonus", torch.int32),
+                                      _dev(new_ctx, "new_ctx", torch.int32), _dev(dev_status, "dev_status", torch.int32),
+                                      _stream(stream))
+    _check(st, "ptd_verify_and_compact")
     return last_launch_count()
 
 

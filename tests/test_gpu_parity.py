@@ -365,6 +365,52 @@ def test_compact_matches_oracle(name):
                 assert np.array_equal(seq_a[:new_ctx], ref[:new_ctx])
 
 
+@pytest.mark.parametrize("name", ["llama3-8b-gqa", "batched-paged", "tiny-fp32"])
+def test_verify_and_compact_equals_the_two_calls(name):
+    """ptd_verify_and_compact (one launch) leaves exactly what ptd_verify_greedy followed by
+    ptd_kv_compact leave: path, length, bonus, status, new context and cache bytes; also with
+    one tree made invalid."""
+    cfg = syn.CONFIGS[name]
+    over = dict(vocab=min(cfg.vocab, 64))
+    if name == "llama3-8b-gqa":
+        over.update(layers=3, ctx=(300, 300))
+    outs = []
+    for fused in (False, True):
+        w = syn.Workload(syn.shrink(cfg, **over), 43)
+        dw = DeviceWorkload(w)
+        target = np.random.default_rng(7).integers(0, w.cfg.vocab, size=(w.n_total, w.cfg.k)).astype(np.int32)
+        tokens = w.tokens.copy()
+        for b, par in enumerate(w.trees):   # most edges eligible: deep, tied paths
+            o = int(w.node_offsets[b])
+            for i in range(1, len(par)):
+                if (i * 7 + b) % 5:
+                    tokens[o + i] = target[o + par[i], 0]
+        bad = w.parents.copy()
+        if w.cfg.batch > 1:
+            o1 = int(w.node_offsets[1])
+            bad[o1 + 2] = 5                   # tree 1: a parent after its child
+        dw.parents.copy_(torch.tensor(bad))
+        dw.tokens.copy_(torch.tensor(tokens))
+        dw.topk_idx.copy_(torch.tensor(target))
+        dw.dev_status.zero_()
+        if fused:
+            assert dw.verify_and_compact() == 1
+        else:
+            dw.verify()
+            dw.compact()
+        torch.cuda.synchronize()
+        kk = dw.k.cpu()
+        kk = kk.view(torch.int16) if kk.dtype == torch.bfloat16 else kk.view(torch.int32)
+        outs.append((dw.accepted.cpu(), dw.accept_len.cpu(), dw.bonus.cpu(), dw.new_ctx.cpu(),
+                     int(dw.dev_status.item()), kk))
+    for x, y in zip(outs[0], outs[1]):
+        if isinstance(x, int):
+            assert x == y
+        else:
+            assert torch.equal(x, y)
+    assert int(outs[0][1].max()) > 2
+
+
 # ------------------------------------------------------------------------------ whole step
 
 @pytest.mark.parametrize("case", ["tiny-fp32", "llama3-gqa-2layers", "batched-paged-short"])
@@ -375,7 +421,7 @@ def test_whole_step_matches_oracle(case):
     dw = DeviceWorkload(w)
     k_before = dw.k.cpu()
     n = dw.step()
-    assert n >= 4
+    assert n == 3                                    # attention, top-k, verify + compact
     torch.cuda.synchronize()
     assert int(dw.dev_status.item()) == 0
     got = dw.attn_out.float().cpu().numpy()
@@ -394,6 +440,47 @@ def test_whole_step_matches_oracle(case):
         ref, new_ctx = oracle.kv_compact(w.seq_view(kb[0], b), path, int(w.ctx_lens[b]))
         assert int(dw.new_ctx[b]) == new_ctx
         assert np.array_equal(w.seq_view(ka[0], b)[:new_ctx], ref[:new_ctx])
+
+
+@pytest.mark.parametrize("base,tree,seed", [("llama3-8b-gqa", "binary", 3), ("llama3-8b-gqa", "branching", 5),
+                                            ("llama3-8b-gqa", "chain", 6), ("batched-paged", "random-depth", 4)])
+def test_step_verify_compact_on_eligible_trees(base, tree, seed):
+    """The step's fused verification + compaction on trees where most edges are eligible
+    (draft token = the parent's greedy token) and several paths tie in depth, so the
+    lexicographic choice and the compaction of a long path are exercised."""
+    over = dict(layers=2, ctx=(150, 150), vocab=64, tree=tree)
+    if tree in ("binary", "chain"):
+        over["nodes"] = (63, 63)
+    if base == "batched-paged":
+        over.update(batch=2, hq=8, hkv=2)
+    cfg = syn.shrink(syn.CONFIGS[base], **over)
+    w = syn.Workload(cfg, seed)
+    dw = DeviceWorkload(w)
+    idx_ref, _ = oracle.topk_rows(syn.widen(w.logits, cfg.dtype), cfg.k)
+    greedy = idx_ref[:, 0]
+    rng = np.random.default_rng(seed)
+    tokens = w.tokens.copy()
+    for b, par in enumerate(w.trees):
+        o = int(w.node_offsets[b])
+        for i in range(1, len(par)):
+            tokens[o + i] = greedy[o + par[i]] if rng.random() < 0.8 else int(rng.integers(cfg.vocab))
+    dw.tokens.copy_(torch.tensor(tokens, dtype=torch.int32))
+    k_before = dw.k.cpu().view(torch.int16).numpy()
+    assert dw.step() == 3
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == 0
+    ka = dw.k.cpu().view(torch.int16).numpy()
+    for b, par in enumerate(w.trees):
+        sl = w.nodes_of(b)
+        path, nacc, bonus = oracle.verify_greedy(par, tokens[sl], greedy[sl])
+        assert nacc > 2
+        assert int(dw.accept_len[b]) == nacc and int(dw.bonus[b]) == bonus
+        acc = dw.accepted[b].cpu().tolist()
+        assert acc[:nacc] == path and all(x == -1 for x in acc[nacc:])
+        for l in range(cfg.layers):
+            ref, new_ctx = oracle.kv_compact(w.seq_view(k_before[l], b), path, int(w.ctx_lens[b]))
+            assert int(dw.new_ctx[b]) == new_ctx
+            assert np.array_equal(w.seq_view(ka[l], b)[:new_ctx], ref[:new_ctx])
 
 
 def test_host_step_matches_device_step():
@@ -419,7 +506,7 @@ def test_host_step_matches_device_step():
     dw.q.zero_()
     dw.logits.zero_()
     n = ptd.tree_verify_step_host(dw.tree, dw.cache, dw.bufs, io)
-    assert n >= 4
+    assert n == 3                                    # attention, top-k, verify + compact
     torch.cuda.synchronize()
     idx_ref, _ = oracle.topk_rows(syn.widen(w.logits, cfg.dtype), cfg.k)
     assert np.array_equal(io_t["topk_idx_h"].numpy(), idx_ref)
