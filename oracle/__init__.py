@@ -11,9 +11,11 @@ from .ptd_oracle import (  # noqa: F401
     depths,
     eligible_edges,
     kv_compact,
+    softmax_row,
     topk,
     topk_rows,
     tree_attention,
     verify_greedy,
+    verify_sampling,
     visibility,
 )

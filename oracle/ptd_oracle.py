@@ -22,6 +22,9 @@ cites the passage it follows:
                                  X' = (n_0, ..., n_k, V_{n_k}); Alg. 1 steps 5-6.
   kv_compact ................... Alg. 1 step 6 (X' is appended to X): the accepted
                                  nodes' K/V become the next committed slots.
+  verify_sampling .............. Sec. 3.2, "sampling decoding strategy", and Alg. 2
+                                 (Candidate Tree Recursive Sampling), whose output
+                                 distribution App. E proves to be P.
 
 Readings where the paper is silent (each listed in the design notes):
   * node 0 of every tree is the current input token (slot C of the cache); draft
@@ -34,6 +37,16 @@ Readings where the paper is silent (each listed in the design notes):
     by the lexicographically smallest sequence of node indices;
   * accept_len counts accepted nodes including the root; the bonus token is
     V_{n_k} of the last accepted node.
+  * sampling verification: P_v = softmax(logits_v / temperature); each child of the
+    current node is tried once, in node order, with its own uniform r: accepted when
+    r < P(token)/S, S being the mass of P_v not yet rejected (Alg. 2 writes "<", the
+    text of Sec. 3.2 "<=": they differ on a set of measure zero); a rejected token's
+    probability becomes 0 (a later sibling with the same token then has probability
+    0).  Alg. 2 wraps this in "while C is not empty", which as printed never ends when
+    every child is rejected; App. E and Sec. 3.2 try each candidate once, as here.
+    With no child accepted (or at a leaf) the bonus token is drawn from the residual
+    P_v / S by inverse CDF in vocabulary order with the tree's own uniform.  The
+    uniforms are inputs, so the kernel and this oracle see the same random numbers.
 """
 from __future__ import annotations
 
@@ -187,6 +200,63 @@ def verify_greedy(parents, tokens, target):
 
     walk([0])
     return best, len(best), int(target[best[-1]])
+
+
+# ---------------------------------------------------------------------------
+# Sampling verification (Sec. 3.2 "sampling decoding strategy"; Alg. 2; App. E)
+# ---------------------------------------------------------------------------
+
+def softmax_row(logits_row, temperature: float = 1.0) -> np.ndarray:
+    """P_v: the target model's distribution over the next token at node v (Sec. 3.2),
+    softmax of the node's logits divided by the temperature, in float64."""
+    x = np.asarray(logits_row, dtype=np.float64) / float(temperature)
+    e = np.exp(x - x.max())
+    return e / e.sum()
+
+
+def verify_sampling(parents, tokens, logits, temperature, u_accept, u_bonus):
+    """Sampling verification of one tree (Alg. 2, Candidate Tree Recursive Sampling).
+
+    From the root, the children sigma(v) of the current node v are tried in node order;
+    child n is accepted when u_accept[n] < P_v[tokens[n]] / S, where S is the mass of P_v
+    not yet rejected; a rejected child's token gets probability 0 (P renormalised over
+    the rest).  An accepted child becomes the current node.  When no child is accepted
+    (or v is a leaf) the bonus token is drawn from the residual P_v / S by inverse CDF
+    with u_bonus.  logits: [T, V] rows of this tree.  Returns (path, accept_len, bonus,
+    margin) where margin is the smallest distance between a uniform and the threshold it
+    was compared with (acceptance tests and the bonus CDF), a measure of how far every
+    decision is from flipping."""
+    check_tree(parents)
+    sigma = children_sets(parents)
+    path = [0]
+    v = 0
+    margin = math.inf
+    while True:
+        P = softmax_row(logits[v], temperature)
+        S = 1.0
+        chosen = None
+        for n in sigma[v]:
+            t = int(tokens[n])
+            p_hat = P[t] / S if S > 0.0 else 0.0
+            r = float(u_accept[n])
+            margin = min(margin, abs(r - p_hat))
+            if r < p_hat:
+                chosen = n
+                break
+            S -= P[t]
+            P[t] = 0.0
+        if chosen is None:
+            break
+        path.append(chosen)
+        v = chosen
+    # no child selected: a sample from the residual distribution of the current node
+    target = float(u_bonus) * S
+    cdf = np.cumsum(P)
+    above = np.nonzero(cdf > target)[0]
+    bonus = int(above[0]) if len(above) else int(np.nonzero(P > 0.0)[0][-1])
+    lo = cdf[bonus - 1] if bonus > 0 else 0.0
+    margin = min(margin, abs(target - lo) / max(S, 1e-300), abs(cdf[bonus] - target) / max(S, 1e-300))
+    return path, len(path), bonus, margin
 
 
 # ---------------------------------------------------------------------------

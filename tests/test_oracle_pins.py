@@ -333,3 +333,107 @@ def test_compact_matches_gather_and_keeps_prefix():
         assert nc == C + len(path)
         assert np.array_equal(new[:C], cache[:C])
         assert np.array_equal(new[C:nc], cache[C + np.array(path)])
+
+
+# --------------------------------------------------------------------------- sampling verification
+
+def _chi2_pvalue(counts, probs):
+    """p-value of Pearson's chi-square statistic (library routine)."""
+    stats = pytest.importorskip("scipy.stats")
+    n = counts.sum()
+    keep = probs > 0
+    assert counts[~keep].sum() == 0            # a token of probability 0 is never emitted
+    return stats.chisquare(counts[keep], n * probs[keep] / probs[keep].sum()).pvalue
+
+
+def _emitted_first_token(parents, tokens, logits, u_acc, u_bon):
+    path, alen, bonus, _ = oracle.verify_sampling(parents, tokens, logits, 1.0, u_acc, u_bon)
+    return int(tokens[path[1]]) if alen > 1 else bonus
+
+
+def test_sampling_star_tree_emits_P():
+    """App. E: trying the candidates in order with renormalisation after each rejection,
+    and falling back to the residual, emits token i with probability exactly P_i.  The
+    candidate tokens include a repeat (its second copy has probability 0 once the first is
+    rejected)."""
+    g = np.random.default_rng(11)
+    V = 6
+    row = g.normal(0.0, 1.0, V)
+    P = oracle.softmax_row(row)
+    parents = [-1, 0, 0, 0, 0]
+    tokens = np.array([0, 2, 0, 2, 5])
+    logits = np.tile(row, (5, 1))
+    trials = 40000
+    counts = np.zeros(V, np.int64)
+    for _ in range(trials):
+        u = g.random(5)
+        counts[_emitted_first_token(parents, tokens, logits, u, g.random())] += 1
+    assert _chi2_pvalue(counts, P) > 1e-4
+    # and the acceptance of the first candidate is exactly P[token] (base case of App. E)
+    g2 = np.random.default_rng(12)
+    acc1 = sum(oracle.verify_sampling(parents, tokens, logits, 1.0, g2.random(5), 0.5)[0][1:2] == [1]
+               for _ in range(20000))
+    assert abs(acc1 / 20000 - P[2]) < 4 * math.sqrt(P[2] * (1 - P[2]) / 20000)
+
+
+def test_sampling_leaf_root_bonus_is_P_and_temperature():
+    g = np.random.default_rng(13)
+    V = 5
+    row = g.normal(0.0, 2.0, V)
+    for temp in (1.0, 0.5):
+        P = np.exp(row / temp - (row / temp).max())
+        P /= P.sum()
+        assert np.allclose(oracle.softmax_row(row, temp), P)
+        counts = np.zeros(V, np.int64)
+        for _ in range(30000):
+            counts[oracle.verify_sampling([-1], [3], row[None, :], temp, [0.0], g.random())[2]] += 1
+        assert _chi2_pvalue(counts, P) > 1e-4
+
+
+def test_sampling_one_hot_reduces_to_greedy():
+    """With all of P_v on argmax_v (a logit margin of 1e4) sampling accepts exactly the
+    children whose token is the parent's argmax, so it walks the greedy path (siblings
+    carry distinct tokens, as the workload generator guarantees)."""
+    g = np.random.default_rng(14)
+    V = 12
+    for _ in range(200):
+        T = int(g.integers(1, 40))
+        parents = [-1] + [int(g.integers(0, i)) for i in range(1, T)]
+        arg = g.integers(0, V, size=T)
+        logits = g.normal(0.0, 1.0, (T, V))
+        logits[np.arange(T), arg] += 1e4
+        tokens = np.zeros(T, np.int64)
+        for p, kids in enumerate(oracle.children_sets(parents)):
+            perm = g.permutation(V)
+            for j, c in enumerate(kids):   # distinct tokens among siblings, argmax[p] with probability 0.6
+                tokens[c] = arg[p] if (j == 0 and g.random() < 0.6) else perm[(j + 1) % V]
+        sig = oracle.children_sets(parents)
+        for p, kids in enumerate(sig):     # keep siblings distinct after the substitution
+            seen = set()
+            for c in kids:
+                while int(tokens[c]) in seen:
+                    tokens[c] = (tokens[c] + 1) % V
+                seen.add(int(tokens[c]))
+        path, alen, bonus, _ = oracle.verify_sampling(parents, tokens, logits, 1.0, g.random(T), g.random())
+        gpath, galen, gbonus = oracle.verify_greedy(parents, tokens, arg)
+        assert (path, alen, bonus) == (gpath, galen, gbonus)
+
+
+def test_sampling_invariants_on_random_trees():
+    """Every accepted edge had positive probability, the bonus is not a token rejected at
+    the last node and has positive probability, and the path fits in the tree."""
+    g = np.random.default_rng(15)
+    V = 20
+    for _ in range(300):
+        T = int(g.integers(1, 50))
+        parents = [-1] + [int(g.integers(0, i)) for i in range(1, T)]
+        logits = g.normal(0.0, 3.0, (T, V))
+        tokens = g.integers(0, 4, size=T)            # few distinct tokens: repeats among siblings
+        path, alen, bonus, margin = oracle.verify_sampling(parents, tokens, logits, 0.8, g.random(T), g.random())
+        assert alen == len(path) and path[0] == 0 and alen - 1 <= int(oracle.depths(parents).max())
+        for a, b in zip(path, path[1:]):
+            assert parents[b] == a and oracle.softmax_row(logits[a], 0.8)[tokens[b]] > 0
+        last = path[-1]
+        rejected = {int(tokens[c]) for c in oracle.children_sets(parents)[last]}
+        assert bonus not in rejected or len(rejected) == V
+        assert oracle.softmax_row(logits[last], 0.8)[bonus] > 0 and margin >= 0
