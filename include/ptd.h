@@ -14,7 +14,8 @@
  *   ptd_verify_greedy    eligible edges I and accepted sequence X' (Sec. 3.2)
  *   ptd_kv_compact       move the accepted nodes' K/V behind the prefix (Alg. 1 step 6)
  *
- * plus ptd_verify_and_compact (the last two as one launch) and ptd_tree_verify_step (the
+ * plus ptd_verify_sampling (verification under the sampling strategy, Alg. 2),
+ * ptd_verify_and_compact (the last two as one launch) and ptd_tree_verify_step (the
  * whole step: attention, top-k, verification and compaction on one stream)
  *
  * Conventions shared by every call
@@ -184,6 +185,27 @@ ptd_status ptd_verify_greedy(const ptd_tree* tree, const int32_t* tokens, const 
 ptd_status ptd_kv_compact(const ptd_tree* tree, const ptd_kv_cache* cache,
                           const int32_t* accepted_nodes, const int32_t* accept_len,
                           int32_t* new_ctx_lens, void* stream);
+
+/* Sampling verification (Sec. 3.2, "sampling decoding strategy"; Alg. 2, Candidate Tree
+ * Recursive Sampling; App. E proves that the emitted token follows P).  For every tree,
+ * from the root: P_v = softmax(logits_v / temperature); the children of the current node
+ * v are tried once each, in node order; child n is accepted when u_accept[n] <
+ * P_v(tokens[n]) / S, where S is the mass of P_v not yet rejected, and a rejected child's
+ * token gets probability 0 (a later sibling with the same token is then rejected too).
+ * An accepted child becomes the current node.  When no child is accepted (or at a leaf)
+ * the bonus token is the inverse CDF, in vocabulary order, of the residual P_v / S at
+ * u_bonus[b].  The random numbers are inputs, so the result is a function of them.
+ *   logits: rows of `vocab` entries, `row_stride` elements apart, one per node (dtype
+ *           bf16 or f32); temperature > 0.
+ *   u_accept: [N_tot] fp32 in [0, 1), the draw of node n's test (the root's is unused);
+ *   u_bonus: [B] fp32 in [0, 1), the draw of tree b's bonus token.
+ *   accepted_nodes, accept_len, bonus_token, dev_status: as in ptd_verify_greedy.
+ * Probabilities use fp32 exponentials and fp64 sums: a uniform within ~1e-6 of the
+ * probability it is compared with may decide either way. */
+ptd_status ptd_verify_sampling(const ptd_tree* tree, const int32_t* tokens, const void* logits, ptd_dtype dtype,
+                               int32_t vocab, int64_t row_stride, float temperature, const float* u_accept,
+                               const float* u_bonus, int32_t* accepted_nodes, int32_t* accept_len,
+                               int32_t* bonus_token, int32_t* dev_status, void* stream);
 
 /* ptd_verify_greedy followed by ptd_kv_compact, in one launch: the same outputs (accepted
  * path, accept length, bonus token, status, compacted cache, new context lengths) with the

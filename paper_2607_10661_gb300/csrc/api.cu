@@ -12,6 +12,7 @@
 #include <mutex>
 
 #include "../../include/ptd.h"
+#include "verify_sampling.cuh"
 #include "attention.cuh"
 #include "topk.cuh"
 #include "verify_compact.cuh"
@@ -285,6 +286,27 @@ ptd_status ptd_kv_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const
                                        cache->page_size, cache->seq_capacity, cache->num_pages, cache->block_table,
                                        cache->max_pages, tree->ctx_lens, accepted_nodes, accept_len,
                                        tree->max_nodes, new_ctx_lens, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+ptd_status ptd_verify_sampling(const ptd_tree* tree, const int32_t* tokens, const void* logits, ptd_dtype dtype,
+                               int32_t vocab, int64_t row_stride, float temperature, const float* u_accept,
+                               const float* u_bonus, int32_t* accepted_nodes, int32_t* accept_len,
+                               int32_t* bonus_token, int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  ptd_status st = check_tree(tree);
+  if (st != PTD_OK) return st;
+  if (!tokens || !logits || !u_accept || !u_bonus || !accepted_nodes || !accept_len || !bonus_token || !dev_status)
+    return PTD_ERR_INVALID_ARG;
+  if (dtype != PTD_BF16 && dtype != PTD_F32) return PTD_ERR_INVALID_ARG;
+  if (vocab < 1 || row_stride < vocab || !(temperature > 0.f) || !std::isfinite(temperature))
+    return PTD_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(logits) % dtype_size(dtype)) != 0) return PTD_ERR_INVALID_ARG;
+  st = cuda_status(ptd::launch_verify_sampling(tree->node_offsets, tree->parents, tokens, logits, dtype == PTD_BF16,
+                                               vocab, row_stride, 1.0f / temperature, u_accept, u_bonus, tree->batch,
+                                               tree->total_nodes, tree->max_nodes, accepted_nodes, accept_len,
+                                               bonus_token, dev_status, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }

@@ -25,7 +25,7 @@ MAX_TOPK = 16
 EXPORTED = (
     "ptd_attention_workspace_size", "ptd_tree_attention", "ptd_topk_draft", "ptd_verify_greedy",
     "ptd_kv_compact", "ptd_tree_verify_step", "ptd_tree_verify_step_host", "ptd_last_launch_count",
-    "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact",
+    "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact", "ptd_verify_sampling",
 )
 
 
@@ -92,6 +92,8 @@ def lib() -> ctypes.CDLL:
         L.ptd_verify_greedy.argtypes = [P(_Tree), vp, vp, i32, vp, vp, vp, vp, vp]
         L.ptd_kv_compact.restype = ctypes.c_int
         L.ptd_kv_compact.argtypes = [P(_Tree), P(_Cache), vp, vp, vp, vp]
+        L.ptd_verify_sampling.restype = ctypes.c_int
+        L.ptd_verify_sampling.argtypes = [P(_Tree), vp, vp, ctypes.c_int, i32, i64, f32, vp, vp, vp, vp, vp, vp, vp]
         L.ptd_verify_and_compact.restype = ctypes.c_int
         L.ptd_verify_and_compact.argtypes = [P(_Tree), P(_Cache), vp, vp, i32, vp, vp, vp, vp, vp, vp]
         L.ptd_tree_verify_step.restype = ctypes.c_int
@@ -233,6 +235,23 @@ def kv_compact(tree: Tree, cache: KVCache, accepted: torch.Tensor, accept_len: t
                               _dev(accept_len, "accept_len", torch.int32), _dev(new_ctx, "new_ctx", torch.int32),
                               _stream(stream))
     _check(st, "ptd_kv_compact")
+    return last_launch_count()
+
+
+def verify_sampling(tree: Tree, tokens: torch.Tensor, logits: torch.Tensor, temperature: float,
+                    u_accept: torch.Tensor, u_bonus: torch.Tensor, accepted: torch.Tensor, accept_len: torch.Tensor,
+                    bonus: torch.Tensor, dev_status: torch.Tensor, stream=None) -> int:
+    """ptd_verify_sampling; logits [N_tot, V] (bf16 or fp32), uniforms fp32."""
+    if logits.dim() != 2 or logits.stride(1) != 1:
+        raise ValueError("logits must be [rows, vocab] with unit column stride")
+    dt = BF16 if logits.dtype == torch.bfloat16 else F32
+    st = lib().ptd_verify_sampling(ctypes.byref(tree.c), _dev(tokens, "tokens", torch.int32),
+                                   _dev(logits, "logits", logits.dtype), dt, logits.shape[1], logits.stride(0),
+                                   float(temperature), _dev(u_accept, "u_accept", torch.float32),
+                                   _dev(u_bonus, "u_bonus", torch.float32), _dev(accepted, "accepted", torch.int32),
+                                   _dev(accept_len, "accept_len", torch.int32), _dev(bonus, "bonus", torch.int32),
+                                   _dev(dev_status, "dev_status", torch.int32), _stream(stream))
+    _check(st, "ptd_verify_sampling")
     return last_launch_count()
 
 

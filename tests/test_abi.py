@@ -57,6 +57,11 @@ def test_host_checks_reject_without_gpu(lib):
     assert lib.ptd_verify_greedy(None, null, null, 1, null, null, null, null, null) == ptd.INVALID_ARG
     assert lib.ptd_kv_compact(None, None, null, null, null, null) == ptd.INVALID_ARG
     assert lib.ptd_verify_and_compact(None, None, null, null, 1, null, null, null, null, null, null) == ptd.INVALID_ARG
+    t1 = ptd._Tree(1, 10, 10, 0, 8, 8, 8)
+    assert lib.ptd_verify_sampling(ctypes.byref(t1), 16, 16, ptd.BF16, 100, 100, 0.0, 16, 16, 16, 16, 16, 16,
+                                   None) == ptd.INVALID_ARG   # temperature must be > 0
+    assert lib.ptd_verify_sampling(ctypes.byref(t1), 16, None, ptd.BF16, 100, 100, 1.0, 16, 16, 16, 16, 16, 16,
+                                   None) == ptd.INVALID_ARG
     t = ptd._Tree(1, 200, 200, 0, 8, 8, 8)          # max_nodes above 128
     c = ptd._Cache(16, 16, ptd.BF16, 1, 8, 128, 0, 300, 0, None, 0)
     assert lib.ptd_tree_attention(ctypes.byref(t), ctypes.byref(c), 0, 1, 16, 32, 0.0, 16, None, 0, 16,

@@ -516,3 +516,90 @@ def test_host_step_matches_device_step():
     assert int(io_t["new_ctx_h"][0]) == C + nacc and int(io_t["status_h"][0]) == 0
     got = dw.attn_out.float().cpu().numpy()
     _check_attn(got[1], _attn_ref(w, 1, 0), "bf16", "host step")
+
+
+# ------------------------------------------------------------------------------ sampling verification
+
+SAMPLING_CASES = {
+    # name: (base config, overrides, temperature)
+    "llama3-full-vocab-peaked": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8)), 0.1),
+    "llama3-full-vocab-flat": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8)), 1.0),
+    "batched-3-trees": ("batched-paged", dict(batch=3, layers=1, ctx=(16, 32), vocab=32000, hq=8, hkv=2), 0.5),
+    "tiny-fp32": ("tiny-fp32", {}, 0.8),
+    "single-node": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8), vocab=5000, tree="chain", nodes=(1, 1)), 1.0),
+}
+MARGIN = 2e-6   # fp32 exponentials vs the oracle's float64: keep every decision this far from flipping
+
+
+def _sampling_inputs(w, temp, seed, u_scale=1.0):
+    """Tokens that are mostly the parent's argmax (long accepted paths at low temperature)
+    and uniforms whose every decision is at least MARGIN from its threshold."""
+    cfg = w.cfg
+    logits = syn.widen(w.logits, cfg.dtype)
+    arg = logits.argmax(axis=1)
+    g = np.random.default_rng(seed)
+    tokens = w.tokens.copy()
+    for b, par in enumerate(w.trees):
+        o = int(w.node_offsets[b])
+        for i in range(1, len(par)):
+            tokens[o + i] = arg[o + par[i]] if g.random() < 0.6 else int(g.integers(cfg.vocab))
+    u_acc = np.zeros(w.n_total, np.float32)
+    u_bon = np.zeros(cfg.batch, np.float32)
+    refs = []
+    for b, par in enumerate(w.trees):
+        sl = w.nodes_of(b)
+        for _ in range(200):
+            ua = (g.random(len(par)) * u_scale).astype(np.float32)
+            ub = np.float32(g.random())
+            ref = oracle.verify_sampling(par, tokens[sl], logits[sl], temp, ua.astype(np.float64), float(ub))
+            if ref[3] > MARGIN:
+                break
+        assert ref[3] > MARGIN
+        u_acc[sl] = ua
+        u_bon[b] = ub
+        refs.append(ref)
+    return tokens, u_acc, u_bon, refs
+
+
+@pytest.mark.parametrize("case", list(SAMPLING_CASES))
+def test_verify_sampling_matches_oracle(case):
+    base, over, temp = SAMPLING_CASES[case]
+    w = syn.Workload(syn.shrink(syn.CONFIGS[base], **over), 71)
+    dw = DeviceWorkload(w)
+    # peaked: acceptance uniforms in [0, 0.05) accept every child carrying its parent's argmax
+    tokens, u_acc, u_bon, refs = _sampling_inputs(w, temp, 72, 0.05 if case.endswith("peaked") else 1.0)
+    dw.tokens.copy_(torch.tensor(tokens, dtype=torch.int32))
+    dw.dev_status.zero_()
+    ua, ub = torch.tensor(u_acc, device="cuda"), torch.tensor(u_bon, device="cuda")
+    assert ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, temp, ua, ub, dw.accepted, dw.accept_len, dw.bonus,
+                               dw.dev_status) == 1
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == 0
+    acc = dw.accepted.cpu().numpy()
+    for b, (path, alen, bonus, _) in enumerate(refs):
+        assert int(dw.accept_len[b]) == alen, (case, b)
+        assert acc[b, :alen].tolist() == path and (acc[b, alen:] == -1).all()
+        assert int(dw.bonus[b]) == bonus, (case, b)
+    if case == "llama3-full-vocab-peaked":
+        assert max(r[1] for r in refs) >= 3     # long accepted paths are exercised
+
+
+def test_verify_sampling_invalid_tree_and_argument_checks():
+    w = syn.Workload(syn.shrink(syn.CONFIGS["batched-paged"], batch=2, layers=1, ctx=(16, 16), vocab=1000, hq=8,
+                                hkv=2), 73)
+    dw = DeviceWorkload(w)
+    bad = w.parents.copy()
+    bad[int(w.node_offsets[1]) + 3] = 7            # tree 1: a parent after its child
+    dw.parents.copy_(torch.tensor(bad))
+    dw.dev_status.zero_()
+    ua = torch.rand(w.n_total, device="cuda")
+    ub = torch.rand(2, device="cuda")
+    ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, 1.0, ua, ub, dw.accepted, dw.accept_len, dw.bonus,
+                        dw.dev_status)
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == ptd.INVALID_TREE
+    assert int(dw.accept_len[1]) == 0 and int(dw.bonus[1]) == -1 and (dw.accepted[1] == -1).all()
+    assert int(dw.accept_len[0]) >= 1                # the valid tree is still verified
+    with pytest.raises(RuntimeError):
+        ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, 0.0, ua, ub, dw.accepted, dw.accept_len, dw.bonus,
+                            dw.dev_status)
