@@ -167,6 +167,13 @@ def run_gpu(args, rank: int, world: int, dist):
     dw = DeviceWorkload(w, device=f"cuda:{local}")
     stream = torch.cuda.current_stream()
     nb = step_bytes(w)
+    sampling = args.verify == "sampling"
+    if sampling:
+        # Alg. 2 at temperature 1: the uniforms are inputs of the step, like the logits
+        gu = torch.Generator(device=f"cuda:{local}")
+        gu.manual_seed(5000 + rank)
+        u_acc = torch.rand(w.n_total, device=f"cuda:{local}", generator=gu)
+        u_bon = torch.rand(cfg.batch, device=f"cuda:{local}", generator=gu)
 
     def one_step(ev=None):
         n = 0
@@ -176,7 +183,12 @@ def run_gpu(args, rank: int, world: int, dist):
         if ev is not None:
             ev[1].record(stream)
         n += dw.topk()
-        n += dw.verify_and_compact()
+        if sampling:
+            n += ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, 1.0, u_acc, u_bon, dw.accepted, dw.accept_len,
+                                     dw.bonus, dw.dev_status)
+            n += dw.compact()
+        else:
+            n += dw.verify_and_compact()
         return n
 
     dw.dev_status.zero_()              # sticky status word: cleared once, read after the run
@@ -271,6 +283,7 @@ def run_gpu(args, rank: int, world: int, dist):
         "data": "synthetic (seeded N(0,1) Q/K/V, N(0,2) logits with a planted +6 token, random pruned tree)",
         "config": {"workload": _workload_desc(cfg), "batch": cfg.batch, "layers": cfg.layers,
                    "context": cfg.ctx[0], "tree_nodes": w.n_total, "vocab": cfg.vocab, "k": cfg.k,
+                   "verify": "sampling (Alg. 2, temperature 1)" if sampling else "greedy",
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 (%.2f GB read per step vs 129 MB L2)" % (nb["roofline"] / 1e9)},
         "step_roofline_bytes": nb["roofline"],
@@ -284,12 +297,13 @@ def run_gpu(args, rank: int, world: int, dist):
                      "tensor_tflops": round(flops / (attn_ms * 1e-3) / 1e12, 1)},
         "clocks": clocks,
         "e2e": {"value": round(world * Ke / (e2e_ms * 1e-3), 3), "unit": "steps/s", "steps": Ke,
-                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "status_ok": e2e_ok},
+                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "status_ok": e2e_ok,
+                "verify": "greedy (the host step call)"},
         "gpu_launches": int(launches),
         "status": ptd.status_string(status),
     }
     if rank == 0 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
+        out["cpu_baseline"] = cpu_baseline(args.cpu_seconds, sampling)
     return out
 
 
@@ -323,8 +337,12 @@ for i in range({warmup} + {steps}):
     t1 = time.time()
     idx, _ = oracle.topk(lg[i % w.n_total], cfg.k)
     t2 = time.time()
-    target = np.full(w.n_total, int(idx[0]), np.int64)
-    path, n, bonus = oracle.verify_greedy(w.trees[0], w.tokens, target)
+    if {sampling}:
+        g = np.random.default_rng(i)
+        path, n, bonus, _ = oracle.verify_sampling(w.trees[0], w.tokens, lg, 1.0, g.random(w.n_total), g.random())
+    else:
+        target = np.full(w.n_total, int(idx[0]), np.int64)
+        path, n, bonus = oracle.verify_greedy(w.trees[0], w.tokens, target)
     t3 = time.time()
     oracle.kv_compact(k if i % 2 == 0 else v, path, C)
     t4 = time.time()
@@ -340,11 +358,11 @@ SAMPLE_DESC = ("per sample: one of the 256 (layer, KV head) attention units, one
                "(BLAS pinned to one thread) and scaled by those counts to one full step")
 
 
-def oracle_samples(steps: int, warmup: int, budget_s: float):
+def oracle_samples(steps: int, warmup: int, budget_s: float, sampling: bool = False):
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
     code = _SAMPLE_CODE.format(root=ROOT, workload=WORKLOAD, budget=float(budget_s), steps=int(steps),
-                               warmup=int(warmup))
+                               warmup=int(warmup), sampling=bool(sampling))
     r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
                        timeout=budget_s * 4 + 300)
     if r.returncode != 0:
@@ -352,10 +370,10 @@ def oracle_samples(steps: int, warmup: int, budget_s: float):
     return json.loads(r.stdout.strip().splitlines()[-1])["per_step"]
 
 
-def cpu_baseline(budget_s: float) -> dict:
+def cpu_baseline(budget_s: float, sampling: bool = False) -> dict:
     """The oracle as it stands on a bounded sample of the workload (about budget_s of CPU)."""
     try:
-        per = oracle_samples(10000, 1, budget_s)
+        per = oracle_samples(10000, 1, budget_s, sampling)
     except Exception as e:  # reported, never fatal for the GPU line
         return {"value": None, "unit": "steps/s", "cores": 1, "kind": "oracle", "error": str(e)[-300:]}
     sec = float(np.mean(per))
@@ -370,7 +388,7 @@ def run_reference(args):
 
     cfg = syn.CONFIGS[WORKLOAD]
     try:
-        per = oracle_samples(args.steps, min(args.warmup, 1), 150.0)
+        per = oracle_samples(args.steps, min(args.warmup, 1), 150.0, args.verify == "sampling")
     except Exception as e:
         return {"impl": "reference", "unavailable": "oracle sample failed: " + str(e)[-200:]}
     sec = float(np.mean(per))
@@ -396,6 +414,8 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling captures)")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--verify", default="greedy", choices=["greedy", "sampling"],
+                    help="verification strategy of the step (Sec. 3.2): greedy, or sampling (Alg. 2)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
 

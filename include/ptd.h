@@ -200,8 +200,9 @@ ptd_status ptd_kv_compact(const ptd_tree* tree, const ptd_kv_cache* cache,
  *   u_accept: [N_tot] fp32 in [0, 1), the draw of node n's test (the root's is unused);
  *   u_bonus: [B] fp32 in [0, 1), the draw of tree b's bonus token.
  *   accepted_nodes, accept_len, bonus_token, dev_status: as in ptd_verify_greedy.
- * Probabilities use fp32 exponentials and fp64 sums: a uniform within ~1e-6 of the
- * probability it is compared with may decide either way. */
+ * Probabilities use fp32 exponentials, compensated fp32 sums over short runs of the
+ * vocabulary and fp64 sums across them: a uniform within ~1e-6 of the probability it is
+ * compared with may decide either way.  One thread-block cluster (up to 8 CTAs) per tree. */
 ptd_status ptd_verify_sampling(const ptd_tree* tree, const int32_t* tokens, const void* logits, ptd_dtype dtype,
                                int32_t vocab, int64_t row_stride, float temperature, const float* u_accept,
                                const float* u_bonus, int32_t* accepted_nodes, int32_t* accept_len,

@@ -118,12 +118,16 @@ def _check(status: int, where: str) -> None:
         raise PtdError(status, where)
 
 
-def _dev(t: torch.Tensor, name: str, dtype=None) -> int:
+def _dev(t: torch.Tensor, name: str, dtype=None, row_strided: bool = False) -> int:
+    """Device pointer of t; row_strided accepts a 2-D tensor whose rows are apart (unit column stride)."""
     if not isinstance(t, torch.Tensor):
         raise TypeError(f"{name} must be a torch.Tensor")
     if not t.is_cuda:
         raise ValueError(f"{name} must be a CUDA tensor")
-    if not t.is_contiguous():
+    if row_strided:
+        if t.dim() != 2 or t.stride(1) != 1 or t.stride(0) < t.shape[1]:
+            raise ValueError(f"{name} must be [rows, cols] with unit column stride")
+    elif not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     if dtype is not None and t.dtype != dtype:
         raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
@@ -246,7 +250,8 @@ def verify_sampling(tree: Tree, tokens: torch.Tensor, logits: torch.Tensor, temp
         raise ValueError("logits must be [rows, vocab] with unit column stride")
     dt = BF16 if logits.dtype == torch.bfloat16 else F32
     st = lib().ptd_verify_sampling(ctypes.byref(tree.c), _dev(tokens, "tokens", torch.int32),
-                                   _dev(logits, "logits", logits.dtype), dt, logits.shape[1], logits.stride(0),
+                                   _dev(logits, "logits", logits.dtype, row_strided=True), dt, logits.shape[1],
+                                   logits.stride(0),
                                    float(temperature), _dev(u_accept, "u_accept", torch.float32),
                                    _dev(u_bonus, "u_bonus", torch.float32), _dev(accepted, "accepted", torch.int32),
                                    _dev(accept_len, "accept_len", torch.int32), _dev(bonus, "bonus", torch.int32),

@@ -521,17 +521,27 @@ def test_host_step_matches_device_step():
 # ------------------------------------------------------------------------------ sampling verification
 
 SAMPLING_CASES = {
-    # name: (base config, overrides, temperature)
+    # name: (base config, overrides, temperature[, workload seed])
     "llama3-full-vocab-peaked": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8)), 0.1),
     "llama3-full-vocab-flat": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8)), 1.0),
     "batched-3-trees": ("batched-paged", dict(batch=3, layers=1, ctx=(16, 32), vocab=32000, hq=8, hkv=2), 0.5),
     "tiny-fp32": ("tiny-fp32", {}, 0.8),
     "single-node": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8), vocab=5000, tree="chain", nodes=(1, 1)), 1.0),
+    # a 4-CTA cluster, and rows that are not 16-byte aligned (scalar loads)
+    "odd-vocab-50001": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8), vocab=50001), 0.7),
+    # fp32 logits over a 5-CTA cluster with vector loads
+    "fp32-vocab-70000": ("tiny-fp32", dict(vocab=70000), 1.0),
+    # chunks longer than 32 logits (the kernel reads them from memory in pieces)
+    "vocab-200000": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8), vocab=200000), 1.0),
+    # acceptance uniforms in [0.5, 1) and a root row whose top token has P ~0.75 (workload
+    # seed 77): a child carrying it is rejected, leaving a small residual for its siblings
+    # and the bonus
+    "llama3-dominant-rejected": ("llama3-8b-gqa", dict(layers=1, ctx=(8, 8)), 0.2, 77),
 }
 MARGIN = 2e-6   # fp32 exponentials vs the oracle's float64: keep every decision this far from flipping
 
 
-def _sampling_inputs(w, temp, seed, u_scale=1.0):
+def _sampling_inputs(w, temp, seed, u_scale=1.0, u_lo=0.0):
     """Tokens that are mostly the parent's argmax (long accepted paths at low temperature)
     and uniforms whose every decision is at least MARGIN from its threshold."""
     cfg = w.cfg
@@ -549,7 +559,7 @@ def _sampling_inputs(w, temp, seed, u_scale=1.0):
     for b, par in enumerate(w.trees):
         sl = w.nodes_of(b)
         for _ in range(200):
-            ua = (g.random(len(par)) * u_scale).astype(np.float32)
+            ua = (u_lo + g.random(len(par)) * (u_scale - u_lo)).astype(np.float32)
             ub = np.float32(g.random())
             ref = oracle.verify_sampling(par, tokens[sl], logits[sl], temp, ua.astype(np.float64), float(ub))
             if ref[3] > MARGIN:
@@ -561,17 +571,27 @@ def _sampling_inputs(w, temp, seed, u_scale=1.0):
     return tokens, u_acc, u_bon, refs
 
 
-@pytest.mark.parametrize("case", list(SAMPLING_CASES))
-def test_verify_sampling_matches_oracle(case):
-    base, over, temp = SAMPLING_CASES[case]
-    w = syn.Workload(syn.shrink(syn.CONFIGS[base], **over), 71)
+def _run_sampling_case(case, pad=None):
+    base, over, temp, *seed = SAMPLING_CASES[case]
+    w = syn.Workload(syn.shrink(syn.CONFIGS[base], **over), seed[0] if seed else 71)
     dw = DeviceWorkload(w)
     # peaked: acceptance uniforms in [0, 0.05) accept every child carrying its parent's argmax
-    tokens, u_acc, u_bon, refs = _sampling_inputs(w, temp, 72, 0.05 if case.endswith("peaked") else 1.0)
+    for seed in range(72, 122):
+        tokens, u_acc, u_bon, refs = _sampling_inputs(w, temp, seed, 0.05 if case.endswith("peaked") else 1.0,
+                                                      0.5 if case.endswith("rejected") else 0.0)
+        # the dominant-rejected case takes the first draw that rejects a dominant token
+        if not case.endswith("rejected") or _max_rejected_p(w, tokens, temp, refs) > 0.5:
+            break
     dw.tokens.copy_(torch.tensor(tokens, dtype=torch.int32))
     dw.dev_status.zero_()
     ua, ub = torch.tensor(u_acc, device="cuda"), torch.tensor(u_bon, device="cuda")
-    assert ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, temp, ua, ub, dw.accepted, dw.accept_len, dw.bonus,
+    logits = dw.logits
+    if pad is not None:   # rows `pad` elements longer than the vocabulary, padding poisoned
+        wide = torch.full((logits.shape[0], logits.shape[1] + pad), 1e4, dtype=logits.dtype, device=logits.device)
+        wide[:, :logits.shape[1]] = logits
+        logits = wide[:, :logits.shape[1]]
+        assert logits.stride(0) == dw.logits.shape[1] + pad
+    assert ptd.verify_sampling(dw.tree, dw.tokens, logits, temp, ua, ub, dw.accepted, dw.accept_len, dw.bonus,
                                dw.dev_status) == 1
     torch.cuda.synchronize()
     assert int(dw.dev_status.item()) == 0
@@ -580,8 +600,42 @@ def test_verify_sampling_matches_oracle(case):
         assert int(dw.accept_len[b]) == alen, (case, b)
         assert acc[b, :alen].tolist() == path and (acc[b, alen:] == -1).all()
         assert int(dw.bonus[b]) == bonus, (case, b)
+    return w, tokens, temp, refs
+
+
+def _max_rejected_p(w, tokens, temp, refs):
+    """Largest P_v(token) among the children rejected along the oracle's decisions."""
+    logits = syn.widen(w.logits, w.cfg.dtype)
+    best = 0.0
+    for b, par in enumerate(w.trees):
+        o = int(w.node_offsets[b])
+        path = refs[b][0]
+        for i, v in enumerate(path):
+            P = oracle.softmax_row(logits[o + v], temp)
+            nxt = path[i + 1] if i + 1 < len(path) else None
+            for n in range(v + 1, len(par)):
+                if par[n] != v:
+                    continue
+                if n == nxt:
+                    break
+                best = max(best, float(P[int(tokens[o + n])]))
+    return best
+
+
+@pytest.mark.parametrize("case", list(SAMPLING_CASES))
+def test_verify_sampling_matches_oracle(case):
+    w, tokens, temp, refs = _run_sampling_case(case)
     if case == "llama3-full-vocab-peaked":
         assert max(r[1] for r in refs) >= 3     # long accepted paths are exercised
+    if case == "llama3-dominant-rejected":
+        assert _max_rejected_p(w, tokens, temp, refs) > 0.5   # a dominant token was rejected
+
+
+@pytest.mark.parametrize("pad", [8, 3])
+def test_verify_sampling_strided_rows(pad):
+    """Rows further apart than the vocabulary: with a pad of 8 they stay 16-byte aligned
+    (vector loads), with 3 they do not (scalar loads); the padding is never read."""
+    _run_sampling_case("llama3-full-vocab-flat", pad)
 
 
 def test_verify_sampling_invalid_tree_and_argument_checks():
