@@ -6,9 +6,11 @@ CPU-baseline / reference arm may import it.  The product path never does.
 from .ptd_oracle import (  # noqa: F401
     InvalidTree,
     ancestor_sets,
+    check_forest,
     check_tree,
     children_sets,
     depths,
+    draft_tree_update,
     eligible_edges,
     kv_compact,
     softmax_row,

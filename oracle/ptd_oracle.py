@@ -25,6 +25,10 @@ cites the passage it follows:
   verify_sampling .............. Sec. 3.2, "sampling decoding strategy", and Alg. 2
                                  (Candidate Tree Recursive Sampling), whose output
                                  distribution App. E proves to be P.
+  draft_tree_update ............ Sec. 3.1 "Progressive Expansion" (every node's draft
+                                 token joins the tree as its child), "Width Control"
+                                 and "Stepping Mechanism (Depth Control)"; Alg. 1
+                                 step 3 (expand, then StepAndPrune past d_max).
 
 Readings where the paper is silent (each listed in the design notes):
   * node 0 of every tree is the current input token (slot C of the cache); draft
@@ -47,6 +51,20 @@ Readings where the paper is silent (each listed in the design notes):
     With no child accepted (or at a leaf) the bonus token is drawn from the residual
     P_v / S by inverse CDF in vocabulary order with the tree's own uniform.  The
     uniforms are inputs, so the kernel and this oracle see the same random numbers.
+  * draft tree update: the draft tree is a forest of seed subtrees (a seed's parent
+    is -1; in a verification pass they hang below node 0) stored in creation order,
+    so a parent precedes its children and "earliest added" means "lowest index".
+    Expansion visits the nodes in index order and each node's draft tokens in rank
+    order (the first `expand` of its top-k row); a token equal to an existing
+    child's is that child (V is a set of (parent, token) nodes), not a new node;
+    width control caps a node's children at `width`; new nodes are appended in that
+    visiting order while the forest has fewer than `capacity` nodes.  Depth control
+    applies per seed subtree ("when a sub-tree exceeds a depth threshold"): depth
+    counts nodes on the longest seed-to-leaf path (a lone seed has depth 1); a
+    subtree deeper than d_max is replaced by the subtree of the seed's lowest-index
+    child, which becomes a seed; everything else under the old seed goes.  Pruning
+    runs once per step, after expansion (Alg. 1 step 3).  Survivors keep their
+    relative order.
 """
 from __future__ import annotations
 
@@ -272,3 +290,98 @@ def kv_compact(cache_seq, path, ctx_len: int):
     for j, n in enumerate(path):
         new[ctx_len + j] = snap[ctx_len + int(n)]
     return new, ctx_len + len(path)
+
+
+# ---------------------------------------------------------------------------
+# Draft tree update (Sec. 3.1 "Progressive Expansion", "Width Control",
+# "Stepping Mechanism"; Alg. 1 step 3)
+# ---------------------------------------------------------------------------
+
+def check_forest(parents) -> None:
+    """A forest in creation order: parents[i] = -1 (a seed) or 0 <= parents[i] < i."""
+    for i, p in enumerate(parents):
+        if not (p == -1 or 0 <= int(p) < i):
+            raise InvalidTree(f"node {i}: parent {p} is neither -1 nor an earlier node")
+
+
+def draft_tree_update(parents, tokens, drafts, expand: int, width: int, max_depth: int, capacity: int):
+    """One step of the draft forest's evolution: T^{t-1} -> T^t.
+
+    parents, tokens: the forest T^{t-1} (seeds have parent -1), creation order.
+    drafts[v]: node v's draft tokens in rank order (its top-k row); the first
+    `expand` are appended as children of v (Sec. 3.1: V^t = V^{t-1} U {d_v},
+    E^t = E^{t-1} U {(v, d_v)}), subject to width control (at most `width` children
+    per node) and to `capacity` nodes in all.  Then every seed subtree deeper than
+    `max_depth` is stepped (Alg. 1 StepAndPrune): its seed's earliest-added child
+    becomes the seed of what is kept, the rest of the subtree is pruned.
+
+    Returns (new_parents, new_tokens, new_depths, old_to_new) where new_depths[i] =
+    |pi(i)| in the new forest (the node's position offset, Sec. 3.1) and
+    old_to_new[j] is the new index of input node j, or -1 if it was pruned."""
+    check_forest(parents)
+    T = len(parents)
+    if T > capacity:
+        raise ValueError("the input forest is larger than the capacity")
+    par = [int(p) for p in parents]
+    tok = [int(t) for t in tokens]
+    origin = list(range(T))            # input index of each node, -1 for a new node
+
+    # ---- Step 3, expansion: every node appends its draft tokens as children
+    for v in range(T):
+        for r in range(expand):
+            d = int(drafts[v][r])
+            kids = [i for i in range(len(par)) if par[i] == v]
+            if any(tok[i] == d for i in kids):
+                continue                 # (v, d) is already in V
+            if len(kids) >= width or len(par) >= capacity:
+                continue                 # width control / no room
+            par.append(v)
+            tok.append(d)
+            origin.append(-1)
+
+    # ---- depth of every node: |pi(v)|
+    n = len(par)
+    depth = [0] * n
+    seed = [0] * n
+    for i in range(n):
+        depth[i] = 1 if par[i] == -1 else depth[par[i]] + 1
+        seed[i] = i if par[i] == -1 else seed[par[i]]
+
+    # ---- StepAndPrune: per seed subtree deeper than max_depth
+    keep = [True] * n
+    new_seed = {}
+    for s in range(n):
+        if par[s] != -1:
+            continue
+        sub_depth = max(depth[i] for i in range(n) if seed[i] == s)
+        if sub_depth <= max_depth:
+            continue
+        first_child = min(i for i in range(n) if par[i] == s)   # earliest added
+        new_seed[s] = first_child
+        for i in range(n):
+            if seed[i] != s:
+                continue
+            a = i                        # is first_child an ancestor of i (or i itself)?
+            while a != -1 and a != first_child:
+                a = par[a]
+            keep[i] = a == first_child
+
+    # ---- survivors, in order
+    new_index = [-1] * n
+    m = 0
+    for i in range(n):
+        if keep[i]:
+            new_index[i] = m
+            m += 1
+    new_par, new_tok, new_dep = [], [], []
+    for i in range(n):
+        if not keep[i]:
+            continue
+        p = par[i]
+        new_par.append(-1 if (p == -1 or not keep[p]) else new_index[p])
+        new_tok.append(tok[i])
+    for i in range(m):
+        new_dep.append(1 if new_par[i] == -1 else new_dep[new_par[i]] + 1)
+    old_to_new = [new_index[j] for j in range(T)]
+    return (np.array(new_par, np.int64), np.array(new_tok, np.int64), np.array(new_dep, np.int64),
+            np.array(old_to_new, np.int64))

@@ -437,3 +437,154 @@ def test_sampling_invariants_on_random_trees():
         rejected = {int(tokens[c]) for c in oracle.children_sets(parents)[last]}
         assert bonus not in rejected or len(rejected) == V
         assert oracle.softmax_row(logits[last], 0.8)[bonus] > 0 and margin >= 0
+
+
+# ---------------------------------------------------------------------------
+# Draft tree update (Sec. 3.1 Progressive Expansion, Width Control, Stepping
+# Mechanism; Alg. 1 step 3)
+# ---------------------------------------------------------------------------
+
+def test_draft_update_worked_examples():
+    for case in _load("draft_update_worked.json")["cases"]:
+        got = oracle.draft_tree_update(case["parents"], case["tokens"], case["drafts"], case["expand"],
+                                       case["width"], case["max_depth"], case["capacity"])
+        for name, arr in zip(("new_parents", "new_tokens", "new_depths", "old_to_new"), got):
+            assert arr.tolist() == case[name], (case["why"], name)
+
+
+class _TrieNode:
+    """A draft-forest node as a token-keyed trie entry with a creation stamp."""
+
+    def __init__(self, token, stamp, origin):
+        self.token, self.stamp, self.origin, self.kids = token, stamp, origin, []
+
+
+def _trie_update(parents, tokens, drafts, expand, width, max_depth, capacity):
+    """The same step written over nested trie objects instead of index arrays:
+    expansion walks the original nodes by stamp, a child is found by token, a stepped
+    subtree is re-rooted at kids[0] (its earliest stamp), and the survivors are
+    flattened by stamp."""
+    nodes = [_TrieNode(int(t), i, i) for i, t in enumerate(tokens)]
+    roots = []
+    for i, p in enumerate(parents):
+        (roots if p == -1 else nodes[p].kids).append(nodes[i])
+    count = len(nodes)
+    for v in list(nodes):
+        for d in drafts[v.origin][:expand]:
+            if any(c.token == int(d) for c in v.kids) or len(v.kids) >= width or count >= capacity:
+                continue
+            v.kids.append(_TrieNode(int(d), count, -1))
+            count += 1
+
+    def height(n):
+        return 1 + max((height(c) for c in n.kids), default=0)
+
+    roots = [r.kids[0] if height(r) > max_depth else r for r in roots]
+    out = []                                        # (stamp, node, parent node or None)
+
+    def collect(n, parent):
+        out.append((n.stamp, n, parent))
+        for c in n.kids:
+            collect(c, n)
+
+    for r in roots:
+        collect(r, None)
+    out.sort(key=lambda e: e[0])
+    index = {id(n): k for k, (_, n, _) in enumerate(out)}
+    new_par = [-1 if par is None else index[id(par)] for _, _, par in out]
+    new_tok = [n.token for _, n, _ in out]
+    new_dep = []
+    for k, p in enumerate(new_par):
+        new_dep.append(1 if p == -1 else new_dep[p] + 1)
+    old_to_new = [-1] * len(parents)
+    for k, (_, n, _) in enumerate(out):
+        if n.origin >= 0:
+            old_to_new[n.origin] = k
+    return new_par, new_tok, new_dep, old_to_new
+
+
+def _random_forest(g, T, n_tokens):
+    parents = []
+    for i in range(T):
+        parents.append(-1 if (i == 0 or g.random() < 0.15) else int(g.integers(0, i)))
+    tokens = []
+    kids_tokens = {}
+    for i, p in enumerate(parents):      # siblings carry distinct tokens, as in a trie
+        used = kids_tokens.setdefault(p, set()) if p >= 0 else set()
+        t = int(g.integers(0, n_tokens))
+        while t in used:
+            t = (t + 1) % n_tokens
+        used.add(t)
+        tokens.append(t)
+    return parents, tokens
+
+
+def test_draft_update_matches_trie_formulation():
+    g = np.random.default_rng(21)
+    for _ in range(600):
+        T = int(g.integers(1, 30))
+        parents, tokens = _random_forest(g, T, 12)
+        expand = int(g.integers(0, 4))
+        drafts = g.integers(0, 12, size=(T, 4))
+        width = int(g.integers(0, 5))
+        max_depth = int(g.integers(1, 8))
+        capacity = T + int(g.integers(0, 3 * T + 2))
+        got = oracle.draft_tree_update(parents, tokens, drafts, expand, width, max_depth, capacity)
+        want = _trie_update(parents, tokens, drafts, expand, width, max_depth, capacity)
+        for a, b in zip(got, want):
+            assert a.tolist() == list(b)
+
+
+def test_draft_update_invariants():
+    """The result is a forest in creation order; no subtree is deeper than d_max when the
+    input was within it; width and sibling-token distinctness are preserved; every kept
+    node's root-to-node token path is its old path, less the stepped seed's token."""
+    g = np.random.default_rng(22)
+    for _ in range(400):
+        T = int(g.integers(1, 40))
+        parents, tokens = _random_forest(g, T, 30)
+        dep = []
+        for p in parents:
+            dep.append(1 if p == -1 else dep[p] + 1)
+        max_depth = max(dep) + int(g.integers(0, 2))
+        width = 8
+        drafts = g.integers(0, 30, size=(T, 3))
+        new_par, new_tok, new_dep, o2n = oracle.draft_tree_update(parents, tokens, drafts, 2, width, max_depth, 128)
+        oracle.check_forest(new_par)
+        assert int(new_dep.max()) <= max_depth
+        for v in range(len(new_par)):
+            kids = [i for i in range(len(new_par)) if new_par[i] == v]
+            assert len(kids) <= width
+            assert len({int(new_tok[i]) for i in kids}) == len(kids)
+
+        def path(par, tok, i):
+            out = []
+            while i != -1:
+                out.append(int(tok[i]))
+                i = par[i]
+            return out[::-1]
+
+        for j, k in enumerate(o2n):
+            if k < 0:
+                continue
+            old, new = path(parents, tokens, j), path(list(new_par), new_tok, int(k))
+            assert old == new or old[1:] == new
+
+
+def test_draft_update_identity_and_sliding_window():
+    """With nothing to add and no depth limit the step is the identity; on a chain fed
+    the next token of a sequence every step, the stepping mechanism keeps exactly the
+    last d_max tokens (a sliding window, Sec. 3.1 and Fig. 3)."""
+    g = np.random.default_rng(23)
+    parents, tokens = _random_forest(g, 25, 9)
+    got = oracle.draft_tree_update(parents, tokens, np.zeros((25, 1), np.int64), 0, 4, 99, 64)
+    assert got[0].tolist() == parents and got[1].tolist() == tokens and got[3].tolist() == list(range(25))
+    seq = list(g.integers(0, 1000, size=40))
+    d_max = 6
+    par, tok = [-1], [int(seq[0])]
+    for step in range(1, 40):
+        drafts = [[tok[i + 1]] if i + 1 < len(tok) else [int(seq[step])] for i in range(len(tok))]
+        par, tok, dep, _ = oracle.draft_tree_update(par, tok, drafts, 1, 1, d_max, 64)
+        par, tok = par.tolist(), tok.tolist()
+        assert tok == [int(x) for x in seq[max(0, step + 1 - d_max):step + 1]]
+        assert par == [-1] + list(range(len(tok) - 1)) and dep.tolist() == list(range(1, len(tok) + 1))
