@@ -174,6 +174,16 @@ def run_gpu(args, rank: int, world: int, dist):
         gu.manual_seed(5000 + rank)
         u_acc = torch.rand(w.n_total, device=f"cuda:{local}", generator=gu)
         u_bon = torch.rand(cfg.batch, device=f"cuda:{local}", generator=gu)
+    if args.draft_update:
+        # the step's tree as a one-seed draft forest, grown by every node's top-1 (width 4,
+        # depth 6: the paper's best setting); the output is the next step's draft tree
+        if cfg.batch != 1:
+            raise SystemExit("--draft-update times the one-tree workload only")
+        du_dev = f"cuda:{local}"
+        du_cnt = torch.tensor([w.n_total], dtype=torch.int32, device=du_dev)
+        du_out = [torch.empty((1,), dtype=torch.int32, device=du_dev)] + \
+                 [torch.empty((1, ptd.MAX_TREE_NODES), dtype=torch.int32, device=du_dev) for _ in range(3)] + \
+                 [torch.empty((1, w.n_total), dtype=torch.int32, device=du_dev)]
 
     def one_step(ev=None):
         n = 0
@@ -183,6 +193,9 @@ def run_gpu(args, rank: int, world: int, dist):
         if ev is not None:
             ev[1].record(stream)
         n += dw.topk()
+        if args.draft_update:
+            n += ptd.draft_tree_update(du_cnt, dw.parents.view(1, -1), dw.tokens.view(1, -1), dw.topk_idx, 1, 4, 6,
+                                       ptd.MAX_TREE_NODES, *du_out, dw.dev_status)
         if sampling:
             n += ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, 1.0, u_acc, u_bon, dw.accepted, dw.accept_len,
                                      dw.bonus, dw.dev_status)
@@ -284,6 +297,7 @@ def run_gpu(args, rank: int, world: int, dist):
         "config": {"workload": _workload_desc(cfg), "batch": cfg.batch, "layers": cfg.layers,
                    "context": cfg.ctx[0], "tree_nodes": w.n_total, "vocab": cfg.vocab, "k": cfg.k,
                    "verify": "sampling (Alg. 2, temperature 1)" if sampling else "greedy",
+                   "draft_update": "top-1 expansion, width 4, depth 6 (Alg. 1 step 3)" if args.draft_update else None,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 (%.2f GB read per step vs 129 MB L2)" % (nb["roofline"] / 1e9)},
         "step_roofline_bytes": nb["roofline"],
@@ -414,6 +428,8 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling captures)")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--draft-update", action="store_true",
+                    help="add the draft tree update (Sec. 3.1 expansion and depth control) to every step")
     ap.add_argument("--verify", default="greedy", choices=["greedy", "sampling"],
                     help="verification strategy of the step (Sec. 3.2): greedy, or sampling (Alg. 2)")
     args = ap.parse_args()

@@ -15,6 +15,7 @@
  *   ptd_kv_compact       move the accepted nodes' K/V behind the prefix (Alg. 1 step 6)
  *
  * plus ptd_verify_sampling (verification under the sampling strategy, Alg. 2),
+ * ptd_draft_tree_update (the draft forest's expansion and depth control, Alg. 1 step 3),
  * ptd_verify_and_compact (the last two as one launch) and ptd_tree_verify_step (the
  * whole step: attention, top-k, verification and compaction on one stream)
  *
@@ -217,6 +218,36 @@ ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cach
                                   const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
                                   int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
                                   int32_t* dev_status, void* stream);
+
+/* Draft tree update: one step of the draft forest's evolution T^{t-1} -> T^t (Sec. 3.1
+ * "Progressive Expansion": every node's draft token joins the tree as its child,
+ * V^t = V^{t-1} U {d_v}, E^t = E^{t-1} U {(v, d_v)}; "Width Control"; "Stepping Mechanism
+ * (Depth Control)"; Alg. 1 step 3: expand, then StepAndPrune past d_max).
+ *
+ * A draft forest is a set of seed subtrees in creation order: parents[i] = -1 (a seed) or
+ * 0 <= parents[i] < i, so "earliest added" is "lowest index".  Forest b's input nodes are
+ * in_parents / in_tokens [b * in_stride, b * in_stride + in_count[b]) (device); its output
+ * goes to out_parents / out_tokens / out_depths [b * capacity, (b + 1) * capacity), the
+ * first out_count[b] entries valid and the rest -1.
+ *   Expansion: node v, in index order, tries the first `expand` (<= 16) tokens of its draft
+ *   row drafts[(b * in_stride + v) * draft_stride ..] (a top-k row), in rank order; a token
+ *   equal to an existing child's token is that child (nothing is added); otherwise a new
+ *   child is appended while v has fewer than `width` children and the forest fewer than
+ *   `capacity` (<= PTD_MAX_TREE_NODES) nodes.
+ *   Depth control: depth counts nodes on a seed-to-leaf path (a lone seed has depth 1);
+ *   a seed subtree deeper than `max_depth` (>= 1) keeps only the subtree of the seed's
+ *   lowest-index child, which becomes a seed; the rest of it is dropped.  Once per call.
+ *   Survivors keep their relative order; out_depths[i] = |pi(i)| in the new forest (the
+ *   node's position offset, Sec. 3.1); old_to_new[b * in_stride + j] is the new index of
+ *   input node j, or -1 (also for j >= in_count[b]).
+ * A forest that is not one (a parent that is neither -1 nor earlier, in_count[b] < 0 or
+ * above in_stride or capacity) sets PTD_ERR_INVALID_TREE in dev_status and gets
+ * out_count[b] = 0.  Outputs must not alias inputs.  One launch, one CTA per forest. */
+ptd_status ptd_draft_tree_update(int32_t batch, int32_t in_stride, const int32_t* in_count, const int32_t* in_parents,
+                                 const int32_t* in_tokens, const int32_t* drafts, int32_t draft_stride, int32_t expand,
+                                 int32_t width, int32_t max_depth, int32_t capacity, int32_t* out_count,
+                                 int32_t* out_parents, int32_t* out_tokens, int32_t* out_depths, int32_t* old_to_new,
+                                 int32_t* dev_status, void* stream);
 
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.

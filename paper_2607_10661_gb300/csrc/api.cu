@@ -13,6 +13,7 @@
 
 #include "../../include/ptd.h"
 #include "verify_sampling.cuh"
+#include "draft_update.cuh"
 #include "attention.cuh"
 #include "topk.cuh"
 #include "verify_compact.cuh"
@@ -329,6 +330,28 @@ ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cach
       accepted_nodes, accept_len, bonus_token, dev_status, cache->k, cache->v, row_bytes, cache->num_layers,
       tree->batch, cache->page_size, cache->seq_capacity, cache->num_pages, cache->block_table, cache->max_pages,
       tree->ctx_lens, new_ctx_lens, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+ptd_status ptd_draft_tree_update(int32_t batch, int32_t in_stride, const int32_t* in_count, const int32_t* in_parents,
+                                 const int32_t* in_tokens, const int32_t* drafts, int32_t draft_stride, int32_t expand,
+                                 int32_t width, int32_t max_depth, int32_t capacity, int32_t* out_count,
+                                 int32_t* out_parents, int32_t* out_tokens, int32_t* out_depths, int32_t* old_to_new,
+                                 int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  if (batch < 1 || batch > 65535 || in_stride < 1 || capacity < 1 || capacity > PTD_MAX_TREE_NODES ||
+      expand < 0 || expand > ptd::kMaxExpand || draft_stride < 1 || expand > draft_stride || width < 0 ||
+      max_depth < 1)
+    return PTD_ERR_INVALID_ARG;
+  if (!in_count || !in_parents || !in_tokens || !drafts || !out_count || !out_parents || !out_tokens ||
+      !out_depths || !old_to_new || !dev_status)
+    return PTD_ERR_INVALID_ARG;
+  // the output must not alias the input (other threads of the CTA still read it)
+  if (out_parents == in_parents || out_tokens == in_tokens || out_count == in_count) return PTD_ERR_INVALID_ARG;
+  const ptd_status st = cuda_status(ptd::launch_draft_update(
+      batch, in_stride, in_count, in_parents, in_tokens, drafts, draft_stride, expand, width, max_depth, capacity,
+      out_count, out_parents, out_tokens, out_depths, old_to_new, dev_status, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }

@@ -21,11 +21,13 @@ OK, INVALID_ARG, INVALID_TREE, UNSUPPORTED, CUDA_ERROR, TIMEOUT, WORKSPACE = ran
 F32, BF16 = 0, 1
 MAX_TREE_NODES = 128
 MAX_TOPK = 16
+MAX_EXPAND = 16
 
 EXPORTED = (
     "ptd_attention_workspace_size", "ptd_tree_attention", "ptd_topk_draft", "ptd_verify_greedy",
     "ptd_kv_compact", "ptd_tree_verify_step", "ptd_tree_verify_step_host", "ptd_last_launch_count",
     "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact", "ptd_verify_sampling",
+    "ptd_draft_tree_update",
 )
 
 
@@ -96,6 +98,9 @@ def lib() -> ctypes.CDLL:
         L.ptd_verify_sampling.argtypes = [P(_Tree), vp, vp, ctypes.c_int, i32, i64, f32, vp, vp, vp, vp, vp, vp, vp]
         L.ptd_verify_and_compact.restype = ctypes.c_int
         L.ptd_verify_and_compact.argtypes = [P(_Tree), P(_Cache), vp, vp, i32, vp, vp, vp, vp, vp, vp]
+        L.ptd_draft_tree_update.restype = ctypes.c_int
+        L.ptd_draft_tree_update.argtypes = [i32, i32, vp, vp, vp, vp, i32, i32, i32, i32, i32, vp, vp, vp, vp, vp,
+                                            vp, vp]
         L.ptd_tree_verify_step.restype = ctypes.c_int
         L.ptd_tree_verify_step.argtypes = [P(_Tree), P(_Cache), P(_StepArgs), vp]
         L.ptd_tree_verify_step_host.restype = ctypes.c_int
@@ -316,4 +321,29 @@ def tree_verify_step_host(tree: Tree, cache: KVCache, bufs: StepBuffers, io: Hos
     st = lib().ptd_tree_verify_step_host(ctypes.byref(tree.c), ctypes.byref(cache.c), ctypes.byref(bufs.c),
                                          ctypes.byref(io.c), _stream(stream))
     _check(st, "ptd_tree_verify_step_host")
+    return last_launch_count()
+
+
+def draft_tree_update(in_count: torch.Tensor, in_parents: torch.Tensor, in_tokens: torch.Tensor,
+                      drafts: torch.Tensor, expand: int, width: int, max_depth: int, capacity: int,
+                      out_count: torch.Tensor, out_parents: torch.Tensor, out_tokens: torch.Tensor,
+                      out_depths: torch.Tensor, old_to_new: torch.Tensor, dev_status: torch.Tensor, stream=None) -> int:
+    """ptd_draft_tree_update.  in_parents / in_tokens / old_to_new: [B, in_stride] int32;
+    drafts: [B * in_stride, draft_stride] int32 (a top-k index matrix); out_*: [B, capacity] int32."""
+    if in_parents.dim() != 2 or in_tokens.shape != in_parents.shape or old_to_new.shape != in_parents.shape:
+        raise ValueError("in_parents, in_tokens and old_to_new must be [batch, in_stride]")
+    B, stride = in_parents.shape
+    if drafts.dim() != 2 or drafts.shape[0] != B * stride:
+        raise ValueError("drafts must be [batch * in_stride, draft_stride]")
+    for t, nm in ((out_parents, "out_parents"), (out_tokens, "out_tokens"), (out_depths, "out_depths")):
+        if tuple(t.shape) != (B, capacity):
+            raise ValueError(f"{nm} must be [batch, capacity]")
+    st = lib().ptd_draft_tree_update(
+        B, stride, _dev(in_count, "in_count", torch.int32), _dev(in_parents, "in_parents", torch.int32),
+        _dev(in_tokens, "in_tokens", torch.int32), _dev(drafts, "drafts", torch.int32), drafts.shape[1],
+        int(expand), int(width), int(max_depth), int(capacity), _dev(out_count, "out_count", torch.int32),
+        _dev(out_parents, "out_parents", torch.int32), _dev(out_tokens, "out_tokens", torch.int32),
+        _dev(out_depths, "out_depths", torch.int32), _dev(old_to_new, "old_to_new", torch.int32),
+        _dev(dev_status, "dev_status", torch.int32), _stream(stream))
+    _check(st, "ptd_draft_tree_update")
     return last_launch_count()

@@ -62,6 +62,19 @@ def test_host_checks_reject_without_gpu(lib):
                                    None) == ptd.INVALID_ARG   # temperature must be > 0
     assert lib.ptd_verify_sampling(ctypes.byref(t1), 16, None, ptd.BF16, 100, 100, 1.0, 16, 16, 16, 16, 16, 16,
                                    None) == ptd.INVALID_ARG
+    # draft tree update: capacity above 128, expand above the draft row, aliased output, null pointer
+    du = lambda **k: lib.ptd_draft_tree_update(
+        k.get("batch", 1), 8, 16, k.get("inp", 32), 48, 64, k.get("dstride", 4), k.get("expand", 1), 4,
+        k.get("max_depth", 6), k.get("capacity", 64), 80, k.get("outp", 96), 112, 128, 144, k.get("status", 160),
+        None)
+    assert du(capacity=129) == ptd.INVALID_ARG
+    assert du(capacity=0) == ptd.INVALID_ARG
+    assert du(expand=5, dstride=4) == ptd.INVALID_ARG
+    assert du(expand=17, dstride=32) == ptd.INVALID_ARG
+    assert du(max_depth=0) == ptd.INVALID_ARG
+    assert du(batch=0) == ptd.INVALID_ARG
+    assert du(outp=32) == ptd.INVALID_ARG
+    assert du(status=None) == ptd.INVALID_ARG
     t = ptd._Tree(1, 200, 200, 0, 8, 8, 8)          # max_nodes above 128
     c = ptd._Cache(16, 16, ptd.BF16, 1, 8, 128, 0, 300, 0, None, 0)
     assert lib.ptd_tree_attention(ctypes.byref(t), ctypes.byref(c), 0, 1, 16, 32, 0.0, 16, None, 0, 16,
