@@ -4,6 +4,7 @@ Test infrastructure: only the tests, `__graft_entry__.smoke()` and `bench.py`'s
 CPU-baseline / reference arm may import it.  The product path never does.
 """
 from .ptd_oracle import (  # noqa: F401
+    CandidatePool,
     InvalidTree,
     ancestor_sets,
     check_forest,

@@ -29,6 +29,10 @@ cites the passage it follows:
                                  token joins the tree as its child), "Width Control"
                                  and "Stepping Mechanism (Depth Control)"; Alg. 1
                                  step 3 (expand, then StepAndPrune past d_max).
+  CandidatePool ................ Sec. 3.1 "Draft Extraction via Merging" (the merge
+                                 M(T, T') of two trees with the same root value) and
+                                 Alg. 1 step 4; Sec. 3.2 and Alg. 1 step 1 (retrieve
+                                 the candidate tree C_X for the decoded sequence X).
 
 Readings where the paper is silent (each listed in the design notes):
   * node 0 of every tree is the current input token (slot C of the cache); draft
@@ -65,6 +69,19 @@ Readings where the paper is silent (each listed in the design notes):
     child, which becomes a seed; everything else under the old seed goes.  Pruning
     runs once per step, after expansion (Alg. 1 step 3).  Survivors keep their
     relative order.
+  * candidate pool: a map from a root token to a trie of draft continuations.  The
+    merge M is read as the union of tries: a child of T' whose token is not among the
+    children of T joins T together with its whole subtree (the printed case adds the
+    child node; its subtree follows by applying the same rule below it), and a child
+    whose token is there is merged recursively.  "Any subtree T' of T^t" is every
+    node's subtree: after each step, for every node v of the draft forest in index
+    order, the subtree rooted at v is merged into the pool entry of token(v) (created
+    when absent).  Children keep their order of insertion.  Retrieval for the decoded
+    sequence X takes the entry of X's last token (the current input token, node 0 of
+    the verification pass) and lays it out breadth first: at most `width` children per
+    node, the earliest inserted first, nodes of depth at most `max_depth` (the root
+    has depth 1), at most `max_nodes` nodes in that order.  A token with no entry
+    gives the lone root.
 """
 from __future__ import annotations
 
@@ -385,3 +402,74 @@ def draft_tree_update(parents, tokens, drafts, expand: int, width: int, max_dept
     old_to_new = [new_index[j] for j in range(T)]
     return (np.array(new_par, np.int64), np.array(new_tok, np.int64), np.array(new_dep, np.int64),
             np.array(old_to_new, np.int64))
+
+
+# ---------------------------------------------------------------------------
+# Candidate pool (Sec. 3.1 "Draft Extraction via Merging"; Sec. 3.2; Alg. 1 steps 1, 4)
+# ---------------------------------------------------------------------------
+
+class _PoolNode:
+    __slots__ = ("token", "children")
+
+    def __init__(self, token: int):
+        self.token = token
+        self.children = []            # insertion order
+
+
+class CandidatePool:
+    """Root token -> trie of draft continuations."""
+
+    def __init__(self):
+        self.roots = {}
+
+    def size(self) -> int:
+        """Nodes held (roots included)."""
+        def count(n):
+            return 1 + sum(count(c) for c in n.children)
+        return sum(count(r) for r in self.roots.values())
+
+    def _merge(self, pnode, parents, tokens, kids, v):
+        """M(P, T'_v): merge the children of draft node v under pool node pnode."""
+        for c in kids[v]:
+            tok = int(tokens[c])
+            match = next((x for x in pnode.children if x.token == tok), None)
+            if match is None:                  # sigma(T') \ sigma(T): joins with its subtree
+                match = _PoolNode(tok)
+                pnode.children.append(match)
+            self._merge(match, parents, tokens, kids, c)   # sigma(T') n sigma(T): recurse
+
+    def merge_forest(self, parents, tokens) -> None:
+        """Alg. 1 step 4: every node's subtree of the draft forest T^t joins the pool
+        entry of its root token, nodes in index order."""
+        check_forest(parents)
+        kids = [[] for _ in parents]
+        for i, p in enumerate(parents):
+            if p >= 0:
+                kids[p].append(i)
+        for v in range(len(parents)):
+            tok = int(tokens[v])
+            if tok not in self.roots:
+                self.roots[tok] = _PoolNode(tok)
+            self._merge(self.roots[tok], parents, tokens, kids, v)
+
+    def retrieve(self, root_token: int, width: int, max_depth: int, max_nodes: int):
+        """Alg. 1 step 1: the candidate tree C_X for a sequence whose last token is
+        root_token, breadth first (parents, tokens), node 0 the root."""
+        root = self.roots.get(int(root_token))
+        parents, tokens = [-1], [int(root_token)]
+        if root is None:
+            return np.array(parents, np.int64), np.array(tokens, np.int64)
+        frontier = [(root, 0)]                 # (pool node, its index in the output)
+        depth = 1
+        while frontier and depth < max_depth and len(tokens) < max_nodes:
+            nxt = []
+            for node, idx in frontier:
+                for c in node.children[:width]:
+                    if len(tokens) >= max_nodes:
+                        break
+                    parents.append(idx)
+                    tokens.append(c.token)
+                    nxt.append((c, len(tokens) - 1))
+            frontier = nxt
+            depth += 1
+        return np.array(parents, np.int64), np.array(tokens, np.int64)

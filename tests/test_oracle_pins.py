@@ -588,3 +588,104 @@ def test_draft_update_identity_and_sliding_window():
         par, tok = par.tolist(), tok.tolist()
         assert tok == [int(x) for x in seq[max(0, step + 1 - d_max):step + 1]]
         assert par == [-1] + list(range(len(tok) - 1)) and dep.tolist() == list(range(1, len(tok) + 1))
+
+
+# ---------------------------------------------------------------------------
+# Candidate pool (Sec. 3.1 "Draft Extraction via Merging"; Sec. 3.2; Alg. 1 steps 1, 4)
+# ---------------------------------------------------------------------------
+
+def test_pool_worked_example():
+    gold = _load("candidate_pool_worked.json")
+    pool = oracle.CandidatePool()
+    for step in gold["steps"]:
+        pool.merge_forest(step["parents"], step["tokens"])
+        assert pool.size() == step["pool_size"], step["why"]
+        for r in step["retrieve"]:
+            par, tok = pool.retrieve(r["root"], r["width"], r["max_depth"], r["max_nodes"])
+            assert par.tolist() == r["parents"] and tok.tolist() == r["tokens"], (step["why"], r)
+
+
+def _path_set_pool(forests):
+    """The pool as a set of token paths with first-insertion keys: every (v, u) pair with u
+    in v's subtree inserts the path token(v) .. token(u); a path first inserted at step s by
+    the pair (v, u) gets the key (s, v, u)."""
+    first = {}
+    for s, (parents, tokens) in enumerate(forests):
+        for u in range(len(parents)):
+            chain = []
+            a = u
+            while a != -1:
+                chain.append(a)
+                a = parents[a]
+            chain.reverse()                    # seed .. u
+            for k, v in enumerate(chain):
+                path = tuple(int(tokens[x]) for x in chain[k:])
+                first[path] = min(first.get(path, (s, v, u)), (s, v, u))
+    return first
+
+
+def _path_set_retrieve(first, root, width, max_depth, max_nodes):
+    """Breadth-first over the path set: the children of a path are its one-token
+    extensions, the `width` smallest first-insertion keys first."""
+    if (root,) not in first:
+        return [-1], [root]
+    ext_of = {}
+    for path, key in first.items():
+        if len(path) > 1:
+            ext_of.setdefault(path[:-1], []).append((key, path))
+    parents, tokens, paths = [-1], [root], [(root,)]
+    frontier, depth = [0], 1
+    while frontier and depth < max_depth and len(tokens) < max_nodes:
+        nxt = []
+        for idx in frontier:
+            p = paths[idx]
+            ext = sorted(ext_of.get(p, []))
+            for _, path in ext[:width]:
+                if len(tokens) >= max_nodes:
+                    break
+                parents.append(idx)
+                tokens.append(path[-1])
+                paths.append(path)
+                nxt.append(len(tokens) - 1)
+        frontier, depth = nxt, depth + 1
+    return parents, tokens
+
+
+def test_pool_matches_path_set_formulation():
+    g = np.random.default_rng(31)
+    for _ in range(40):
+        pool = oracle.CandidatePool()
+        forests = []
+        for step in range(int(g.integers(1, 6))):
+            parents, tokens = _random_forest(g, int(g.integers(1, 25)), 6)
+            pool.merge_forest(parents, tokens)
+            forests.append((parents, tokens))
+            first = _path_set_pool(forests)
+            assert pool.size() == len(first)
+            for root in range(7):
+                width, max_depth, max_nodes = int(g.integers(1, 5)), int(g.integers(1, 7)), int(g.integers(1, 40))
+                par, tok = pool.retrieve(root, width, max_depth, max_nodes)
+                want = _path_set_retrieve(first, root, width, max_depth, max_nodes)
+                assert (par.tolist(), tok.tolist()) == want
+
+
+def test_pool_idempotent_and_chain():
+    """Merging the same forest again adds nothing; a chain t1..tn gives every ti an entry
+    holding the rest of the chain."""
+    g = np.random.default_rng(32)
+    parents, tokens = _random_forest(g, 30, 8)
+    pool = oracle.CandidatePool()
+    pool.merge_forest(parents, tokens)
+    size = pool.size()
+    before = [pool.retrieve(r, 3, 5, 50) for r in range(8)]
+    pool.merge_forest(parents, tokens)
+    assert pool.size() == size
+    for r in range(8):
+        a, b = before[r], pool.retrieve(r, 3, 5, 50)
+        assert a[0].tolist() == b[0].tolist() and a[1].tolist() == b[1].tolist()
+    seq = [int(x) for x in g.permutation(100)[:12]]
+    chain = oracle.CandidatePool()
+    chain.merge_forest([-1] + list(range(11)), seq)
+    for i, t in enumerate(seq):
+        par, tok = chain.retrieve(t, 4, 99, 99)
+        assert tok.tolist() == seq[i:] and par.tolist() == [-1] + list(range(len(seq) - i - 1))
