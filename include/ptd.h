@@ -16,6 +16,8 @@
  *
  * plus ptd_verify_sampling (verification under the sampling strategy, Alg. 2),
  * ptd_draft_tree_update (the draft forest's expansion and depth control, Alg. 1 step 3),
+ * ptd_pool_* (the candidate pool: merge of the draft subtrees and retrieval of the
+ * candidate tree, Alg. 1 steps 4 and 1),
  * ptd_verify_and_compact (the last two as one launch) and ptd_tree_verify_step (the
  * whole step: attention, top-k, verification and compaction on one stream)
  *
@@ -56,7 +58,8 @@ typedef enum {
   PTD_ERR_UNSUPPORTED = 3,   /* valid but not implemented (dtype / head_dim combination)  */
   PTD_ERR_CUDA = 4,          /* a CUDA runtime call or kernel launch failed              */
   PTD_ERR_TIMEOUT = 5,       /* (device) a bounded on-chip wait gave up; outputs invalid  */
-  PTD_ERR_WORKSPACE = 6      /* workspace pointer null or smaller than required          */
+  PTD_ERR_WORKSPACE = 6,     /* workspace pointer null or smaller than required          */
+  PTD_ERR_POOL_FULL = 7      /* (device) a candidate-pool merge was refused: no room     */
 } ptd_status;
 
 typedef enum { PTD_F32 = 0, PTD_BF16 = 1 } ptd_dtype;
@@ -248,6 +251,40 @@ ptd_status ptd_draft_tree_update(int32_t batch, int32_t in_stride, const int32_t
                                  int32_t width, int32_t max_depth, int32_t capacity, int32_t* out_count,
                                  int32_t* out_parents, int32_t* out_tokens, int32_t* out_depths, int32_t* old_to_new,
                                  int32_t* dev_status, void* stream);
+
+/* Candidate pool (Sec. 3.1 "Draft Extraction via Merging": any subtree T' of the draft tree
+ * is merged, by M, into the cached candidate tree with the same root value; Sec. 3.2 and
+ * Alg. 1 step 1: the candidate tree C_X retrieved for the decoded sequence X).
+ *
+ * The pool lives in one caller buffer of ptd_pool_bytes(capacity) bytes (device), a hash
+ * table of `capacity` trie nodes (a power of two, 16 .. 2^28); its first int32 is the
+ * number of nodes held.  ptd_pool_init empties it.  Pool calls on one buffer must be
+ * ordered (one stream); a pool is one sequence's. */
+size_t ptd_pool_bytes(int32_t capacity);                        /* 0 if capacity is invalid */
+ptd_status ptd_pool_init(void* pool, int32_t capacity, void* stream);
+
+/* Merge (Alg. 1 step 4): for every node v of the draft forest (count[0] nodes, parents /
+ * tokens device arrays in creation order, a seed's parent -1, at most PTD_MAX_TREE_NODES),
+ * in index order, the subtree rooted at v joins the pool entry of token(v), created when
+ * absent: M is the union of tries (a child whose token is new joins with its subtree, a
+ * child whose token is there merges recursively).  Children keep the order in which the
+ * sequential merge inserts them (step, then v, then the draft node); `step` must grow
+ * from call to call.  A merge that could take the node count past max_load (<= capacity)
+ * is refused as a whole with PTD_ERR_POOL_FULL in dev_status; an invalid forest sets
+ * PTD_ERR_INVALID_TREE.  One launch. */
+ptd_status ptd_pool_merge(void* pool, int32_t capacity, int32_t max_load, int32_t step, const int32_t* count,
+                          const int32_t* parents, const int32_t* tokens, int32_t* dev_status, void* stream);
+
+/* Retrieval (Alg. 1 step 1): the candidate tree for a sequence whose last token is
+ * *root_token (device int32, e.g. the previous step's bonus token): node 0 is the root
+ * token; then breadth first, each node's earliest-inserted children, at most `width`
+ * (1 .. 8) per node, nodes of depth at most max_depth (>= 1, the root has depth 1), at
+ * most max_nodes (1 .. PTD_MAX_TREE_NODES) in all.  A token with no entry gives the lone
+ * root.  Writes out_count[0] and out_parents / out_tokens [max_nodes] (-1 past the count):
+ * the tree layout of ptd_tree (parents[0] = -1, parents[i] < i).  One launch. */
+ptd_status ptd_pool_retrieve(const void* pool, int32_t capacity, const int32_t* root_token, int32_t width,
+                             int32_t max_depth, int32_t max_nodes, int32_t* out_count, int32_t* out_parents,
+                             int32_t* out_tokens, void* stream);
 
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.

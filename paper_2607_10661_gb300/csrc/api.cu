@@ -14,6 +14,7 @@
 #include "../../include/ptd.h"
 #include "verify_sampling.cuh"
 #include "draft_update.cuh"
+#include "pool.cuh"
 #include "attention.cuh"
 #include "topk.cuh"
 #include "verify_compact.cuh"
@@ -132,6 +133,8 @@ const char* ptd_status_string(ptd_status s) {
       return "device wait timed out";
     case PTD_ERR_WORKSPACE:
       return "workspace missing or too small";
+    case PTD_ERR_POOL_FULL:
+      return "candidate pool full: merge refused";
   }
   return "unknown status";
 }
@@ -352,6 +355,47 @@ ptd_status ptd_draft_tree_update(int32_t batch, int32_t in_stride, const int32_t
   const ptd_status st = cuda_status(ptd::launch_draft_update(
       batch, in_stride, in_count, in_parents, in_tokens, drafts, draft_stride, expand, width, max_depth, capacity,
       out_count, out_parents, out_tokens, out_depths, old_to_new, dev_status, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+namespace {
+bool pool_capacity_ok(int32_t capacity) {
+  return capacity >= 16 && capacity <= (1 << 28) && (capacity & (capacity - 1)) == 0;
+}
+}  // namespace
+
+size_t ptd_pool_bytes(int32_t capacity) { return pool_capacity_ok(capacity) ? ptd::pool_bytes(capacity) : 0; }
+
+ptd_status ptd_pool_init(void* pool, int32_t capacity, void* stream) {
+  g_last_launches = 0;
+  if (!pool || !pool_capacity_ok(capacity) || !aligned16(pool)) return PTD_ERR_INVALID_ARG;
+  return cuda_status(ptd::pool_init(pool, capacity, static_cast<cudaStream_t>(stream)));
+}
+
+ptd_status ptd_pool_merge(void* pool, int32_t capacity, int32_t max_load, int32_t step, const int32_t* count,
+                          const int32_t* parents, const int32_t* tokens, int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  if (!pool || !pool_capacity_ok(capacity) || !aligned16(pool) || max_load < 0 || max_load > capacity ||
+      step < 0 || !count || !parents || !tokens || !dev_status)
+    return PTD_ERR_INVALID_ARG;
+  const ptd_status st = cuda_status(ptd::launch_pool_merge(pool, capacity, max_load, step, count, parents, tokens,
+                                                           dev_status, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+ptd_status ptd_pool_retrieve(const void* pool, int32_t capacity, const int32_t* root_token, int32_t width,
+                             int32_t max_depth, int32_t max_nodes, int32_t* out_count, int32_t* out_parents,
+                             int32_t* out_tokens, void* stream) {
+  g_last_launches = 0;
+  if (!pool || !pool_capacity_ok(capacity) || !aligned16(pool) || !root_token || width < 1 ||
+      width > ptd::kPoolKids || max_depth < 1 || max_nodes < 1 || max_nodes > PTD_MAX_TREE_NODES || !out_count ||
+      !out_parents || !out_tokens)
+    return PTD_ERR_INVALID_ARG;
+  const ptd_status st =
+      cuda_status(ptd::launch_pool_retrieve(pool, capacity, root_token, width, max_depth, max_nodes, out_count,
+                                            out_parents, out_tokens, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }

@@ -17,17 +17,18 @@ import torch
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libptd.so")
 
-OK, INVALID_ARG, INVALID_TREE, UNSUPPORTED, CUDA_ERROR, TIMEOUT, WORKSPACE = range(7)
+OK, INVALID_ARG, INVALID_TREE, UNSUPPORTED, CUDA_ERROR, TIMEOUT, WORKSPACE, POOL_FULL = range(8)
 F32, BF16 = 0, 1
 MAX_TREE_NODES = 128
 MAX_TOPK = 16
 MAX_EXPAND = 16
+POOL_KIDS = 8
 
 EXPORTED = (
     "ptd_attention_workspace_size", "ptd_tree_attention", "ptd_topk_draft", "ptd_verify_greedy",
     "ptd_kv_compact", "ptd_tree_verify_step", "ptd_tree_verify_step_host", "ptd_last_launch_count",
     "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact", "ptd_verify_sampling",
-    "ptd_draft_tree_update",
+    "ptd_draft_tree_update", "ptd_pool_bytes", "ptd_pool_init", "ptd_pool_merge", "ptd_pool_retrieve",
 )
 
 
@@ -101,6 +102,14 @@ def lib() -> ctypes.CDLL:
         L.ptd_draft_tree_update.restype = ctypes.c_int
         L.ptd_draft_tree_update.argtypes = [i32, i32, vp, vp, vp, vp, i32, i32, i32, i32, i32, vp, vp, vp, vp, vp,
                                             vp, vp]
+        L.ptd_pool_bytes.restype = sz
+        L.ptd_pool_bytes.argtypes = [i32]
+        L.ptd_pool_init.restype = ctypes.c_int
+        L.ptd_pool_init.argtypes = [vp, i32, vp]
+        L.ptd_pool_merge.restype = ctypes.c_int
+        L.ptd_pool_merge.argtypes = [vp, i32, i32, i32, vp, vp, vp, vp, vp]
+        L.ptd_pool_retrieve.restype = ctypes.c_int
+        L.ptd_pool_retrieve.argtypes = [vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]
         L.ptd_tree_verify_step.restype = ctypes.c_int
         L.ptd_tree_verify_step.argtypes = [P(_Tree), P(_Cache), P(_StepArgs), vp]
         L.ptd_tree_verify_step_host.restype = ctypes.c_int
@@ -347,3 +356,40 @@ def draft_tree_update(in_count: torch.Tensor, in_parents: torch.Tensor, in_token
         _dev(dev_status, "dev_status", torch.int32), _stream(stream))
     _check(st, "ptd_draft_tree_update")
     return last_launch_count()
+
+
+class CandidatePool:
+    """A candidate pool in one device buffer (ptd_pool_bytes / ptd_pool_init)."""
+
+    def __init__(self, capacity: int, device="cuda", stream=None):
+        n = int(lib().ptd_pool_bytes(int(capacity)))
+        if n == 0:
+            raise ValueError("pool capacity must be a power of two in [16, 2^28]")
+        self.capacity = int(capacity)
+        self.buf = torch.empty(n, dtype=torch.uint8, device=device)
+        _check(lib().ptd_pool_init(_dev(self.buf, "pool"), self.capacity, _stream(stream)), "ptd_pool_init")
+
+    def size(self) -> int:
+        """Nodes held (reads the device counter: synchronises)."""
+        return int(self.buf[:4].view(torch.int32).item())
+
+    def merge(self, step: int, count: torch.Tensor, parents: torch.Tensor, tokens: torch.Tensor,
+              dev_status: torch.Tensor, max_load: Optional[int] = None, stream=None) -> int:
+        st = lib().ptd_pool_merge(_dev(self.buf, "pool"), self.capacity,
+                                  self.capacity // 2 if max_load is None else int(max_load), int(step),
+                                  _dev(count, "count", torch.int32), _dev(parents, "parents", torch.int32),
+                                  _dev(tokens, "tokens", torch.int32), _dev(dev_status, "dev_status", torch.int32),
+                                  _stream(stream))
+        _check(st, "ptd_pool_merge")
+        return last_launch_count()
+
+    def retrieve(self, root_token: torch.Tensor, width: int, max_depth: int, max_nodes: int,
+                 out_count: torch.Tensor, out_parents: torch.Tensor, out_tokens: torch.Tensor, stream=None) -> int:
+        if out_parents.numel() < max_nodes or out_tokens.numel() < max_nodes:
+            raise ValueError("out_parents / out_tokens need max_nodes entries")
+        st = lib().ptd_pool_retrieve(_dev(self.buf, "pool"), self.capacity, _dev(root_token, "root_token", torch.int32),
+                                     int(width), int(max_depth), int(max_nodes), _dev(out_count, "out_count", torch.int32),
+                                     _dev(out_parents, "out_parents", torch.int32),
+                                     _dev(out_tokens, "out_tokens", torch.int32), _stream(stream))
+        _check(st, "ptd_pool_retrieve")
+        return last_launch_count()

@@ -43,8 +43,8 @@ def test_every_declared_symbol_is_exported(lib):
 def test_status_strings(lib):
     from paper_2607_10661_gb300 import ptd
 
-    for s in range(7):
-        assert ptd.status_string(s)
+    for s in range(8):
+        assert ptd.status_string(s) and ptd.status_string(s) != "unknown status"
     assert ptd.status_string(0) == "ok"
 
 
@@ -75,6 +75,15 @@ def test_host_checks_reject_without_gpu(lib):
     assert du(batch=0) == ptd.INVALID_ARG
     assert du(outp=32) == ptd.INVALID_ARG
     assert du(status=None) == ptd.INVALID_ARG
+    # candidate pool: capacity not a power of two, width above the kept children, bad budgets
+    assert lib.ptd_pool_bytes(1000) == 0 and lib.ptd_pool_bytes(1 << 20) > (1 << 20) * 48
+    assert lib.ptd_pool_init(None, 1024, None) == ptd.INVALID_ARG
+    assert lib.ptd_pool_init(16, 1000, None) == ptd.INVALID_ARG
+    assert lib.ptd_pool_merge(16, 1024, 2048, 0, 16, 16, 16, 16, None) == ptd.INVALID_ARG     # max_load > capacity
+    assert lib.ptd_pool_merge(16, 1024, 512, -1, 16, 16, 16, 16, None) == ptd.INVALID_ARG    # negative step
+    assert lib.ptd_pool_retrieve(16, 1024, 16, 9, 4, 64, 16, 16, 16, None) == ptd.INVALID_ARG  # width > 8
+    assert lib.ptd_pool_retrieve(16, 1024, 16, 4, 0, 64, 16, 16, 16, None) == ptd.INVALID_ARG  # max_depth 0
+    assert lib.ptd_pool_retrieve(16, 1024, 16, 4, 4, 129, 16, 16, 16, None) == ptd.INVALID_ARG  # max_nodes > 128
     t = ptd._Tree(1, 200, 200, 0, 8, 8, 8)          # max_nodes above 128
     c = ptd._Cache(16, 16, ptd.BF16, 1, 8, 128, 0, 300, 0, None, 0)
     assert lib.ptd_tree_attention(ctypes.byref(t), ctypes.byref(c), 0, 1, 16, 32, 0.0, 16, None, 0, 16,

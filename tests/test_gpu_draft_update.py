@@ -25,8 +25,10 @@ def _forest(g, T, n_tokens, seed_p=0.15):
         p = -1 if (i == 0 or g.random() < seed_p) else int(g.integers(0, i))
         used = kid_tokens.setdefault(p, set()) if p >= 0 else set()
         t = int(g.integers(0, n_tokens))
-        while t in used:
+        while t in used and len(used) < n_tokens:
             t = (t + 1) % n_tokens
+        if t in used:                    # every token taken: a fresh one past the range
+            t = n_tokens + len(used)
         used.add(t)
         parents.append(p)
         tokens.append(t)

@@ -512,8 +512,10 @@ def _random_forest(g, T, n_tokens):
     for i, p in enumerate(parents):      # siblings carry distinct tokens, as in a trie
         used = kids_tokens.setdefault(p, set()) if p >= 0 else set()
         t = int(g.integers(0, n_tokens))
-        while t in used:
+        while t in used and len(used) < n_tokens:
             t = (t + 1) % n_tokens
+        if t in used:                    # every token taken: a fresh one past the range
+            t = n_tokens + len(used)
         used.add(t)
         tokens.append(t)
     return parents, tokens
