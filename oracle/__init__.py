@@ -17,6 +17,8 @@ from .ptd_oracle import (  # noqa: F401
     softmax_row,
     topk,
     topk_rows,
+    tree_positions,
+    rope,
     tree_attention,
     verify_greedy,
     verify_sampling,

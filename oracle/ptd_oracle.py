@@ -29,6 +29,10 @@ cites the passage it follows:
                                  token joins the tree as its child), "Width Control"
                                  and "Stepping Mechanism (Depth Control)"; Alg. 1
                                  step 3 (expand, then StepAndPrune past d_max).
+  tree_positions, rope ......... Sec. 3.1 "Tree Construction": a node's position is
+                                 set by |pi(v)|, here C + |pi(v)| - 1 after the
+                                 committed prefix; the rotary encoding itself is the
+                                 model's (RoFormer's rotation, rotate-half layout).
   CandidatePool ................ Sec. 3.1 "Draft Extraction via Merging" (the merge
                                  M(T, T') of two trees with the same root value) and
                                  Alg. 1 step 4; Sec. 3.2 and Alg. 1 step 1 (retrieve
@@ -69,6 +73,11 @@ Readings where the paper is silent (each listed in the design notes):
     child, which becomes a seed; everything else under the old seed goes.  Pruning
     runs once per step, after expansion (Alg. 1 step 3).  Survivors keep their
     relative order.
+  * tree positions: node v of a tree over a committed prefix of C tokens sits at
+    position C + |pi(v)| - 1 (the root, the current input token, at C: the position
+    the next token of plain decoding would have); the rotary encoding is RoFormer's
+    rotation in the rotate-half layout used by Llama-family models: dims i and i + D/2
+    turn by pos * base^(-2i/D).
   * candidate pool: a map from a root token to a trie of draft continuations.  The
     merge M is read as the union of tries: a child of T' whose token is not among the
     children of T joins T together with its whole subtree (the printed case adds the
@@ -473,3 +482,25 @@ class CandidatePool:
             frontier = nxt
             depth += 1
         return np.array(parents, np.int64), np.array(tokens, np.int64)
+
+
+# ---------------------------------------------------------------------------
+# Tree positions and the rotary encoding (Sec. 3.1 "Tree Construction")
+# ---------------------------------------------------------------------------
+
+def tree_positions(parents, ctx_len: int) -> np.ndarray:
+    """Position of every node: C + |pi(v)| - 1 (|pi(v)| counts v and its ancestors)."""
+    return np.asarray([ctx_len + len(a) - 1 for a in ancestor_sets(parents)], np.int64)
+
+
+def rope(x, positions, base: float) -> np.ndarray:
+    """Rotary encoding of x [N, H, D] at positions [N] (float64): for i < D/2 the pair
+    (x_i, x_{i+D/2}) turns by the angle positions[n] * base^(-2i/D)."""
+    x = np.asarray(x, np.float64)
+    D = x.shape[-1]
+    half = D // 2
+    inv_freq = base ** (-2.0 * np.arange(half, dtype=np.float64) / D)
+    ang = np.asarray(positions, np.float64)[:, None] * inv_freq[None, :]        # [N, D/2]
+    c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
+    a, b = x[..., :half], x[..., half:]
+    return np.concatenate([a * c - b * s, a * s + b * c], axis=-1)

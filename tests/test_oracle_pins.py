@@ -691,3 +691,49 @@ def test_pool_idempotent_and_chain():
     for i, t in enumerate(seq):
         par, tok = chain.retrieve(t, 4, 99, 99)
         assert tok.tolist() == seq[i:] and par.tolist() == [-1] + list(range(len(seq) - i - 1))
+
+
+# ---------------------------------------------------------------------------
+# Tree positions and the rotary encoding (Sec. 3.1 "Tree Construction")
+# ---------------------------------------------------------------------------
+
+def test_tree_positions_closed_forms():
+    """A chain sits at C .. C + T - 1 (ordinary causal positions), a star's leaves all at
+    C + 1, and a node's position is its parent's plus one."""
+    assert oracle.tree_positions([-1, 0, 1, 2, 3], 100).tolist() == [100, 101, 102, 103, 104]
+    assert oracle.tree_positions([-1, 0, 0, 0], 7).tolist() == [7, 8, 8, 8]
+    g = np.random.default_rng(41)
+    parents = [-1] + [int(g.integers(0, i)) for i in range(1, 60)]
+    pos = oracle.tree_positions(parents, 33)
+    assert pos[0] == 33 and all(pos[i] == pos[parents[i]] + 1 for i in range(1, 60))
+
+
+def test_rope_defining_properties():
+    """RoFormer's rotation: position 0 is the identity, norms are kept, rotations compose
+    (rope(rope(x, a), b) = rope(x, a + b)), and q.k after encoding depends only on the
+    offset between the two positions."""
+    g = np.random.default_rng(42)
+    x = g.normal(size=(5, 3, 64))
+    y = g.normal(size=(5, 3, 64))
+    base = 10000.0
+    assert np.allclose(oracle.rope(x, np.zeros(5), base), x)
+    p = g.integers(0, 5000, size=5)
+    r = oracle.rope(x, p, base)
+    assert np.allclose(np.linalg.norm(r, axis=-1), np.linalg.norm(x, axis=-1))
+    q = g.integers(0, 5000, size=5)
+    assert np.allclose(oracle.rope(r, q, base), oracle.rope(x, p + q, base))
+    shift = 1234
+    d1 = np.sum(oracle.rope(x, p, base) * oracle.rope(y, q, base), axis=-1)
+    d2 = np.sum(oracle.rope(x, p + shift, base) * oracle.rope(y, q + shift, base), axis=-1)
+    assert np.allclose(d1, d2)
+    # the lowest pair turns by exactly the position (angle pos * base^0) and the rest slower
+    e = np.zeros((1, 1, 64))
+    e[0, 0, 0] = 1.0
+    out = oracle.rope(e, [3], base)[0, 0]
+    assert np.isclose(out[0], np.cos(3.0)) and np.isclose(out[32], np.sin(3.0))
+    # pair 5 of 32 turns by 3 * 10000^(-10/64) = 3 * 10^-0.625 = 0.71141211 rad
+    e = np.zeros((1, 1, 64))
+    e[0, 0, 5] = 1.0
+    out = oracle.rope(e, [3], base)[0, 0]
+    assert np.isclose(out[5], 0.7574406580936761) and np.isclose(out[37], 0.652904012444876)
+    assert np.count_nonzero(np.abs(out) > 1e-12) == 2
