@@ -174,6 +174,20 @@ def run_gpu(args, rank: int, world: int, dist):
         gu.manual_seed(5000 + rank)
         u_acc = torch.rand(w.n_total, device=f"cuda:{local}", generator=gu)
         u_bon = torch.rand(cfg.batch, device=f"cuda:{local}", generator=gu)
+    if args.ptd_step:
+        args.draft_update = True
+        # the tree's own (unrotated) K and V of every layer, written by the rotary step into
+        # the cache slots the attention reads; the candidate pool the draft tree feeds
+        gk = torch.Generator(device=f"cuda:{local}")
+        gk.manual_seed(6000 + rank)
+        tree_k = torch.randn((cfg.layers, w.n_total, cfg.hkv, cfg.d), generator=gk,
+                             device=f"cuda:{local}").to(dw.tdtype)
+        tree_v = torch.randn_like(tree_k)
+        pool = ptd.CandidatePool(1 << 20, device=f"cuda:{local}")
+        ret = [torch.zeros(1, dtype=torch.int32, device=f"cuda:{local}"),
+               torch.empty(ptd.MAX_TREE_NODES, dtype=torch.int32, device=f"cuda:{local}"),
+               torch.empty(ptd.MAX_TREE_NODES, dtype=torch.int32, device=f"cuda:{local}")]
+        pool_step = [0]
     if args.draft_update:
         # the step's tree as a one-seed draft forest, grown by every node's top-1 (width 4,
         # depth 6: the paper's best setting); the output is the next step's draft tree
@@ -187,6 +201,8 @@ def run_gpu(args, rank: int, world: int, dist):
 
     def one_step(ev=None):
         n = 0
+        if args.ptd_step:   # positions C + |pi(v)| - 1, rotary encoding, tree K/V into the cache
+            n += ptd.tree_rope_append(dw.tree, dw.cache, 0, dw.q, cfg.hq, tree_k, tree_v, 500000.0, dw.dev_status)
         if ev is not None:
             ev[0].record(stream)
         n += dw.attention()
@@ -196,12 +212,17 @@ def run_gpu(args, rank: int, world: int, dist):
         if args.draft_update:
             n += ptd.draft_tree_update(du_cnt, dw.parents.view(1, -1), dw.tokens.view(1, -1), dw.topk_idx, 1, 4, 6,
                                        ptd.MAX_TREE_NODES, *du_out, dw.dev_status)
+        if args.ptd_step:   # the grown draft tree joins the pool; C_X for the next step
+            pool_step[0] += 1
+            n += pool.merge(pool_step[0], du_out[0], du_out[1][0], du_out[2][0], dw.dev_status, max_load=1 << 19)
         if sampling:
             n += ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, 1.0, u_acc, u_bon, dw.accepted, dw.accept_len,
                                      dw.bonus, dw.dev_status)
             n += dw.compact()
         else:
             n += dw.verify_and_compact()
+        if args.ptd_step:
+            n += pool.retrieve(dw.bonus[:1], 4, 6, 64, *ret)
         return n
 
     dw.dev_status.zero_()              # sticky status word: cleared once, read after the run
@@ -298,6 +319,9 @@ def run_gpu(args, rank: int, world: int, dist):
                    "context": cfg.ctx[0], "tree_nodes": w.n_total, "vocab": cfg.vocab, "k": cfg.k,
                    "verify": "sampling (Alg. 2, temperature 1)" if sampling else "greedy",
                    "draft_update": "top-1 expansion, width 4, depth 6 (Alg. 1 step 3)" if args.draft_update else None,
+                   "ptd_step": ("tree positions + rotary encoding + K/V append (32 layers), attention, top-k, "
+                                "verification + compaction, draft update, pool merge, pool retrieval")
+                   if args.ptd_step else None,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 (%.2f GB read per step vs 129 MB L2)" % (nb["roofline"] / 1e9)},
         "step_roofline_bytes": nb["roofline"],
@@ -428,6 +452,9 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling captures)")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ptd-step", action="store_true",
+                    help="the whole PTD step: rotary encoding and tree K/V append, the verify step, the draft "
+                         "tree update and the candidate pool's merge and retrieval (Alg. 1 steps 1-6)")
     ap.add_argument("--draft-update", action="store_true",
                     help="add the draft tree update (Sec. 3.1 expansion and depth control) to every step")
     ap.add_argument("--verify", default="greedy", choices=["greedy", "sampling"],

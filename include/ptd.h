@@ -17,7 +17,8 @@
  * plus ptd_verify_sampling (verification under the sampling strategy, Alg. 2),
  * ptd_draft_tree_update (the draft forest's expansion and depth control, Alg. 1 step 3),
  * ptd_pool_* (the candidate pool: merge of the draft subtrees and retrieval of the
- * candidate tree, Alg. 1 steps 4 and 1),
+ * candidate tree, Alg. 1 steps 4 and 1), ptd_tree_rope_append (tree positions, the
+ * rotary encoding and the tree's K/V into the cache),
  * ptd_verify_and_compact (the last two as one launch) and ptd_tree_verify_step (the
  * whole step: attention, top-k, verification and compaction on one stream)
  *
@@ -285,6 +286,25 @@ ptd_status ptd_pool_merge(void* pool, int32_t capacity, int32_t max_load, int32_
 ptd_status ptd_pool_retrieve(const void* pool, int32_t capacity, const int32_t* root_token, int32_t width,
                              int32_t max_depth, int32_t max_nodes, int32_t* out_count, int32_t* out_parents,
                              int32_t* out_tokens, void* stream);
+
+/* Tree positions and the tree's K/V append (Sec. 3.1 "Tree Construction": the position of
+ * node v is set by |pi(v)|).  Node i of tree b sits at p = C_b + |pi(i)| - 1 (the root at
+ * C_b, where plain decoding would put the next token).  For the cache layers
+ * l in [layer_begin, layer_begin + num_layers), with l' = l - layer_begin:
+ *   q [num_layers][N_tot][num_q_heads][D] (device, cache->dtype) is rotated in place;
+ *   k, v [num_layers][N_tot][num_kv_heads][D]: k[l'] rotated, k[l'] and v[l'] written to
+ *   cache layer l, slot C_b + i;
+ * rotation: for j < D/2 the pair (x_j, x_{j+D/2}) turns by p * rope_base^(-2j/D)
+ * (RoFormer's rotary encoding in the rotate-half layout of Llama-family models; the angle
+ * is carried as an fp32 pair from inverse frequencies computed in double, about 1e-7
+ * relative).  positions_out [N_tot] (device, may be NULL)
+ * receives p.  A tree that is not one, or a slot outside the cache (or a page outside the
+ * pool), sets PTD_ERR_INVALID_TREE in dev_status; that node writes nothing.  q must not
+ * alias k or v.  One launch, one CTA per (node, layer).  This is what puts the tree's K/V
+ * where ptd_tree_attention expects them. */
+ptd_status ptd_tree_rope_append(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
+                                int32_t num_layers, void* q, int32_t num_q_heads, const void* k, const void* v,
+                                float rope_base, int32_t* positions_out, int32_t* dev_status, void* stream);
 
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.

@@ -15,6 +15,7 @@
 #include "verify_sampling.cuh"
 #include "draft_update.cuh"
 #include "pool.cuh"
+#include "tree_rope.cuh"
 #include "attention.cuh"
 #include "topk.cuh"
 #include "verify_compact.cuh"
@@ -396,6 +397,37 @@ ptd_status ptd_pool_retrieve(const void* pool, int32_t capacity, const int32_t* 
   const ptd_status st =
       cuda_status(ptd::launch_pool_retrieve(pool, capacity, root_token, width, max_depth, max_nodes, out_count,
                                             out_parents, out_tokens, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+ptd_status ptd_tree_rope_append(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
+                                int32_t num_layers, void* q, int32_t num_q_heads, const void* k, const void* v,
+                                float rope_base, int32_t* positions_out, int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  ptd_status st = check_tree(tree);
+  if (st != PTD_OK) return st;
+  if ((st = check_cache(cache)) != PTD_OK) return st;
+  const int D = cache->head_dim, hkv = cache->num_kv_heads;
+  if (layer_begin < 0 || num_layers < 1 || num_layers > 65535 || layer_begin + num_layers > cache->num_layers ||
+      num_q_heads < hkv || num_q_heads % hkv != 0 || D % 2 != 0 ||
+      D / 2 > ptd::kMaxRopeHalf || !q || !k || !v || !dev_status || !(rope_base > 1.f) || !std::isfinite(rope_base))
+    return PTD_ERR_INVALID_ARG;
+  const size_t es = dtype_size(cache->dtype);
+  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v)) % es != 0)
+    return PTD_ERR_INVALID_ARG;
+  ptd::RopeFreqs f = {};
+  for (int j = 0; j < D / 2; ++j) {
+    const double x = std::pow((double)rope_base, -2.0 * j / D);
+    f.hi[j] = (float)x;
+    f.lo[j] = (float)(x - (double)f.hi[j]);
+  }
+  st = cuda_status(ptd::launch_tree_rope(tree->node_offsets, tree->parents, tree->ctx_lens, tree->batch,
+                                         tree->total_nodes, cache->dtype == PTD_BF16, D, num_q_heads, hkv, q, k, v,
+                                         cache->k, cache->v, layer_begin, num_layers, cache->page_size,
+                                         cache->seq_capacity,
+                                         cache->num_pages, cache->block_table, cache->max_pages, f, positions_out,
+                                         dev_status, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }

@@ -29,6 +29,7 @@ EXPORTED = (
     "ptd_kv_compact", "ptd_tree_verify_step", "ptd_tree_verify_step_host", "ptd_last_launch_count",
     "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact", "ptd_verify_sampling",
     "ptd_draft_tree_update", "ptd_pool_bytes", "ptd_pool_init", "ptd_pool_merge", "ptd_pool_retrieve",
+    "ptd_tree_rope_append",
 )
 
 
@@ -110,6 +111,8 @@ def lib() -> ctypes.CDLL:
         L.ptd_pool_merge.argtypes = [vp, i32, i32, i32, vp, vp, vp, vp, vp]
         L.ptd_pool_retrieve.restype = ctypes.c_int
         L.ptd_pool_retrieve.argtypes = [vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]
+        L.ptd_tree_rope_append.restype = ctypes.c_int
+        L.ptd_tree_rope_append.argtypes = [P(_Tree), P(_Cache), i32, i32, vp, i32, vp, vp, f32, vp, vp, vp]
         L.ptd_tree_verify_step.restype = ctypes.c_int
         L.ptd_tree_verify_step.argtypes = [P(_Tree), P(_Cache), P(_StepArgs), vp]
         L.ptd_tree_verify_step_host.restype = ctypes.c_int
@@ -393,3 +396,19 @@ class CandidatePool:
                                      _dev(out_tokens, "out_tokens", torch.int32), _stream(stream))
         _check(st, "ptd_pool_retrieve")
         return last_launch_count()
+
+
+def tree_rope_append(tree: Tree, cache: KVCache, layer_begin: int, q: torch.Tensor, num_q_heads: int,
+                     k: torch.Tensor, v: torch.Tensor, rope_base: float, dev_status: torch.Tensor,
+                     positions_out: Optional[torch.Tensor] = None, stream=None) -> int:
+    """ptd_tree_rope_append: q [L, N_tot, Hq, D] rotated in place; k, v [L, N_tot, Hkv, D]
+    into cache layers layer_begin .. layer_begin + L - 1 (a 3-D q, k, v is one layer)."""
+    dt = cache.k.dtype
+    n_layers = q.shape[0] if q.dim() == 4 else 1
+    st = lib().ptd_tree_rope_append(ctypes.byref(tree.c), ctypes.byref(cache.c), int(layer_begin), int(n_layers),
+                                    _dev(q, "q", dt),
+                                    int(num_q_heads), _dev(k, "k", dt), _dev(v, "v", dt), float(rope_base),
+                                    None if positions_out is None else _dev(positions_out, "positions_out", torch.int32),
+                                    _dev(dev_status, "dev_status", torch.int32), _stream(stream))
+    _check(st, "ptd_tree_rope_append")
+    return last_launch_count()

@@ -84,6 +84,16 @@ def test_host_checks_reject_without_gpu(lib):
     assert lib.ptd_pool_retrieve(16, 1024, 16, 9, 4, 64, 16, 16, 16, None) == ptd.INVALID_ARG  # width > 8
     assert lib.ptd_pool_retrieve(16, 1024, 16, 4, 0, 64, 16, 16, 16, None) == ptd.INVALID_ARG  # max_depth 0
     assert lib.ptd_pool_retrieve(16, 1024, 16, 4, 4, 129, 16, 16, 16, None) == ptd.INVALID_ARG  # max_nodes > 128
+    # tree positions / rotary encoding: no tree, layer range past the cache, odd head_dim, base <= 1
+    assert lib.ptd_tree_rope_append(None, None, 0, 1, 16, 32, 16, 16, 10000.0, None, 16, None) == ptd.INVALID_ARG
+    tr_ = ptd._Tree(1, 10, 10, 0, 16, 16, 16)
+    cr = ptd._Cache(16, 16, ptd.BF16, 2, 8, 128, 0, 300, 0, None, 0)
+    assert lib.ptd_tree_rope_append(ctypes.byref(tr_), ctypes.byref(cr), 1, 2, 16, 32, 16, 16, 10000.0, None, 16,
+                                    None) == ptd.INVALID_ARG
+    assert lib.ptd_tree_rope_append(ctypes.byref(tr_), ctypes.byref(cr), 0, 1, 16, 32, 16, 16, 1.0, None, 16,
+                                    None) == ptd.INVALID_ARG
+    assert lib.ptd_tree_rope_append(ctypes.byref(tr_), ctypes.byref(cr), 0, 1, 16, 12, 16, 16, 1e4, None, 16,
+                                    None) == ptd.INVALID_ARG     # 12 query heads over 8 KV heads
     t = ptd._Tree(1, 200, 200, 0, 8, 8, 8)          # max_nodes above 128
     c = ptd._Cache(16, 16, ptd.BF16, 1, 8, 128, 0, 300, 0, None, 0)
     assert lib.ptd_tree_attention(ctypes.byref(t), ctypes.byref(c), 0, 1, 16, 32, 0.0, 16, None, 0, 16,
