@@ -14,6 +14,8 @@ from .ptd_oracle import (  # noqa: F401
     draft_tree_update,
     eligible_edges,
     kv_compact,
+    lm_head_logits,
+    lm_head_topk,
     softmax_row,
     topk,
     topk_rows,

@@ -29,6 +29,9 @@ cites the passage it follows:
                                  token joins the tree as its child), "Width Control"
                                  and "Stepping Mechanism (Depth Control)"; Alg. 1
                                  step 3 (expand, then StepAndPrune past d_max).
+  lm_head_topk ................. the per-node logits P(y_T | ...) of Alg. 1 step 2 as
+                                 the LM-head product h_v W^T, followed by topk_rows
+                                 (the drafts d_v and verification tokens V_n).
   tree_positions, rope ......... Sec. 3.1 "Tree Construction": a node's position is
                                  set by |pi(v)|, here C + |pi(v)| - 1 after the
                                  committed prefix; the rotary encoding itself is the
@@ -504,3 +507,17 @@ def rope(x, positions, base: float) -> np.ndarray:
     c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
     a, b = x[..., :half], x[..., half:]
     return np.concatenate([a * c - b * s, a * s + b * c], axis=-1)
+
+
+# ---------------------------------------------------------------------------
+# LM head with top-k (Alg. 1 step 2: the per-node logits; Sec. 3.1 / 3.2: their top-k)
+# ---------------------------------------------------------------------------
+
+def lm_head_logits(hidden, weight) -> np.ndarray:
+    """Logits of every node: hidden [N, d] times weight [V, d] transposed, in float64."""
+    return np.asarray(hidden, np.float64) @ np.asarray(weight, np.float64).T
+
+
+def lm_head_topk(hidden, weight, k: int):
+    """topk_rows of the LM-head logits: (indices [N, k], values [N, k])."""
+    return topk_rows(lm_head_logits(hidden, weight), k)

@@ -737,3 +737,30 @@ def test_rope_defining_properties():
     out = oracle.rope(e, [3], base)[0, 0]
     assert np.isclose(out[5], 0.7574406580936761) and np.isclose(out[37], 0.652904012444876)
     assert np.count_nonzero(np.abs(out) > 1e-12) == 2
+
+
+# ---------------------------------------------------------------------------
+# LM head with top-k
+# ---------------------------------------------------------------------------
+
+def test_lm_head_worked_example_and_brute_force():
+    """A 2-node, 5-token example worked by hand, and random cases against a brute-force
+    dot product per (node, token) with a sort by (-value, index)."""
+    h = [[1.0, 2.0], [0.5, -1.0]]
+    w = [[1, 0], [0, 1], [1, 1], [-1, 0], [2, -1]]
+    # node 0: logits 1, 2, 3, -1, 0 -> top-2 tokens 2, 1; node 1: 0.5, -1, -0.5, -0.5, 2 -> 4, 0
+    idx, val = oracle.lm_head_topk(h, w, 2)
+    assert idx.tolist() == [[2, 1], [4, 0]] and val.tolist() == [[3.0, 2.0], [2.0, 0.5]]
+    idx, _ = oracle.lm_head_topk([[0.0, 1.0]], [[1, 2], [3, 2], [5, 2]], 3)   # a three-way tie
+    assert idx.tolist() == [[0, 1, 2]]
+    g = np.random.default_rng(51)
+    for _ in range(20):
+        N, d, V = int(g.integers(1, 6)), int(g.integers(1, 9)), int(g.integers(1, 40))
+        k = min(V, int(g.integers(1, 6)))
+        hh = g.integers(-3, 4, size=(N, d)).astype(float)
+        ww = g.integers(-3, 4, size=(V, d)).astype(float)   # small integers: many exact ties
+        idx, val = oracle.lm_head_topk(hh, ww, k)
+        for n in range(N):
+            logits = [sum(hh[n, j] * ww[t, j] for j in range(d)) for t in range(V)]
+            order = sorted(range(V), key=lambda t: (-logits[t], t))[:k]
+            assert idx[n].tolist() == order and val[n].tolist() == [logits[t] for t in order]
