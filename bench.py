@@ -174,6 +174,18 @@ def run_gpu(args, rank: int, world: int, dist):
         gu.manual_seed(5000 + rank)
         u_acc = torch.rand(w.n_total, device=f"cuda:{local}", generator=gu)
         u_bon = torch.rand(cfg.batch, device=f"cuda:{local}", generator=gu)
+    if args.lm_head:
+        # the LM head feeds top-k from the nodes' hidden states: W [vocab][d_model] bf16 and H
+        # [N_tot][d_model] (synthetic, seeded; Llama-3-8B's head is 128256 x 4096)
+        d_model = 4096
+        gh = torch.Generator(device=f"cuda:{local}")
+        gh.manual_seed(7000 + rank)
+        lm_w = (torch.randn((cfg.vocab, d_model), generator=gh, device=f"cuda:{local}") / d_model ** 0.5).to(
+            torch.bfloat16)
+        lm_h = torch.randn((w.n_total, d_model), generator=gh, device=f"cuda:{local}").to(torch.bfloat16)
+        lm_ws = torch.empty(ptd.lm_head_workspace_size(w.n_total, cfg.vocab), dtype=torch.uint8,
+                            device=f"cuda:{local}")
+        lm_evs = []
     if args.ptd_step:
         args.draft_update = True
         # the tree's own (unrotated) K and V of every layer, written by the rotary step into
@@ -208,7 +220,16 @@ def run_gpu(args, rank: int, world: int, dist):
         n += dw.attention()
         if ev is not None:
             ev[1].record(stream)
-        n += dw.topk()
+        if args.lm_head:
+            if ev is not None:
+                e2 = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                e2[0].record(stream)
+            n += ptd.lm_head_topk(lm_h, lm_w, cfg.k, dw.topk_idx, dw.topk_val, lm_ws, dw.dev_status)
+            if ev is not None:
+                e2[1].record(stream)
+                lm_evs.append(e2)
+        else:
+            n += dw.topk()
         if args.draft_update:
             n += ptd.draft_tree_update(du_cnt, dw.parents.view(1, -1), dw.tokens.view(1, -1), dw.topk_idx, 1, 4, 6,
                                        ptd.MAX_TREE_NODES, *du_out, dw.dev_status)
@@ -252,6 +273,7 @@ def run_gpu(args, rank: int, world: int, dist):
         dist.barrier()
     ms = start.elapsed_time(end)
     attn_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    lm_ms = float(np.mean([a.elapsed_time(b) for a, b in lm_evs])) if args.lm_head else None
     clocks = sampler.summary(t_wall0, t_wall1)
     sampler.stop()
     status = int(dw.dev_status.item())
@@ -319,6 +341,8 @@ def run_gpu(args, rank: int, world: int, dist):
                    "context": cfg.ctx[0], "tree_nodes": w.n_total, "vocab": cfg.vocab, "k": cfg.k,
                    "verify": "sampling (Alg. 2, temperature 1)" if sampling else "greedy",
                    "draft_update": "top-1 expansion, width 4, depth 6 (Alg. 1 step 3)" if args.draft_update else None,
+                   "top_k_source": ("LM head from hidden states (63 x 4096 by 128256 x 4096 bf16, logits not "
+                                    "written)" if args.lm_head else "resident logits"),
                    "ptd_step": ("tree positions + rotary encoding + K/V append (32 layers), attention, top-k, "
                                 "verification + compaction, draft update, pool merge, pool retrieval")
                    if args.ptd_step else None,
@@ -337,6 +361,12 @@ def run_gpu(args, rank: int, world: int, dist):
         "e2e": {"value": round(world * Ke / (e2e_ms * 1e-3), 3), "unit": "steps/s", "steps": Ke,
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "status_ok": e2e_ok,
                 "verify": "greedy (the host step call)"},
+        "lm_head": ({"kernel": "lm_head_topk_kernel", "avg_launch_ms": round(lm_ms, 5),
+                     "bytes_per_launch": int(lm_w.numel() * 2 + lm_h.numel() * 2),
+                     "achieved_gbs": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9, 1),
+                     "frac": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9
+                                   / _peak_hbm()[0], 4), "peak_kind": _peak_hbm()[1]}
+                    if args.lm_head else None),
         "gpu_launches": int(launches),
         "status": ptd.status_string(status),
     }
@@ -452,6 +482,9 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling captures)")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--lm-head", action="store_true",
+                    help="top-k from the LM head (ptd_lm_head_topk, logits never written) instead of from "
+                         "resident logits")
     ap.add_argument("--ptd-step", action="store_true",
                     help="the whole PTD step: rotary encoding and tree K/V append, the verify step, the draft "
                          "tree update and the candidate pool's merge and retrieval (Alg. 1 steps 1-6)")

@@ -18,7 +18,8 @@
  * ptd_draft_tree_update (the draft forest's expansion and depth control, Alg. 1 step 3),
  * ptd_pool_* (the candidate pool: merge of the draft subtrees and retrieval of the
  * candidate tree, Alg. 1 steps 4 and 1), ptd_tree_rope_append (tree positions, the
- * rotary encoding and the tree's K/V into the cache),
+ * rotary encoding and the tree's K/V into the cache), ptd_lm_head_topk (the LM-head
+ * product with a fused top-k: the logits are never written),
  * ptd_verify_and_compact (the last two as one launch) and ptd_tree_verify_step (the
  * whole step: attention, top-k, verification and compaction on one stream)
  *
@@ -305,6 +306,26 @@ ptd_status ptd_pool_retrieve(const void* pool, int32_t capacity, const int32_t* 
 ptd_status ptd_tree_rope_append(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
                                 int32_t num_layers, void* q, int32_t num_q_heads, const void* k, const void* v,
                                 float rope_base, int32_t* positions_out, int32_t* dev_status, void* stream);
+
+/* LM head with a fused top-k: for every node row r of hidden, the logits h_r W^T (the
+ * model's next-token scores P(y_T | ...) of Alg. 1 step 2) and their k largest entries,
+ * as ptd_topk_draft would give them (descending, the lower token first on equal values,
+ * -0.0 == +0.0; Sec. 3.1 draft tokens d_v, Sec. 3.2 verification tokens V_n), without the
+ * logits ever reaching memory.
+ *   hidden: [rows][hidden_stride] bf16 (device), rows 1 .. PTD_MAX_TREE_NODES;
+ *   weight: [vocab][weight_stride] bf16 (device); d_model a multiple of 64; strides
+ *           multiples of 8 elements, both base pointers 16-byte aligned;
+ *   out_idx [rows][k] int32, out_val [rows][k] fp32 (the fp32-accumulated logits);
+ *           k in 1 .. 16.
+ * Logits are accumulated in fp32 by the tensor cores in an order of their own: entries
+ * within ~1e-6 relative of each other may swap places against an exact evaluation.
+ * workspace: ptd_lm_head_topk_workspace_size(rows, vocab) bytes, 16-byte aligned (per-CTA
+ * candidate lists).  Two launches: the product with per-CTA top-k, then a per-row merge. */
+size_t ptd_lm_head_topk_workspace_size(int32_t rows, int32_t vocab);
+ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_stride, const void* weight,
+                            int32_t vocab, int64_t weight_stride, int32_t d_model, int32_t k, int32_t* out_idx,
+                            float* out_val, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                            void* stream);
 
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.

@@ -16,6 +16,7 @@
 #include "draft_update.cuh"
 #include "pool.cuh"
 #include "tree_rope.cuh"
+#include "lm_head.cuh"
 #include "attention.cuh"
 #include "topk.cuh"
 #include "verify_compact.cuh"
@@ -429,6 +430,47 @@ ptd_status ptd_tree_rope_append(const ptd_tree* tree, const ptd_kv_cache* cache,
                                          cache->num_pages, cache->block_table, cache->max_pages, f, positions_out,
                                          dev_status, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+size_t ptd_lm_head_topk_workspace_size(int32_t rows, int32_t vocab) {
+  if (rows < 1 || rows > PTD_MAX_TREE_NODES || vocab < 1) return 0;
+  return ptd::lm_head_workspace_bytes(ptd::lm_head_ctas(num_sms_of_current_device(), vocab), rows);
+}
+
+ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_stride, const void* weight,
+                            int32_t vocab, int64_t weight_stride, int32_t d_model, int32_t k, int32_t* out_idx,
+                            float* out_val, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                            void* stream) {
+  g_last_launches = 0;
+  if (!hidden || !weight || !out_idx || !out_val || !dev_status) return PTD_ERR_INVALID_ARG;
+  if (rows < 1 || rows > PTD_MAX_TREE_NODES || d_model < 64 || d_model % 64 != 0 || k < 1 || k > ptd::kLmMaxK ||
+      vocab < k || hidden_stride < d_model || weight_stride < d_model || hidden_stride % 8 != 0 ||
+      weight_stride % 8 != 0 || !aligned16(hidden) || !aligned16(weight))
+    return PTD_ERR_INVALID_ARG;
+  const int ctas = ptd::lm_head_ctas(num_sms_of_current_device(), vocab);
+  if (!workspace || workspace_bytes < ptd::lm_head_workspace_bytes(ctas, rows) || !aligned16(workspace))
+    return PTD_ERR_WORKSPACE;
+  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+  if (!enc) return PTD_ERR_CUDA;
+  CUtensorMap map_h, map_w;
+  const cuuint32_t box[2] = {64, 128}, estride[2] = {1, 1};
+  const cuuint64_t hdim[2] = {(cuuint64_t)d_model, (cuuint64_t)rows};
+  const cuuint64_t hstride[1] = {(cuuint64_t)hidden_stride * 2};
+  const cuuint64_t wdim[2] = {(cuuint64_t)d_model, (cuuint64_t)vocab};
+  const cuuint64_t wstride[1] = {(cuuint64_t)weight_stride * 2};
+  if (enc(&map_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(hidden), hdim, hstride, box, estride,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return PTD_ERR_CUDA;
+  if (enc(&map_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(weight), wdim, wstride, box, estride,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return PTD_ERR_CUDA;
+  const ptd_status st = cuda_status(ptd::launch_lm_head_topk(map_h, map_w, rows, d_model, vocab, k, out_idx, out_val,
+                                                              workspace, ctas, dev_status,
+                                                              static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 2;
   return st;
 }
 

@@ -29,7 +29,7 @@ EXPORTED = (
     "ptd_kv_compact", "ptd_tree_verify_step", "ptd_tree_verify_step_host", "ptd_last_launch_count",
     "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact", "ptd_verify_sampling",
     "ptd_draft_tree_update", "ptd_pool_bytes", "ptd_pool_init", "ptd_pool_merge", "ptd_pool_retrieve",
-    "ptd_tree_rope_append",
+    "ptd_tree_rope_append", "ptd_lm_head_topk_workspace_size", "ptd_lm_head_topk",
 )
 
 
@@ -113,6 +113,10 @@ def lib() -> ctypes.CDLL:
         L.ptd_pool_retrieve.argtypes = [vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]
         L.ptd_tree_rope_append.restype = ctypes.c_int
         L.ptd_tree_rope_append.argtypes = [P(_Tree), P(_Cache), i32, i32, vp, i32, vp, vp, f32, vp, vp, vp]
+        L.ptd_lm_head_topk_workspace_size.restype = sz
+        L.ptd_lm_head_topk_workspace_size.argtypes = [i32, i32]
+        L.ptd_lm_head_topk.restype = ctypes.c_int
+        L.ptd_lm_head_topk.argtypes = [vp, i32, i64, vp, i32, i64, i32, i32, vp, vp, vp, sz, vp, vp]
         L.ptd_tree_verify_step.restype = ctypes.c_int
         L.ptd_tree_verify_step.argtypes = [P(_Tree), P(_Cache), P(_StepArgs), vp]
         L.ptd_tree_verify_step_host.restype = ctypes.c_int
@@ -411,4 +415,23 @@ def tree_rope_append(tree: Tree, cache: KVCache, layer_begin: int, q: torch.Tens
                                     None if positions_out is None else _dev(positions_out, "positions_out", torch.int32),
                                     _dev(dev_status, "dev_status", torch.int32), _stream(stream))
     _check(st, "ptd_tree_rope_append")
+    return last_launch_count()
+
+
+def lm_head_workspace_size(rows: int, vocab: int) -> int:
+    return int(lib().ptd_lm_head_topk_workspace_size(int(rows), int(vocab)))
+
+
+def lm_head_topk(hidden: torch.Tensor, weight: torch.Tensor, k: int, out_idx: torch.Tensor, out_val: torch.Tensor,
+                 workspace: torch.Tensor, dev_status: torch.Tensor, stream=None) -> int:
+    """ptd_lm_head_topk: hidden [rows, d] and weight [vocab, d] bf16 (rows may be strided)."""
+    if hidden.dim() != 2 or weight.dim() != 2 or hidden.shape[1] != weight.shape[1]:
+        raise ValueError("hidden [rows, d] and weight [vocab, d] must share d")
+    st = lib().ptd_lm_head_topk(_dev(hidden, "hidden", torch.bfloat16, row_strided=True), hidden.shape[0],
+                                hidden.stride(0), _dev(weight, "weight", torch.bfloat16, row_strided=True),
+                                weight.shape[0], weight.stride(0), hidden.shape[1], int(k),
+                                _dev(out_idx, "out_idx", torch.int32), _dev(out_val, "out_val", torch.float32),
+                                _dev(workspace, "workspace"), workspace.numel() * workspace.element_size(),
+                                _dev(dev_status, "dev_status", torch.int32), _stream(stream))
+    _check(st, "ptd_lm_head_topk")
     return last_launch_count()
