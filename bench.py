@@ -35,7 +35,11 @@ WORKLOAD = "llama3-8b-gqa"
 # DRAM bytes (read + write) of one full 32-layer attention launch from an ncu capture
 # (19-layer case scaled by 32/19; traffic grows with the layer count), keyed by the
 # sha256 prefix of the kernel source it was taken on.  A changed kernel reports null.
-PROFILED_ATTENTION_TRAFFIC = {"5ff2a101cd14a326": 1115897424}
+# dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture of the full
+# Llama-3-8B-shaped workload (mean of two launches), keyed by the kernel source's sha256
+# prefix: a changed kernel reports null until it is captured again
+PROFILED_ATTENTION_TRAFFIC = {"6a37ec05ccfb7d53": 1162815616}
+PROFILED_LM_HEAD_TRAFFIC = {"541fa109411fd935": 1053963264}
 MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
@@ -126,13 +130,15 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(inside)}
 
 
-def _attention_traffic(layers: int):
+def _profiled_traffic(table: dict, source: str):
     import hashlib
 
-    src = os.path.join(ROOT, "paper_2607_10661_gb300", "csrc", "attention_tc.cu")
-    with open(src, "rb") as f:
-        sha = hashlib.sha256(f.read()).hexdigest()[:16]
-    t = PROFILED_ATTENTION_TRAFFIC.get(sha)
+    with open(os.path.join(ROOT, "paper_2607_10661_gb300", "csrc", source), "rb") as f:
+        return table.get(hashlib.sha256(f.read()).hexdigest()[:16])
+
+
+def _attention_traffic(layers: int):
+    t = _profiled_traffic(PROFILED_ATTENTION_TRAFFIC, "attention_tc.cu")
     return None if t is None or layers != 32 else t
 
 
@@ -365,7 +371,10 @@ def run_gpu(args, rank: int, world: int, dist):
                      "bytes_per_launch": int(lm_w.numel() * 2 + lm_h.numel() * 2),
                      "achieved_gbs": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9, 1),
                      "frac": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9
-                                   / _peak_hbm()[0], 4), "peak_kind": _peak_hbm()[1]}
+                                   / _peak_hbm()[0], 4), "peak_kind": _peak_hbm()[1],
+                     "traffic": (_profiled_traffic(PROFILED_LM_HEAD_TRAFFIC, "lm_head.cu")
+                                 if cfg.vocab == 128256 else None),
+                     "note": "two launches: the product with per-CTA top-k, then the per-row merge"}
                     if args.lm_head else None),
         "gpu_launches": int(launches),
         "status": ptd.status_string(status),
