@@ -317,13 +317,45 @@ def run_gpu(args, rank: int, world: int, dist):
         stream.synchronize()             # the host reads the step's result before the next step
     e1.record(stream)
     torch.cuda.synchronize()
+    sync_ms = e0.elapsed_time(e1)
+    sync_ok = int(io_t["status_h"][0]) == 0
+    # the same steps through the pipelined host-buffer API: step i + 1's uploads and step
+    # i - 1's downloads overlap step i's computation; the host reads every step's result
+    tree_b, bufs_b = dw.twin_step_buffers()
+    stage_n = 2 * L * N * cfg.hkv * cfg.d * dw.k.element_size()
+    staging = [torch.empty(stage_n, dtype=torch.uint8, device=f"cuda:{local}") for _ in range(2)]
+    pipe = ptd.Pipeline(dw.cache, (dw.tree, tree_b), (dw.bufs, bufs_b), staging)
+    io_t2 = {k: (pin(v.clone()) if k in ("topk_idx_h", "topk_val_h", "accepted_h", "accept_len_h", "bonus_h",
+                                         "new_ctx_h", "status_h") else v) for k, v in io_t.items()}
+    ios = [io, ptd.HostIO(**io_t2)]
+    outs_t = [io_t, io_t2]
+
+    def run_pipeline(n):
+        ok, prev = True, None
+        for i in range(n):
+            tk = pipe.submit(ios[i & 1])
+            if prev is not None:
+                pipe.wait(prev)
+                ok = ok and int(outs_t[(i - 1) & 1]["status_h"][0]) == 0
+            prev = tk
+        pipe.wait(prev)
+        return ok and int(outs_t[(n - 1) & 1]["status_h"][0]) == 0
+
+    run_pipeline(4)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    e0.record(stream)
+    e2e_ok = run_pipeline(Ke) and sync_ok
+    e1.record(stream)
+    torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
-    e2e_ok = int(io_t["status_h"][0]) == 0
+    pipe.close()
 
     if dist is not None:
-        t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device=f"cuda:{local}")
+        t = torch.tensor([ms, e2e_ms, sync_ms], dtype=torch.float64, device=f"cuda:{local}")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, e2e_ms = float(t[0]), float(t[1])
+        ms, e2e_ms, sync_ms = float(t[0]), float(t[1]), float(t[2])
 
     peak, peak_kind = _peak_hbm()
     achieved = nb["attention"] / (attn_ms * 1e-3) / 1e9
@@ -366,7 +398,11 @@ def run_gpu(args, rank: int, world: int, dist):
         "clocks": clocks,
         "e2e": {"value": round(world * Ke / (e2e_ms * 1e-3), 3), "unit": "steps/s", "steps": Ke,
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "status_ok": e2e_ok,
-                "verify": "greedy (the host step call)"},
+                "verify": "greedy",
+                "api": "ptd_pipeline_submit / ptd_pipeline_wait (uploads and downloads overlapped with compute, "
+                       "two steps in flight); every step's inputs uploaded from pinned host memory and its result "
+                       "read by the host",
+                "one_step_call_value": round(world * Ke / (sync_ms * 1e-3), 3)},
         "lm_head": ({"kernel": "lm_head_topk_kernel", "avg_launch_ms": round(lm_ms, 5),
                      "bytes_per_launch": int(lm_w.numel() * 2 + lm_h.numel() * 2),
                      "achieved_gbs": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9, 1),

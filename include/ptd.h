@@ -387,6 +387,28 @@ ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* c
                                      const ptd_step_args* args, const ptd_host_io* io,
                                      void* stream);
 
+/* Host-buffer steps with the copies overlapped (a software pipeline over two device buffer
+ * sets): step i + 1's inputs go up, and step i - 1's results come down, while step i
+ * computes.  Each submitted step is ptd_tree_verify_step_host's step (the same inputs,
+ * outputs and rules; contiguous caches only), except that the tree's K/V rows first land
+ * in a staging buffer and reach the cache slots from there at the start of the step's
+ * computation, so that an upload never touches rows the previous step still reads.
+ *   trees[2], args[2]: two complete sets of device buffers (slot s serves steps
+ *           s, s + 2, ...); they share `cache`.
+ *   staging[2]: device buffers of at least 2 * L * N_tot * Hkv * D elements each.
+ *   compute_stream: where the steps compute, in submission order.
+ * The pipeline creates two streams and six events of its own (freed by destroy); the
+ * device memory stays the caller's.  submit enqueues one step and returns its ticket; the
+ * step's host outputs are valid once wait(ticket) returns.  A step's `io` buffers must
+ * stay untouched until then; alternate two `io` sets to keep two steps in flight. */
+typedef struct ptd_pipeline ptd_pipeline;
+ptd_status ptd_pipeline_create(const ptd_kv_cache* cache, const ptd_tree* trees, const ptd_step_args* args,
+                               void* const* staging, size_t staging_bytes, void* compute_stream,
+                               ptd_pipeline** out);
+ptd_status ptd_pipeline_submit(ptd_pipeline* pipeline, const ptd_host_io* io, int64_t* ticket);
+ptd_status ptd_pipeline_wait(ptd_pipeline* pipeline, int64_t ticket);
+ptd_status ptd_pipeline_destroy(ptd_pipeline* pipeline);
+
 /* Number of kernels the last successful call of each entry point enqueued on this
  * host thread (a diagnostic for launch accounting). */
 int32_t ptd_last_launch_count(void);

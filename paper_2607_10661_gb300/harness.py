@@ -81,3 +81,19 @@ class DeviceWorkload:
 
     def compact(self, stream=None) -> int:
         return ptd.kv_compact(self.tree, self.cache, self.accepted, self.accept_len, self.new_ctx, stream=stream)
+
+    def twin_step_buffers(self):
+        """A second (Tree, StepBuffers) set of the same shapes over the same cache: the other
+        slot of a two-deep pipeline (ptd.Pipeline).  Nothing is shared with this set."""
+        w, c, dev = self.w, self.w.cfg, self.device
+        i32 = dict(dtype=torch.int32, device=dev)
+        node_offsets, parents, ctx_lens = self.node_offsets.clone(), self.parents.clone(), self.ctx_lens.clone()
+        tree = ptd.Tree(node_offsets, parents, ctx_lens, w.max_nodes, w.max_ctx)
+        tree.keep = (node_offsets, parents, ctx_lens)
+        ws = torch.empty_like(self.workspace) if self.workspace is not None else None
+        bufs = ptd.StepBuffers(self.q.clone(), c.hq, torch.zeros_like(self.attn_out), self.logits.clone(), c.k,
+                               self.tokens.clone(), torch.zeros_like(self.topk_idx), torch.zeros_like(self.topk_val),
+                               torch.zeros_like(self.accepted), torch.zeros((c.batch,), **i32),
+                               torch.zeros((c.batch,), **i32), torch.zeros((c.batch,), **i32),
+                               torch.zeros(1, **i32), ws)
+        return tree, bufs

@@ -29,7 +29,8 @@ EXPORTED = (
     "ptd_kv_compact", "ptd_tree_verify_step", "ptd_tree_verify_step_host", "ptd_last_launch_count",
     "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact", "ptd_verify_sampling",
     "ptd_draft_tree_update", "ptd_pool_bytes", "ptd_pool_init", "ptd_pool_merge", "ptd_pool_retrieve",
-    "ptd_tree_rope_append", "ptd_lm_head_topk_workspace_size", "ptd_lm_head_topk",
+    "ptd_tree_rope_append", "ptd_lm_head_topk_workspace_size", "ptd_lm_head_topk", "ptd_pipeline_create",
+    "ptd_pipeline_submit", "ptd_pipeline_wait", "ptd_pipeline_destroy",
 )
 
 
@@ -117,6 +118,14 @@ def lib() -> ctypes.CDLL:
         L.ptd_lm_head_topk_workspace_size.argtypes = [i32, i32]
         L.ptd_lm_head_topk.restype = ctypes.c_int
         L.ptd_lm_head_topk.argtypes = [vp, i32, i64, vp, i32, i64, i32, i32, vp, vp, vp, sz, vp, vp]
+        L.ptd_pipeline_create.restype = ctypes.c_int
+        L.ptd_pipeline_create.argtypes = [P(_Cache), P(_Tree), P(_StepArgs), P(vp), sz, vp, P(vp)]
+        L.ptd_pipeline_submit.restype = ctypes.c_int
+        L.ptd_pipeline_submit.argtypes = [vp, P(_HostIO), P(i64)]
+        L.ptd_pipeline_wait.restype = ctypes.c_int
+        L.ptd_pipeline_wait.argtypes = [vp, i64]
+        L.ptd_pipeline_destroy.restype = ctypes.c_int
+        L.ptd_pipeline_destroy.argtypes = [vp]
         L.ptd_tree_verify_step.restype = ctypes.c_int
         L.ptd_tree_verify_step.argtypes = [P(_Tree), P(_Cache), P(_StepArgs), vp]
         L.ptd_tree_verify_step_host.restype = ctypes.c_int
@@ -435,3 +444,38 @@ def lm_head_topk(hidden: torch.Tensor, weight: torch.Tensor, k: int, out_idx: to
                                 _dev(dev_status, "dev_status", torch.int32), _stream(stream))
     _check(st, "ptd_lm_head_topk")
     return last_launch_count()
+
+
+class Pipeline:
+    """ptd_pipeline_*: host-buffer steps with uploads and downloads overlapped with compute.
+    trees, bufs: two Tree / StepBuffers sets sharing `cache`; staging: two device byte
+    tensors of at least 2 * L * N_tot * Hkv * D elements."""
+
+    def __init__(self, cache: KVCache, trees, bufs, staging, stream=None):
+        self.keep = (cache, trees, bufs, staging)
+        tr = (_Tree * 2)(trees[0].c, trees[1].c)
+        ar = (_StepArgs * 2)(bufs[0].c, bufs[1].c)
+        st = (ctypes.c_void_p * 2)(_dev(staging[0], "staging"), _dev(staging[1], "staging"))
+        nbytes = min(x.numel() * x.element_size() for x in staging)
+        self.h = ctypes.c_void_p()
+        _check(lib().ptd_pipeline_create(ctypes.byref(cache.c), tr, ar, st, nbytes, _stream(stream),
+                                         ctypes.byref(self.h)), "ptd_pipeline_create")
+
+    def submit(self, io: "HostIO") -> int:
+        t = ctypes.c_int64()
+        _check(lib().ptd_pipeline_submit(self.h, ctypes.byref(io.c), ctypes.byref(t)), "ptd_pipeline_submit")
+        return t.value
+
+    def wait(self, ticket: int) -> None:
+        _check(lib().ptd_pipeline_wait(self.h, int(ticket)), "ptd_pipeline_wait")
+
+    def close(self) -> None:
+        if self.h:
+            lib().ptd_pipeline_destroy(self.h)
+            self.h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
