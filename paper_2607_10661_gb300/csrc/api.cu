@@ -243,9 +243,23 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return PTD_ERR_CUDA;
 
+  // Q tiles by TMA: one M tile is 128 / G nodes x G heads, a 3-D box over [rows][Hq][D]
+  CUtensorMap map_q;
+  std::memset(&map_q, 0, sizeof(map_q));
+  const int G = p.group;
+  p.q_tma = 0;
+  if (G >= 1 && G <= 128 && 128 % G == 0 && aligned16(q)) {
+    const cuuint64_t qdim[3] = {(cuuint64_t)D, (cuuint64_t)num_q_heads, (cuuint64_t)num_layers * tree->total_nodes};
+    const cuuint64_t qstride[2] = {(cuuint64_t)D * 2, (cuuint64_t)num_q_heads * D * 2};
+    const cuuint32_t qbox[3] = {64, (cuuint32_t)G, (cuuint32_t)(128 / G)};
+    if (enc(&map_q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), qdim, qstride, qbox, estride,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS)
+      p.q_tma = 1;
+  }
   if (persistent && cudaMemsetAsync(p.counters, 0, (size_t)units * 8 * sizeof(int32_t), s) != cudaSuccess)
     return PTD_ERR_CUDA;
-  if ((st = cuda_status(ptd::launch_tree_attn_tc(map_k, map_v, p, grid, s))) != PTD_OK) return st;
+  if ((st = cuda_status(ptd::launch_tree_attn_tc(map_k, map_v, map_q, p, grid, s))) != PTD_OK) return st;
   g_last_launches = 1;   // (the counter clear before it is a memset, not a kernel of this library)
   return PTD_OK;
 }

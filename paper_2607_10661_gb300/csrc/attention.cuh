@@ -27,14 +27,15 @@ struct AttnParams {
   int n_total, max_nodes;
   int pairs;                   // 256-row M-tile pairs per (tree, KV head)
   int persistent;              // 1: balanced persistent schedule, one CTA per SM
+  int q_tma;                   // 1: Q tiles arrive by TMA (map_q), else by per-thread loads
   int page_size, seq_capacity, num_pages, max_pages;
   float scale_log2;            // scale * log2(e)
   float scale;
 };
 
 size_t tc_smem_bytes();
-cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const AttnParams& p,
-                                dim3 grid, cudaStream_t stream);
+cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const CUtensorMap& map_q,
+                                const AttnParams& p, dim3 grid, cudaStream_t stream);
 cudaError_t launch_tree_attn_simt(const AttnParams& p, cudaStream_t stream);
 
 }  // namespace ptd

@@ -282,10 +282,10 @@ __device__ __noinline__ void rescale_tmem(uint32_t tO, uint32_t tS, int n_o, int
   }
 }
 
-template <bool kPaged>
+template <bool kPaged, bool kQTma>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
-                        const AttnParams p) {
+                        const __grid_constant__ CUtensorMap map_q, const AttnParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint32_t base = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
@@ -328,7 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(sfull_bar(t), 1);
       mbar_init(pfull_bar(t), 4);    // one arrival per softmax warp
       mbar_init(ofull_bar(t), 1);
-      mbar_init(qready_bar(t), 4);   // one arrival per softmax warp
+      mbar_init(qready_bar(t), kQTma ? 1 : 4);   // the TMA issuer, or one arrival per softmax warp
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
@@ -563,9 +563,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int node = grow / G, g = grow - node * G;
       const bool row_valid = node < T;
       const bool has_keys = sgv->kt_end > sgv->kt_begin;
-      // Q rows first: their loads overlap the tree work below
+      // Q rows first: their loads overlap the tree work below (per-thread path only)
       uint4 v[16];
-      {
+      if constexpr (!kQTma) {
         const size_t orow = (((size_t)sgv->lq * p.n_total + node0 + node) * p.hq + (size_t)sgv->hkv * G + g) * 128;
         const uint4* srcq = reinterpret_cast<const uint4*>(p.q) + (row_valid ? orow : 0) / 8;
 #pragma unroll
@@ -611,7 +611,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane < kSegWords)
         reinterpret_cast<volatile int*>(&wa->run[k].s)[lane] = reinterpret_cast<const volatile int*>(sgv)[lane];
       if (lane == 0) wa->run[k].invalid = invalid ? 1 : 0;
-      if (has_keys) {
+      if (kQTma && has_keys) {
+        // Q tile of this segment by TMA (every S_t GEMM of the previous segment has
+        // completed): 128 / G nodes x G heads of the pair's M tile, two 64-column halves
+        if ((warp & 3) == 0 && lane == 0) {
+          const int qrow = sgv->lq * p.n_total + node0 + ((2 * mp + t) * 128) / G;
+          const uint32_t dst = base + kOffQ + (uint32_t)t * kTileBytes;
+          mbar_arrive_expect_tx(qready_bar(t), 2 * kHalfBytes);
+          tma_load_3d(dst, &map_q, qready_bar(t), 0, sgv->hkv * G, qrow);
+          tma_load_3d(dst + kHalfBytes, &map_q, qready_bar(t), 64, sgv->hkv * G, qrow);
+        }
+      } else if (has_keys) {
         // Q rows of this segment (every S_t GEMM of the previous segment has completed)
 #pragma unroll
         for (int c = 0; c < 16; ++c) {
@@ -892,19 +902,28 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ------------------------------------------------------------------- host launchers
 size_t tc_smem_bytes() { return tc::kSmemBytes; }
 
-cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const AttnParams& p,
-                                dim3 grid, cudaStream_t stream) {
+cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const CUtensorMap& map_q,
+                                const AttnParams& p, dim3 grid, cudaStream_t stream) {
+#define PTD_TC_LAUNCH(PAGED, QTMA)                                                                            \
+  do {                                                                                                       \
+    cudaError_t e = cudaFuncSetAttribute(tc::tree_attn_tc_kernel<PAGED, QTMA>,                               \
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc::kSmemBytes);  \
+    if (e != cudaSuccess) return e;                                                                          \
+    tc::tree_attn_tc_kernel<PAGED, QTMA><<<grid, tc::kThreads, tc::kSmemBytes, stream>>>(map_k, map_v, map_q, \
+                                                                                          p);               \
+  } while (0)
   if (p.page_size > 0) {
-    cudaError_t e = cudaFuncSetAttribute(tc::tree_attn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)tc::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    tc::tree_attn_tc_kernel<true><<<grid, tc::kThreads, tc::kSmemBytes, stream>>>(map_k, map_v, p);
+    if (p.q_tma)
+      PTD_TC_LAUNCH(true, true);
+    else
+      PTD_TC_LAUNCH(true, false);
   } else {
-    cudaError_t e = cudaFuncSetAttribute(tc::tree_attn_tc_kernel<false>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    tc::tree_attn_tc_kernel<false><<<grid, tc::kThreads, tc::kSmemBytes, stream>>>(map_k, map_v, p);
+    if (p.q_tma)
+      PTD_TC_LAUNCH(false, true);
+    else
+      PTD_TC_LAUNCH(false, false);
   }
+#undef PTD_TC_LAUNCH
   return cudaGetLastError();
 }
 
