@@ -142,6 +142,24 @@ def _attention_traffic(layers: int):
     return None if t is None or layers != 32 else t
 
 
+def reduce_over_ranks(dist, values, device="cpu"):
+    """Each value's maximum over the ranks (every rank gets it); the values themselves with
+    one process.  The timed steps of every rank are bracketed by barriers, so the slowest
+    rank's time is the job's."""
+    if dist is None:
+        return [float(v) for v in values]
+    import torch
+
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
+def aggregate_rate(world: int, steps: int, ms: float) -> float:
+    """Whole-job steps/s: every rank ran `steps` steps of its own replica in `ms` (max)."""
+    return world * steps / (ms * 1e-3)
+
+
 def _peak_hbm():
     try:
         with open(MEASURED_PEAKS) as f:
@@ -352,15 +370,12 @@ def run_gpu(args, rank: int, world: int, dist):
     e2e_ms = e0.elapsed_time(e1)
     pipe.close()
 
-    if dist is not None:
-        t = torch.tensor([ms, e2e_ms, sync_ms], dtype=torch.float64, device=f"cuda:{local}")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, e2e_ms, sync_ms = float(t[0]), float(t[1]), float(t[2])
+    ms, e2e_ms, sync_ms = reduce_over_ranks(dist, [ms, e2e_ms, sync_ms], f"cuda:{local}")
 
     peak, peak_kind = _peak_hbm()
     achieved = nb["attention"] / (attn_ms * 1e-3) / 1e9
     ms_step = ms / K
-    value = world * K / (ms * 1e-3)
+    value = aggregate_rate(world, K, ms)
     flops = attention_flops(w)
     out = {
         "metric": "tree-verify steps/sec (HBM GB/s and fraction of ~8 TB/s alongside)",
@@ -396,13 +411,13 @@ def run_gpu(args, rank: int, world: int, dist):
                      "avg_launch_ms": round(attn_ms, 5),
                      "tensor_tflops": round(flops / (attn_ms * 1e-3) / 1e12, 1)},
         "clocks": clocks,
-        "e2e": {"value": round(world * Ke / (e2e_ms * 1e-3), 3), "unit": "steps/s", "steps": Ke,
+        "e2e": {"value": round(aggregate_rate(world, Ke, e2e_ms), 3), "unit": "steps/s", "steps": Ke,
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "status_ok": e2e_ok,
                 "verify": "greedy",
                 "api": "ptd_pipeline_submit / ptd_pipeline_wait (uploads and downloads overlapped with compute, "
                        "two steps in flight); every step's inputs uploaded from pinned host memory and its result "
                        "read by the host",
-                "one_step_call_value": round(world * Ke / (sync_ms * 1e-3), 3)},
+                "one_step_call_value": round(aggregate_rate(world, Ke, sync_ms), 3)},
         "lm_head": ({"kernel": "lm_head_topk_kernel", "avg_launch_ms": round(lm_ms, 5),
                      "bytes_per_launch": int(lm_w.numel() * 2 + lm_h.numel() * 2),
                      "achieved_gbs": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9, 1),
@@ -496,12 +511,12 @@ def cpu_baseline(budget_s: float, sampling: bool = False) -> dict:
 
 def run_reference(args):
     """--impl reference: the CPU oracle on the host cores, one bounded sample per step; the
-    run stops early (reporting the steps it timed) once about 150 s of samples are taken."""
+    run stops early (reporting the steps it timed) once about --ref-seconds of samples are taken."""
     from paper_2607_10661_gb300 import synthetic as syn
 
     cfg = syn.CONFIGS[WORKLOAD]
     try:
-        per = oracle_samples(args.steps, min(args.warmup, 1), 150.0, args.verify == "sampling")
+        per = oracle_samples(args.steps, min(args.warmup, 1), args.ref_seconds, args.verify == "sampling")
     except Exception as e:
         return {"impl": "reference", "unavailable": "oracle sample failed: " + str(e)[-200:]}
     sec = float(np.mean(per))
@@ -526,6 +541,8 @@ def main():
     ap.add_argument("--impl", default="ptd", choices=["ptd", "reference"])
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling captures)")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
+    ap.add_argument("--ref-seconds", type=float, default=150.0,
+                    help="--impl reference: stop sampling the oracle after about this many seconds")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--lm-head", action="store_true",
                     help="top-k from the LM head (ptd_lm_head_topk, logits never written) instead of from "

@@ -1,0 +1,79 @@
+"""The multi-process path of bench.py on the CPU (gloo, world size 2): the step does not
+shard, so N GPUs run N independent replicas; what crosses ranks is the timing protocol (the
+slowest rank's times, every rank's steps in the whole-job rate) and, for the reference arm,
+that rank 0 alone runs and prints while the others exit 0."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, q):
+    sys.path.insert(0, ROOT)
+    import bench
+
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world)
+    try:
+        dist.barrier()
+        # each rank's own timings: rank 1 is the slow one for the first, rank 0 for the second
+        mine = [10.0 + 5.0 * rank, 20.0 - 3.0 * rank, 7.0]
+        got = bench.reduce_over_ranks(dist, mine)
+        dist.barrier()
+        q.put((rank, got, bench.aggregate_rate(world, 100, got[0])))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_timing_protocol_over_two_gloo_ranks():
+    world, port = 2, _free_port()
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    procs = [ctx.Process(target=_rank_main, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    out = [q.get(timeout=120) for _ in range(world)]
+    for p in procs:
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    for rank, got, rate in out:
+        assert got == [15.0, 20.0, 7.0]            # the maximum over the ranks, on every rank
+        assert rate == pytest.approx(2 * 100 / 15e-3)   # both replicas' steps over the slowest time
+    assert sorted(r for r, _, _ in out) == [0, 1]
+
+
+def test_single_process_reduction_is_identity():
+    sys.path.insert(0, ROOT)
+    import bench
+
+    assert bench.reduce_over_ranks(None, [1, 2.5]) == [1.0, 2.5]
+    assert bench.aggregate_rate(1, 50, 20.0) == pytest.approx(2500.0)
+
+
+def test_reference_arm_under_torchrun_prints_once():
+    """`bench.py --impl reference` launched as the driver launches it for N = 2: rank 0 runs the
+    oracle and prints one JSON line, the other rank exits 0 without work."""
+    port = _free_port()
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2", "--master-addr",
+           "127.0.0.1", "--master-port", str(port), os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus",
+           "2", "--steps", "2", "--warmup", "1", "--ref-seconds", "5"]
+    r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=300,
+                       env=dict(os.environ, CUDA_VISIBLE_DEVICES="", OMP_NUM_THREADS="1"))
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["value"] > 0 and d["n_gpus"] == 2 and d["unit"] == "steps/s"
