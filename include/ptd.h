@@ -409,6 +409,12 @@ ptd_status ptd_pipeline_submit(ptd_pipeline* pipeline, const ptd_host_io* io, in
 ptd_status ptd_pipeline_wait(ptd_pipeline* pipeline, int64_t ticket);
 ptd_status ptd_pipeline_destroy(ptd_pipeline* pipeline);
 
+/* Diagnostic of the failure path: one thread waits on an mbarrier that nothing arrives on,
+ * through the bounded wait every kernel here uses; after its limit (2 s of %globaltimer)
+ * it atomicMax'es PTD_ERR_TIMEOUT into dev_status and the kernel returns, the context
+ * still usable.  No fault, trap or endless loop is involved. */
+ptd_status ptd_check_bounded_wait(int32_t* dev_status, void* stream);
+
 /* Number of kernels the last successful call of each entry point enqueued on this
  * host thread (a diagnostic for launch accounting). */
 int32_t ptd_last_launch_count(void);

@@ -17,6 +17,10 @@
 #include "pool.cuh"
 #include "tree_rope.cuh"
 #include "lm_head.cuh"
+
+namespace ptd {
+cudaError_t launch_bounded_wait_check(int32_t* dev_status, cudaStream_t stream);
+}
 #include "attention.cuh"
 #include "topk.cuh"
 #include "verify_compact.cuh"
@@ -443,6 +447,14 @@ ptd_status ptd_tree_rope_append(const ptd_tree* tree, const ptd_kv_cache* cache,
                                          cache->seq_capacity,
                                          cache->num_pages, cache->block_table, cache->max_pages, f, positions_out,
                                          dev_status, static_cast<cudaStream_t>(stream)));
+  if (st == PTD_OK) g_last_launches = 1;
+  return st;
+}
+
+ptd_status ptd_check_bounded_wait(int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  if (!dev_status) return PTD_ERR_INVALID_ARG;
+  const ptd_status st = cuda_status(ptd::launch_bounded_wait_check(dev_status, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }

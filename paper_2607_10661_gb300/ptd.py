@@ -30,7 +30,7 @@ EXPORTED = (
     "ptd_status_string", "ptd_tree_attention_noalloc", "ptd_verify_and_compact", "ptd_verify_sampling",
     "ptd_draft_tree_update", "ptd_pool_bytes", "ptd_pool_init", "ptd_pool_merge", "ptd_pool_retrieve",
     "ptd_tree_rope_append", "ptd_lm_head_topk_workspace_size", "ptd_lm_head_topk", "ptd_pipeline_create",
-    "ptd_pipeline_submit", "ptd_pipeline_wait", "ptd_pipeline_destroy",
+    "ptd_pipeline_submit", "ptd_pipeline_wait", "ptd_pipeline_destroy", "ptd_check_bounded_wait",
 )
 
 
@@ -126,6 +126,8 @@ def lib() -> ctypes.CDLL:
         L.ptd_pipeline_wait.argtypes = [vp, i64]
         L.ptd_pipeline_destroy.restype = ctypes.c_int
         L.ptd_pipeline_destroy.argtypes = [vp]
+        L.ptd_check_bounded_wait.restype = ctypes.c_int
+        L.ptd_check_bounded_wait.argtypes = [vp, vp]
         L.ptd_tree_verify_step.restype = ctypes.c_int
         L.ptd_tree_verify_step.argtypes = [P(_Tree), P(_Cache), P(_StepArgs), vp]
         L.ptd_tree_verify_step_host.restype = ctypes.c_int
@@ -479,3 +481,10 @@ class Pipeline:
             self.close()
         except Exception:
             pass
+
+
+def check_bounded_wait(dev_status: torch.Tensor, stream=None) -> int:
+    """ptd_check_bounded_wait: a wait that runs out, reported as PTD_ERR_TIMEOUT."""
+    _check(lib().ptd_check_bounded_wait(_dev(dev_status, "dev_status", torch.int32), _stream(stream)),
+           "ptd_check_bounded_wait")
+    return last_launch_count()
