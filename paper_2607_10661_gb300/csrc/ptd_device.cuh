@@ -107,6 +107,13 @@ __device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity, unsign
   }
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// Block until the preceding grid in the stream has completed and its writes are visible.
+// With a launch that allows programmatic stream serialization, the code before this call
+// (set-up that touches no global memory) overlaps the previous kernel's end; otherwise it
+// returns at once.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---------------------------------------------------------------- proxies and fences
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

@@ -153,6 +153,7 @@ __global__ void __launch_bounds__(kThreads) topk_cluster_kernel(const T* __restr
   const int csize = (int)cluster.num_blocks();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
+  grid_dependency_wait();   // the logits and outputs belong to the stream's previous work
   for (int64_t r = blockIdx.y; r < rows; r += gridDim.y) {
     const T* row = logits + r * row_stride;
     // vector body [a0, a1): 16-byte aligned; head [0, a0) and tail [a1, vocab) scalar
@@ -289,6 +290,7 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
     fence_mbar_init();
   }
   __syncthreads();
+  grid_dependency_wait();   // the logits and outputs belong to the stream's previous work
   uint32_t phase = 0;
 
   for (int64_t r = blockIdx.y; r < rows; r += gridDim.y, phase ^= 1u) {
@@ -501,13 +503,15 @@ cudaError_t launch_km(const T* logits, int64_t rows, int vocab, int64_t row_stri
   cfg.gridDim = dim3((unsigned)cluster, (unsigned)gy, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = (unsigned)cluster;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // set-up overlaps the previous kernel
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   if constexpr (kFast) {
     const int nvec = vocab / 8 + 1;
     const int per = (nvec + cluster - 1) / cluster;

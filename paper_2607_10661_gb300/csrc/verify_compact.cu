@@ -303,6 +303,7 @@ __global__ void __launch_bounds__(kCompactThreads)
   __shared__ int depth_s[kVerifyThreads], onpath_s[kVerifyThreads];
   __shared__ TreeVerdict verdict;
   const int layer = blockIdx.x, b = blockIdx.y;
+  grid_dependency_wait();   // the targets and the cache belong to the stream's previous work
   if (threadIdx.x < 32)
     verify_tree_warp(node_offsets, parents, tokens, target, target_stride, n_total, max_nodes, b, par_s, jump_s,
                      reach_s, depth_s, onpath_s, &verdict);
@@ -381,11 +382,20 @@ cudaError_t launch_verify_compact(const int32_t* node_offsets, const int32_t* pa
                                   void* v, int row_bytes, int layers, int batch, int page_size, int seq_capacity,
                                   int num_pages, const int32_t* block_table, int max_pages, const int32_t* ctx_lens,
                                   int32_t* new_ctx, cudaStream_t stream) {
-  vc::verify_compact_kernel<<<dim3(layers, batch, 2), vc::kCompactThreads, 0, stream>>>(
-      node_offsets, parents, tokens, target, target_stride, n_total, max_nodes, accepted, accept_len, bonus,
-      dev_status, static_cast<uint8_t*>(k), static_cast<uint8_t*>(v), row_bytes, batch, page_size, seq_capacity,
-      num_pages, block_table, max_pages, ctx_lens, new_ctx);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(layers, batch, 2);
+  cfg.blockDim = dim3(vc::kCompactThreads, 1, 1);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // set-up overlaps the previous kernel
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, vc::verify_compact_kernel, node_offsets, parents, tokens, target, target_stride,
+                            n_total, max_nodes, accepted, accept_len, bonus, dev_status, static_cast<uint8_t*>(k),
+                            static_cast<uint8_t*>(v), row_bytes, batch, page_size, seq_capacity, num_pages,
+                            block_table, max_pages, ctx_lens, new_ctx);
 }
 
 cudaError_t launch_compact(void* k, void* v, int row_bytes, int layers, int batch, int page_size, int seq_capacity,
