@@ -302,6 +302,24 @@ def run_gpu(args, rank: int, world: int, dist):
     sampler.stop()
     status = int(dw.dev_status.item())
 
+    # ---- the same step through its one-call entry (ptd_tree_verify_step), with no events
+    # between its launches: there the top-k may start while the attention grid drains
+    step_call_ms, Kc = None, max(10, K // 4)
+    if not (args.lm_head or args.draft_update or args.ptd_step or sampling):
+        for _ in range(3):
+            ptd.tree_verify_step(dw.tree, dw.cache, dw.bufs, stream)
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+        c0.record(stream)
+        for _ in range(Kc):
+            ptd.tree_verify_step(dw.tree, dw.cache, dw.bufs, stream)
+        c1.record(stream)
+        torch.cuda.synchronize()
+        step_call_ms = c0.elapsed_time(c1)
+        status |= int(dw.dev_status.item())
+
     # ---- end to end: pinned host inputs and outputs through ptd_tree_verify_step_host
     N, L = w.n_total, cfg.layers
     C = int(w.ctx_lens[0])
@@ -370,7 +388,9 @@ def run_gpu(args, rank: int, world: int, dist):
     e2e_ms = e0.elapsed_time(e1)
     pipe.close()
 
-    ms, e2e_ms, sync_ms = reduce_over_ranks(dist, [ms, e2e_ms, sync_ms], f"cuda:{local}")
+    ms, e2e_ms, sync_ms, sc_ms = reduce_over_ranks(dist, [ms, e2e_ms, sync_ms, step_call_ms or 0.0],
+                                                   f"cuda:{local}")
+    step_call_ms = sc_ms if step_call_ms is not None else None
 
     peak, peak_kind = _peak_hbm()
     achieved = nb["attention"] / (attn_ms * 1e-3) / 1e9
@@ -411,6 +431,9 @@ def run_gpu(args, rank: int, world: int, dist):
                      "avg_launch_ms": round(attn_ms, 5),
                      "tensor_tflops": round(flops / (attn_ms * 1e-3) / 1e12, 1)},
         "clocks": clocks,
+        "step_call": (None if step_call_ms is None else
+                      {"value": round(aggregate_rate(world, Kc, step_call_ms), 3), "unit": "steps/s", "steps": Kc,
+                       "api": "ptd_tree_verify_step (device buffers, no events between the launches)"}),
         "e2e": {"value": round(aggregate_rate(world, Ke, e2e_ms), 3), "unit": "steps/s", "steps": Ke,
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "status_ok": e2e_ok,
                 "verify": "greedy",

@@ -268,8 +268,8 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
   return PTD_OK;
 }
 
-ptd_status ptd_topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab, int64_t row_stride,
-                          int32_t k, int32_t* out_idx, float* out_val, void* stream) {
+static ptd_status topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab, int64_t row_stride,
+                             int32_t k, int32_t* out_idx, float* out_val, bool early, void* stream) {
   g_last_launches = 0;
   if (!logits || !out_idx || !out_val || rows < 1 || vocab < 1 || row_stride < vocab || k < 1 ||
       k > PTD_MAX_TOPK || k > vocab)
@@ -277,9 +277,14 @@ ptd_status ptd_topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int
   if (dtype != PTD_BF16 && dtype != PTD_F32) return PTD_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(logits) % dtype_size(dtype)) != 0) return PTD_ERR_INVALID_ARG;
   const ptd_status st = cuda_status(ptd::launch_topk(logits, dtype == PTD_BF16, rows, vocab, row_stride, k, out_idx,
-                                                     out_val, nullptr, static_cast<cudaStream_t>(stream)));
+                                                     out_val, nullptr, early, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
+}
+
+ptd_status ptd_topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab, int64_t row_stride,
+                          int32_t k, int32_t* out_idx, float* out_val, void* stream) {
+  return topk_draft(logits, dtype, rows, vocab, row_stride, k, out_idx, out_val, false, stream);
 }
 
 ptd_status ptd_verify_greedy(const ptd_tree* tree, const int32_t* tokens, const int32_t* target,
@@ -508,8 +513,11 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
                                      a->attn_out, a->workspace, a->workspace_bytes, a->dev_status, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
-  st = ptd_topk_draft(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
-                      a->topk_val, stream);
+  // The logits are an input of the step, complete before the attention launch began: the
+  // top-k reads them while the attention grid drains, on the SMs its CTAs leave, and ends
+  // only after it (verification and compaction then wait on the top-k grid alone).
+  st = topk_draft(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
+                  a->topk_val, true, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
   st = ptd_verify_and_compact(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len,

@@ -316,6 +316,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   Seg* my_seg = reinterpret_cast<Seg*>(smem + kOffSched + 64) + warp;   // this warp's schedule slot
   static_assert(64 + (kThreads / 32) * sizeof(Seg) <= kSchedBytes, "schedule area");
 
+  // A grid launched after this one with programmatic stream serialization (the step's top-k)
+  // may be scheduled now; its CTAs take the SMs this grid's CTAs leave at its end.
+  if (threadIdx.x == 0) grid_launch_dependents();
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(fullk_bar(s), 1);

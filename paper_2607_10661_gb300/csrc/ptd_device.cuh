@@ -113,6 +113,12 @@ __device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity, unsign
 // (set-up that touches no global memory) overlaps the previous kernel's end; otherwise it
 // returns at once.
 __device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Let the next grid in the stream (launched with programmatic stream serialization) be
+// scheduled once every CTA of this grid has issued this or exited; its CTAs still find the
+// SMs only as this grid's CTAs leave them.  Nothing is made visible by it.
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 // ---------------------------------------------------------------- proxies and fences
 __device__ __forceinline__ void fence_proxy_async_smem() {
