@@ -483,6 +483,46 @@ def test_step_verify_compact_on_eligible_trees(base, tree, seed):
             assert np.array_equal(w.seq_view(ka[l], b)[:new_ctx], ref[:new_ctx])
 
 
+def test_full_size_step_compaction_after_attention():
+    """The one-call step at the benchmark's size (32 layers, context 8192, 63 nodes, vocab
+    128256), with draft tokens made mostly eligible so the accepted path leaves the first
+    children and the compaction overwrites tree slots that the attention reads.  The top-k of
+    this entry starts while the attention grid drains and the compaction waits on the top-k
+    grid only: every sampled attention output must still match the oracle on the cache as it
+    was before the step, and every layer's cache must hold the compacted path."""
+    w = syn.Workload(syn.CONFIGS["llama3-8b-gqa"], 1001)
+    cfg = w.cfg
+    dw = DeviceWorkload(w)
+    idx_ref, _ = oracle.topk_rows(syn.widen(w.logits, cfg.dtype), cfg.k)
+    greedy = idx_ref[:, 0]
+    par = w.trees[0]
+    rng = np.random.default_rng(7)
+    tokens = w.tokens.copy()
+    # eligible everywhere except the first child of the root, so the path leaves node 1
+    first_child = min(i for i in range(1, len(par)) if par[i] == 0)
+    for i in range(1, len(par)):
+        tokens[i] = greedy[par[i]] if (i != first_child and rng.random() < 0.9) else (greedy[par[i]] + 1) % cfg.vocab
+    dw.tokens.copy_(torch.tensor(tokens, dtype=torch.int32))
+    path, nacc, bonus = oracle.verify_greedy(par, tokens, greedy)
+    assert nacc > 2 and any(path[j] != j for j in range(nacc))
+    k_before = dw.k.cpu().view(torch.int16).numpy()
+    assert dw.step() == 3
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == 0
+    assert int(dw.accept_len[0]) == nacc and int(dw.bonus[0]) == bonus
+    assert dw.accepted[0, :nacc].cpu().tolist() == path
+    got = dw.attn_out.float().cpu().numpy()
+    G = cfg.hq // cfg.hkv
+    for l, kvh in ((0, 1), (17, 4), (31, 6)):
+        ref = _attn_ref(w, l, 0, heads=kvh * G)
+        _check_attn(got[l][:, kvh * G:(kvh + 1) * G], ref, "bf16", f"step l{l} kv{kvh}")
+    ka = dw.k.cpu().view(torch.int16).numpy()
+    for l in range(cfg.layers):
+        ref, new_ctx = oracle.kv_compact(w.seq_view(k_before[l], 0), path, int(w.ctx_lens[0]))
+        assert int(dw.new_ctx[0]) == new_ctx
+        assert np.array_equal(w.seq_view(ka[l], 0)[:new_ctx], ref[:new_ctx])
+
+
 def test_host_step_matches_device_step():
     """ptd_tree_verify_step_host (pinned host inputs and outputs) gives the device step's results."""
     cfg = syn.shrink(syn.CONFIGS["llama3-8b-gqa"], layers=2, ctx=(700, 700), vocab=3000)
