@@ -330,7 +330,11 @@ ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_str
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.
  * Equivalent to ptd_tree_attention, ptd_topk_draft and ptd_verify_and_compact in that
- * order on `stream` (three launches). */
+ * order on `stream` (three launches), with one difference in timing only: the top-k grid
+ * may start while the attention grid drains and read the logits then (they, like every
+ * input, must be complete when the step is enqueued, which stream order guarantees for work
+ * enqueued before it); it ends only after the attention grid, so the compaction, which
+ * overwrites cache rows the attention reads, still follows every attention read. */
 typedef struct {
   const void* q;               /* [L][N_tot][Hq][D]                                    */
   int32_t num_q_heads;
