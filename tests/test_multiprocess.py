@@ -61,6 +61,9 @@ def test_single_process_reduction_is_identity():
 
     assert bench.reduce_over_ranks(None, [1, 2.5]) == [1.0, 2.5]
     assert bench.aggregate_rate(1, 50, 20.0) == pytest.approx(2500.0)
+    # processes running the oracle at once add their rates: two at 2 s and 4 s per step
+    assert bench.oracle_rate([[2.0, 2.0], [4.0]]) == pytest.approx(0.5 + 0.25)
+    assert bench.host_cores() >= 1
 
 
 def test_reference_arm_under_torchrun_prints_once():
@@ -77,3 +80,6 @@ def test_reference_arm_under_torchrun_prints_once():
     assert len(lines) == 1
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["value"] > 0 and d["n_gpus"] == 2 and d["unit"] == "steps/s"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
+    assert d["e2e"] == {"value": d["value"], "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
