@@ -8,13 +8,17 @@ vocabulary 128256, top-4).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
-Prints one JSON line (rank 0).  `value` is whole-job steps/s with inputs resident in HBM;
-`e2e` is the same metric through ptd_tree_verify_step_host with pinned host buffers (per
-step: host->device inputs, the step, device->host results, then a stream sync).
-Every step reads ~1.13 GB (more than the 129 MB L2), so no step finds the previous one's
-data in L2.  Under torchrun each rank runs an independent replica (the step has no
+Prints one JSON line (rank 0).  `value` is whole-job steps/s with inputs resident in HBM,
+the entry points called one by one with CUDA events around every attention launch (the
+`roofline` figures come from those events); `step_call` is the same step through the
+one-call entry ptd_tree_verify_step; `e2e` is the same metric through the pipelined
+host-buffer API (ptd_pipeline_*: every step's inputs uploaded from pinned host memory and its
+results read back by the host), with the one-step host call (a stream sync per step) beside
+it.  Every step reads ~1.13 GB (more than the 129 MB L2), so no step finds the previous
+one's data in L2.  Under torchrun each rank runs an independent replica (the step has no
 cross-sequence exchange), timing is max over ranks, and value sums all ranks' steps.
-`--impl reference` times the CPU oracle on a bounded sample of the same workload.
+`cpu_baseline` and `--impl reference` time the CPU oracle on a bounded sample of the same
+workload, one process per host core.
 """
 from __future__ import annotations
 
@@ -32,12 +36,10 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOAD = "llama3-8b-gqa"
-# DRAM bytes (read + write) of one full 32-layer attention launch from an ncu capture
-# (19-layer case scaled by 32/19; traffic grows with the layer count), keyed by the
-# sha256 prefix of the kernel source it was taken on.  A changed kernel reports null.
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture of the full
-# Llama-3-8B-shaped workload (mean of two launches), keyed by the kernel source's sha256
-# prefix: a changed kernel reports null until it is captured again
+# Llama-3-8B-shaped workload (the attention: median of 20 launches of the one-pass launch
+# list), keyed by the kernel source's sha256 prefix: a changed kernel reports null until it
+# is captured again
 PROFILED_ATTENTION_TRAFFIC = {"367a999933f00987": 1161794560}
 PROFILED_LM_HEAD_TRAFFIC = {"541fa109411fd935": 1053963264}
 MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
