@@ -192,21 +192,29 @@ struct TreeVerdict {
 __device__ void verify_tree_warp(const int32_t* __restrict__ node_offsets, const int32_t* __restrict__ parents,
                                  const int32_t* __restrict__ tokens, const int32_t* __restrict__ target,
                                  int target_stride, int n_total, int max_nodes, int b, int* par_s, int* jump_s,
-                                 int* reach_s, int* depth_s, int* onpath_s, TreeVerdict* out) {
+                                 int* reach_s, int* depth_s, int* onpath_s, int* tgt_s, TreeVerdict* out) {
   const int lane = threadIdx.x & 31;
   const int node0 = node_offsets[b];
   const int T = node_offsets[b + 1] - node0;
   const bool bad_shape = T < 1 || T > max_nodes || T > kVerifyThreads || node0 < 0 || node0 + T > n_total;
   bool bad = false;
-  int par[4];
+  int par[4], tok[4];
+  // every node's parent, token and own greedy token V_i at once (no load waits on another)
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const int i = lane + 32 * q;
     par[q] = -1;
+    tok[q] = 0;
     if (!bad_shape && i < T) {
       par[q] = parents[node0 + i];
-      bad = bad || (i == 0 ? (par[q] != -1) : (par[q] < 0 || par[q] >= i));
+      tok[q] = tokens[node0 + i];
+      tgt_s[i] = target[(size_t)(node0 + i) * target_stride];
     }
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = lane + 32 * q;
+    if (!bad_shape && i < T) bad = bad || (i == 0 ? (par[q] != -1) : (par[q] < 0 || par[q] >= i));
   }
   if (__any_sync(0xffffffffu, bad) || bad_shape) {
     if (lane == 0) {
@@ -216,12 +224,13 @@ __device__ void verify_tree_warp(const int32_t* __restrict__ node_offsets, const
     }
     return;
   }
+  __syncwarp();   // tgt_s complete
   // eligible edge into node i: tokens[i] == V_{parent}
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const int i = lane + 32 * q;
     if (i < T) {
-      const int elig = i == 0 ? 1 : (tokens[node0 + i] == target[(size_t)(node0 + par[q]) * target_stride]);
+      const int elig = i == 0 ? 1 : (tok[q] == tgt_s[par[q]]);
       par_s[i] = par[q];
       jump_s[i] = i == 0 ? 0 : par[q];
       reach_s[i] = elig;
@@ -286,7 +295,7 @@ __device__ void verify_tree_warp(const int32_t* __restrict__ node_offsets, const
   }
   if (lane == 0) {
     out->len = D + 1;
-    out->bonus = target[(size_t)(node0 + cur) * target_stride];
+    out->bonus = tgt_s[cur];
     out->invalid = 0;
   }
 }
@@ -300,17 +309,17 @@ __global__ void __launch_bounds__(kCompactThreads)
                           int num_pages, const int32_t* __restrict__ block_table, int max_pages,
                           const int32_t* __restrict__ ctx_lens, int32_t* __restrict__ new_ctx) {
   __shared__ int par_s[kVerifyThreads], jump_s[kVerifyThreads], reach_s[kVerifyThreads];
-  __shared__ int depth_s[kVerifyThreads], onpath_s[kVerifyThreads];
+  __shared__ int depth_s[kVerifyThreads], onpath_s[kVerifyThreads], tgt_s[kVerifyThreads];
   __shared__ TreeVerdict verdict;
   const int layer = blockIdx.x, b = blockIdx.y;
   grid_dependency_wait();   // the targets and the cache belong to the stream's previous work
+  const int C = ctx_lens[b];   // in flight while warp 0 verifies
   if (threadIdx.x < 32)
     verify_tree_warp(node_offsets, parents, tokens, target, target_stride, n_total, max_nodes, b, par_s, jump_s,
-                     reach_s, depth_s, onpath_s, &verdict);
+                     reach_s, depth_s, onpath_s, tgt_s, &verdict);
   __syncthreads();
   int len = verdict.len;
   if (len > max_nodes) len = max_nodes;
-  const int C = ctx_lens[b];
   if (layer == 0 && blockIdx.z == 0) {
     int32_t* acc_row = accepted + (size_t)b * max_nodes;
     for (int j = threadIdx.x; j < max_nodes; j += kCompactThreads) acc_row[j] = j < len ? verdict.path[j] : -1;
