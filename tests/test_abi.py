@@ -103,3 +103,34 @@ def test_host_checks_reject_without_gpu(lib):
     assert lib.ptd_tree_attention(ctypes.byref(t), ctypes.byref(c), 0, 1, 16, 32, 0.0, 16, None, 0, 16,
                                   None) == ptd.UNSUPPORTED
     assert lib.ptd_attention_workspace_size(ctypes.byref(t), ctypes.byref(c), 32, 1) == 0
+
+
+def test_binding_rejects_host_tensors_and_bad_dtypes(lib):
+    """The Python binding checks device, layout and dtype before any call into the library:
+    there is no host fallback, a CPU tensor is an error."""
+    import torch
+    from paper_2607_10661_gb300 import ptd
+
+    logits = torch.zeros((4, 100), dtype=torch.bfloat16)
+    idx = torch.zeros((4, 2), dtype=torch.int32)
+    val = torch.zeros((4, 2), dtype=torch.float32)
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        ptd.topk_draft(logits, 2, idx, val)
+    with pytest.raises(TypeError):
+        ptd._dev([1, 2, 3], "x")
+    with pytest.raises(ValueError, match="contiguous host"):
+        ptd._host(torch.zeros((4, 4)).t(), "x")
+    with pytest.raises(TypeError):
+        ptd._host(torch.zeros(4, dtype=torch.int64), "x", torch.int32)
+    with pytest.raises(TypeError, match="unsupported dtype"):
+        ptd._ptd_dtype(torch.float16)
+
+
+def test_missing_library_fails_loudly(monkeypatch):
+    """Without the built library every entry point raises: nothing falls back to the host."""
+    from paper_2607_10661_gb300 import ptd
+
+    monkeypatch.setattr(ptd, "_lib", None)
+    monkeypatch.setattr(ptd, "LIB_PATH", os.path.join(ROOT, "no-such-dir", "libptd.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        ptd.lib()
