@@ -22,7 +22,7 @@ TOPK = ["test_topk_worked_example", "test_topk_matches_lexsort_with_ties", "test
 VERIFY = ["test_verify_worked_examples", "test_verify_brute_force_exhaustive",
           "test_verify_brute_force_seven_nodes_sampled"]
 COMPACT = ["test_compact_worked_example", "test_compact_matches_gather_and_keeps_prefix"]
-SAMPLING = ["test_sampling_one_hot_reduces_to_greedy", "test_sampling_invariants_on_random_trees",
+SAMPLING = ["test_sampling_worked_examples", "test_sampling_one_hot_reduces_to_greedy", "test_sampling_invariants_on_random_trees",
             "test_sampling_leaf_root_bonus_is_P_and_temperature", "test_sampling_star_tree_emits_P"]
 DRAFT = ["test_draft_update_worked_examples", "test_draft_update_identity_and_sliding_window",
          "test_draft_update_invariants", "test_draft_update_matches_trie_formulation"]

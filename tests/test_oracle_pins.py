@@ -351,6 +351,18 @@ def _emitted_first_token(parents, tokens, logits, u_acc, u_bon):
     return int(tokens[path[1]]) if alen > 1 else bonus
 
 
+def test_sampling_worked_examples():
+    """Hand-derived steps of Alg. 2 (tests/golden/sampling_worked.json): a rejection
+    followed by renormalisation and an acceptance, a repeated candidate, and a full
+    rejection with the bonus from the residual."""
+    for c in _load("sampling_worked.json")["cases"]:
+        logits = np.log(np.array(c["probs"], np.float64))
+        path, n, bonus, margin = oracle.verify_sampling(c["parents"], np.array(c["tokens"]), logits, 1.0,
+                                                       c["u_accept"], c["u_bonus"])
+        assert (path, n, bonus) == (c["path"], c["accept_len"], c["bonus"]), c["why"]
+        assert margin > 1e-3   # every decision is far from its threshold
+
+
 def test_sampling_star_tree_emits_P():
     """App. E: trying the candidates in order with renormalisation after each rejection,
     and falling back to the residual, emits token i with probability exactly P_i.  The
