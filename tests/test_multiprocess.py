@@ -83,3 +83,29 @@ def test_reference_arm_under_torchrun_prints_once():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_bench_algorithmic_bytes_and_flops_closed_forms():
+    """The roofline numerator of the benchmark's workload from its definition: K and V of
+    32 layers x 8 KV heads x (8192 context + 63 tree slots) x 128 x 2 B, Q read and O written
+    (32 x 63 x 32 heads x 128 x 2 B each), logits 63 x 128256 x 2 B; attention FLOPs
+    4 D Hq L per visible key, a node seeing the context and its own ancestors."""
+    import numpy as np
+
+    import bench
+    from paper_2607_10661_gb300 import synthetic as syn
+
+    w = syn.Workload(syn.CONFIGS["llama3-8b-gqa"], 1000)
+    nb = bench.step_bytes(w)
+    assert nb["kv"] == 32 * 8 * (8192 + 63) * 128 * 2 * 2
+    assert nb["qo"] == 2 * 32 * 63 * 32 * 128 * 2
+    assert nb["logits"] == 63 * 128256 * 2
+    assert nb["attention"] == 1115029504 and nb["roofline"] == nb["kv"] + nb["logits"]
+    par = w.trees[0]
+    depth = [0] * len(par)
+    for i in range(1, len(par)):
+        depth[i] = depth[par[i]] + 1
+    visible = sum(8192 + d + 1 for d in depth)
+    assert bench.attention_flops(w) == 4.0 * 128 * 32 * 32 * visible
+    assert 2.6e11 < bench.attention_flops(w) < 2.8e11   # 272.7 GFLOP per step
+    assert np.isclose(nb["attention"] / 1e6, 1115.0, atol=0.1)
