@@ -268,14 +268,22 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
   return PTD_OK;
 }
 
-static ptd_status topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab, int64_t row_stride,
-                             int32_t k, int32_t* out_idx, float* out_val, bool early, void* stream) {
-  g_last_launches = 0;
+// Host checks of ptd_topk_draft's arguments (no launch).
+static ptd_status check_topk_args(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab,
+                                  int64_t row_stride, int32_t k, const int32_t* out_idx, const float* out_val) {
   if (!logits || !out_idx || !out_val || rows < 1 || vocab < 1 || row_stride < vocab || k < 1 ||
       k > PTD_MAX_TOPK || k > vocab)
     return PTD_ERR_INVALID_ARG;
   if (dtype != PTD_BF16 && dtype != PTD_F32) return PTD_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(logits) % dtype_size(dtype)) != 0) return PTD_ERR_INVALID_ARG;
+  return PTD_OK;
+}
+
+static ptd_status topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab, int64_t row_stride,
+                             int32_t k, int32_t* out_idx, float* out_val, bool early, void* stream) {
+  g_last_launches = 0;
+  ptd_status st0 = check_topk_args(logits, dtype, rows, vocab, row_stride, k, out_idx, out_val);
+  if (st0 != PTD_OK) return st0;
   const ptd_status st = cuda_status(ptd::launch_topk(logits, dtype == PTD_BF16, rows, vocab, row_stride, k, out_idx,
                                                      out_val, nullptr, early, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
@@ -340,11 +348,12 @@ ptd_status ptd_verify_sampling(const ptd_tree* tree, const int32_t* tokens, cons
   return st;
 }
 
-ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
-                                  const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
-                                  int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
-                                  int32_t* dev_status, void* stream) {
-  g_last_launches = 0;
+// Host checks of ptd_verify_and_compact's arguments (no launch).
+static ptd_status check_verify_compact_args(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
+                                            const int32_t* target, int32_t target_stride,
+                                            const int32_t* accepted_nodes, const int32_t* accept_len,
+                                            const int32_t* bonus_token, const int32_t* new_ctx_lens,
+                                            const int32_t* dev_status) {
   ptd_status st = check_tree(tree);
   if (st != PTD_OK) return st;
   if ((st = check_cache(cache)) != PTD_OK) return st;
@@ -352,6 +361,17 @@ ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cach
       !new_ctx_lens)
     return PTD_ERR_INVALID_ARG;
   if (new_ctx_lens == tree->ctx_lens) return PTD_ERR_INVALID_ARG;   // other CTAs still read ctx_lens
+  return PTD_OK;
+}
+
+ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
+                                  const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
+                                  int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
+                                  int32_t* dev_status, void* stream) {
+  g_last_launches = 0;
+  ptd_status st = check_verify_compact_args(tree, cache, tokens, target, target_stride, accepted_nodes, accept_len,
+                                            bonus_token, new_ctx_lens, dev_status);
+  if (st != PTD_OK) return st;
   const int row_bytes = cache->num_kv_heads * cache->head_dim * (int)dtype_size(cache->dtype);
   st = cuda_status(ptd::launch_verify_compact(
       tree->node_offsets, tree->parents, tokens, target, target_stride, tree->total_nodes, tree->max_nodes,
@@ -507,10 +527,19 @@ ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_str
 
 ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a,
                                 void* stream) {
+  g_last_launches = 0;
   if (!a) return PTD_ERR_INVALID_ARG;
+  // Every host check of the three parts before the first launch, so that an error enqueues
+  // nothing (the attention call checks its own arguments before it launches).
+  ptd_status st = check_verify_compact_args(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes,
+                                            a->accept_len, a->bonus_token, a->new_ctx_lens, a->dev_status);
+  if (st != PTD_OK) return st;
+  if ((st = check_topk_args(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
+                            a->topk_val)) != PTD_OK)
+    return st;
   int total = 0;
-  ptd_status st = ptd_tree_attention(tree, cache, 0, cache ? cache->num_layers : 0, a->q, a->num_q_heads, a->scale,
-                                     a->attn_out, a->workspace, a->workspace_bytes, a->dev_status, stream);
+  st = ptd_tree_attention(tree, cache, 0, cache->num_layers, a->q, a->num_q_heads, a->scale, a->attn_out,
+                          a->workspace, a->workspace_bytes, a->dev_status, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
   // The logits are an input of the step, complete before the attention launch began: the
@@ -539,6 +568,19 @@ ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* c
       !io->tree_k_h || !io->tree_v_h || !io->topk_idx_h || !io->topk_val_h || !io->accepted_h ||
       !io->accept_len_h || !io->bonus_h || !io->new_ctx_h || !io->status_h)
     return PTD_ERR_INVALID_ARG;
+  // the checks of the step itself and of the host tree layout before the first copy, so
+  // that an error enqueues nothing
+  if (!a->q || !a->logits) return PTD_ERR_INVALID_ARG;
+  if ((st = check_verify_compact_args(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len,
+                                      a->bonus_token, a->new_ctx_lens, a->dev_status)) != PTD_OK)
+    return st;
+  if ((st = check_topk_args(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
+                            a->topk_val)) != PTD_OK)
+    return st;
+  for (int b = 0; b < tree->batch; ++b) {
+    const int T = io->node_offsets_h[b + 1] - io->node_offsets_h[b], C = io->ctx_lens_h[b];
+    if (T < 1 || C < 0 || C + T > cache->seq_capacity) return PTD_ERR_INVALID_ARG;
+  }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int B = tree->batch, N = tree->total_nodes, L = cache->num_layers;
   const size_t es = dtype_size(cache->dtype);

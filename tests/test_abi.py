@@ -134,3 +134,63 @@ def test_missing_library_fails_loudly(monkeypatch):
     monkeypatch.setattr(ptd, "LIB_PATH", os.path.join(ROOT, "no-such-dir", "libptd.so"))
     with pytest.raises(RuntimeError, match="not built"):
         ptd.lib()
+
+
+def _step_structs(ptd, **kw):
+    """A Llama-3-8B-shaped step description over fake, aligned device addresses: the host
+    checks read only the sizes and the pointers' presence and alignment."""
+    A = 1 << 20
+    t = ptd._Tree(1, 63, 63, 8192, A, A + 1024, A + 2048)
+    c = ptd._Cache(A * 2, A * 4, ptd.BF16, 32, 8, 128, 0, 8320, 0, None, 0)
+    d = dict(q=A * 8, num_q_heads=32, scale=0.0, attn_out=A * 16, logits=A * 32, logits_dtype=ptd.BF16,
+             vocab=128256, k=4, tokens=A + 4096, topk_idx=A + 8192, topk_val=A + 12288, accepted_nodes=A + 16384,
+             accept_len=A + 20480, bonus_token=A + 20544, new_ctx_lens=A + 20608, dev_status=A + 20672,
+             workspace=None, workspace_bytes=0)
+    d.update(kw)
+    return t, c, ptd._StepArgs(**d)
+
+
+def _no_cuda():
+    import torch
+
+    return not torch.cuda.is_available()
+
+
+# Host-logic checks on fake device addresses: they run only where no GPU is visible.
+host_only = pytest.mark.skipif(not _no_cuda(), reason="host-side checks with fake device addresses")
+
+
+@host_only
+@pytest.mark.parametrize("bad", [dict(k=0), dict(k=17), dict(logits=None), dict(logits_dtype=7), dict(tokens=None),
+                                 dict(new_ctx_lens=(1 << 20) + 2048), dict(dev_status=None), dict(topk_idx=None)])
+def test_step_checks_every_part_before_the_first_launch(lib, bad):
+    """ptd_tree_verify_step rejects a bad argument of its top-k or verification part before
+    it launches the attention (whose own checks would pass here): the call returns
+    INVALID_ARG, not the CUDA error that any launch attempt gives on a machine without a GPU."""
+    from paper_2607_10661_gb300 import ptd
+
+    t, c, a = _step_structs(ptd, **bad)
+    assert lib.ptd_tree_verify_step(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a), None) == ptd.INVALID_ARG
+
+
+@host_only
+def test_host_step_checks_before_the_first_copy(lib):
+    """ptd_tree_verify_step_host rejects bad step arguments and a tree that does not fit the
+    cache before it enqueues any copy (no CUDA call is reached here)."""
+    import numpy as np
+    from paper_2607_10661_gb300 import ptd
+
+    offs = np.array([0, 63], np.int32)
+    ctx = np.array([8192], np.int32)
+    fake = 1 << 24
+    io = ptd._HostIO(*([fake] * 4 + [offs.ctypes.data, ctx.ctypes.data] + [fake] * 9))
+    t, c, a = _step_structs(ptd, k=0)
+    assert lib.ptd_tree_verify_step_host(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a), ctypes.byref(io),
+                                         None) == ptd.INVALID_ARG
+    t, c, a = _step_structs(ptd, q=None)
+    assert lib.ptd_tree_verify_step_host(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a), ctypes.byref(io),
+                                         None) == ptd.INVALID_ARG
+    ctx[0] = 8300                     # 8300 + 63 slots > the cache's 8320
+    t, c, a = _step_structs(ptd)
+    assert lib.ptd_tree_verify_step_host(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a), ctypes.byref(io),
+                                         None) == ptd.INVALID_ARG
