@@ -24,6 +24,7 @@ cudaError_t launch_bounded_wait_check(int32_t* dev_status, cudaStream_t stream);
 #include "attention.cuh"
 #include "topk.cuh"
 #include "verify_compact.cuh"
+#include "step_checks.cuh"
 
 namespace {
 
@@ -631,3 +632,14 @@ ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* c
 }
 
 }  // extern "C"
+
+namespace ptd {
+ptd_status check_step_args(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a) {
+  if (!a || !a->q || !a->logits) return PTD_ERR_INVALID_ARG;
+  ptd_status st = check_verify_compact_args(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes,
+                                            a->accept_len, a->bonus_token, a->new_ctx_lens, a->dev_status);
+  if (st != PTD_OK) return st;
+  return check_topk_args(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
+                         a->topk_val);
+}
+}  // namespace ptd

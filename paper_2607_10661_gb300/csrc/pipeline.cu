@@ -21,6 +21,7 @@
 #include <new>
 
 #include "../../include/ptd.h"
+#include "step_checks.cuh"
 
 struct ptd_pipeline {
   ptd_kv_cache cache;
@@ -48,8 +49,12 @@ ptd_status ptd_pipeline_create(const ptd_kv_cache* cache, const ptd_tree* trees,
                                ptd_pipeline** out) {
   if (!cache || !trees || !args || !staging || !staging[0] || !staging[1] || !out) return PTD_ERR_INVALID_ARG;
   if (cache->page_size != 0) return PTD_ERR_UNSUPPORTED;
-  for (int s = 0; s < 2; ++s)
+  for (int s = 0; s < 2; ++s) {
     if (trees[s].batch != trees[0].batch || trees[s].total_nodes != trees[0].total_nodes) return PTD_ERR_INVALID_ARG;
+    // the step's own checks now, so that a bad argument never leaves uploads enqueued
+    const ptd_status st = ptd::check_step_args(&trees[s], cache, &args[s]);
+    if (st != PTD_OK) return st;
+  }
   const size_t need = 2ull * cache->num_layers * trees[0].total_nodes * cache->num_kv_heads * cache->head_dim *
                       elem_size(cache->dtype);
   if (staging_bytes < need) return PTD_ERR_WORKSPACE;

@@ -194,3 +194,26 @@ def test_host_step_checks_before_the_first_copy(lib):
     t, c, a = _step_structs(ptd)
     assert lib.ptd_tree_verify_step_host(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a), ctypes.byref(io),
                                          None) == ptd.INVALID_ARG
+
+
+@host_only
+@pytest.mark.parametrize("bad", [dict(k=0), dict(logits=None), dict(q=None), dict(new_ctx_lens=(1 << 20) + 2048)])
+def test_pipeline_create_checks_the_step_arguments(lib, bad):
+    """ptd_pipeline_create runs the step's checks on both slots' arguments before it creates
+    anything, so a bad argument cannot surface later with uploads already enqueued."""
+    from paper_2607_10661_gb300 import ptd
+
+    t0, c, a0 = _step_structs(ptd)
+    t1, _, a1 = _step_structs(ptd, **bad)
+    trees = (ptd._Tree * 2)(t0, t1)
+    args = (ptd._StepArgs * 2)(a0, a1)
+    staging = (ctypes.c_void_p * 2)(1 << 26, 1 << 27)
+    out = ctypes.c_void_p(0)
+    st = lib.ptd_pipeline_create(ctypes.byref(c), trees, args, staging, 1 << 40, None, ctypes.byref(out))
+    assert st == ptd.INVALID_ARG and not out.value
+    # the same description with good arguments in both slots passes the checks and gets as
+    # far as creating the pipeline's streams, which fails here only because there is no GPU
+    trees = (ptd._Tree * 2)(t0, t0)
+    args = (ptd._StepArgs * 2)(a0, a0)
+    st = lib.ptd_pipeline_create(ctypes.byref(c), trees, args, staging, 1 << 40, None, ctypes.byref(out))
+    assert st == ptd.CUDA_ERROR and not out.value
