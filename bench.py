@@ -1,31 +1,42 @@
 """Benchmark of the PTD tree-verify step on GB300.
 
 One step = the whole hot path on one batch of synthetic input: tree-masked attention over
-all 32 layers of the KV cache, per-node top-k of the logits, greedy verification and KV
-compaction, through the C ABI (libptd.so), on the Llama-3-8B-shaped GQA workload
-(32 query / 8 KV heads, head dim 128, committed context 8192, 63-node draft tree,
-vocabulary 128256, top-4).
+every layer of the KV cache, per-node top-k of the logits, greedy verification and KV
+compaction, through the C ABI (libptd.so).  The workload is one of the five seeded synthetic
+configurations (`--workload`); the default is the Llama-3-8B-shaped GQA stack (32 query / 8
+KV heads, head dim 128, 32 layers, committed context 8192, 63-node draft tree, vocabulary
+128256, top-4), the configuration the 70 % HBM target is stated for.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl reference]
 
-Prints one JSON line (rank 0).  `value` is whole-job steps/s with inputs resident in HBM,
-the entry points called one by one with CUDA events around every attention launch (the
-`roofline` figures come from those events); `step_call` is the same step through the
-one-call entry ptd_tree_verify_step; `e2e` is the same metric through the pipelined
-host-buffer API (ptd_pipeline_*: every step's inputs uploaded from pinned host memory and its
-results read back by the host), with the one-step host call (a stream sync per step) beside
-it.  Every step reads ~1.13 GB (more than the 129 MB L2), so no step finds the previous
-one's data in L2.  Under torchrun each rank runs an independent replica (the step has no
-cross-sequence exchange), timing is max over ranks, and value sums all ranks' steps.
-`cpu_baseline` and `--impl reference` time the CPU oracle on a bounded sample of the same
-workload, one process per host core.
+Prints one JSON line (rank 0).
+  value      whole-job steps/s through the one-call entry ptd_tree_verify_step, inputs
+             resident in HBM.  A timed region is K steps bracketed by a barrier, a device
+             synchronize and CUDA events; it is repeated until at least one second of wall
+             time has passed and the median region is reported.  Workloads whose step reads
+             less than four times the L2 size get the L2 flushed (a buffer twice its size
+             written) before every step, and every step is then timed on its own.
+  roofline   the attention kernel's algorithmic bytes (or FLOPs) over its mean launch time,
+             from CUDA events around every attention launch of a second, equally repeated
+             loop that calls the step's entry points one by one.
+  e2e        the same metric through the pipelined host-buffer API (ptd_pipeline_*): every
+             step's inputs uploaded from pinned host memory and its results read back.
+  clocks     SM clock and throttle reasons sampled every 10 ms through NVML, only inside
+             the timed regions.
+  cpu_baseline / --impl reference
+             the CPU oracle, whole steps (every attention unit, every top-k row, the
+             verification on this step's own greedy targets, the compaction of every layer),
+             spread over the host cores by worker processes started with spawn.
+Under torchrun each rank runs an independent replica (the step has no cross-sequence
+exchange), timing is the maximum over ranks, and value sums all ranks' steps.
 """
 from __future__ import annotations
 
 import argparse
+import ctypes
 import json
 import os
-import subprocess
+import statistics
 import sys
 import threading
 import time
@@ -35,22 +46,40 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-WORKLOAD = "llama3-8b-gqa"
-# dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture of the full
-# Llama-3-8B-shaped workload (the attention: median of 20 launches of the one-pass launch
-# list), keyed by the kernel source's sha256 prefix: a changed kernel reports null until it
-# is captured again
-PROFILED_ATTENTION_TRAFFIC = {"367a999933f00987": 1161794560}
+DEFAULT_WORKLOAD = "llama3-8b-gqa"
+METRIC = "tree-verify steps/sec (HBM GB/s and fraction of ~8 TB/s alongside)"
+# dram__bytes_read.sum + dram__bytes_write.sum per attention launch from one ncu capture,
+# keyed by (workload, the kernel source's sha256 prefix): a changed kernel reports null
+# until it is captured again
+PROFILED_ATTENTION_TRAFFIC = {}
 PROFILED_LM_HEAD_TRAFFIC = {"541fa109411fd935": 1053963264}
 MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
 NOMINAL_HBM_GBS = 8000.0
+MIN_REGION_WALL_S = 1.0
 
 
-def _workload_desc(cfg) -> str:
-    return (f"{cfg.name}: {cfg.layers} layers, {cfg.hq}q/{cfg.hkv}kv heads, head_dim {cfg.d}, "
-            f"context {cfg.ctx[0]}, draft tree {cfg.nodes[0]} nodes (branching {','.join(map(str, cfg.branching))} "
-            f"pruned), vocab {cfg.vocab}, top-{cfg.k}, batch {cfg.batch}")
+def workload_desc(cfg) -> str:
+    ctx = f"{cfg.ctx[0]}" if cfg.ctx[0] == cfg.ctx[1] else f"{cfg.ctx[0]}-{cfg.ctx[1]} (uniform, per sequence)"
+    nodes = f"{cfg.nodes[0]}" if cfg.nodes[0] == cfg.nodes[1] else f"{cfg.nodes[0]}-{cfg.nodes[1]}"
+    shape = (f"branching {','.join(map(str, cfg.branching))} pruned" if cfg.tree == "branching" else
+             "complete binary" if cfg.tree == "binary" else
+             f"random depth {cfg.depth_range[0]}-{cfg.depth_range[1]}" if cfg.tree == "random-depth" else cfg.tree)
+    cache = f", paged cache of {cfg.page_size}-token pages" if cfg.page_size else ""
+    return (f"{cfg.name}: {cfg.layers} layers, {cfg.hq}q/{cfg.hkv}kv heads, head_dim {cfg.d}, context {ctx}, "
+            f"draft tree {nodes} nodes ({shape}), vocab {cfg.vocab}, top-{cfg.k}, batch {cfg.batch}{cache}, "
+            f"{cfg.dtype}")
+
+
+def bench_config(w, extra: dict | None = None) -> dict:
+    """The `config` object of both arms' lines (the same workload, the same dict)."""
+    c = w.cfg
+    out = {"workload": workload_desc(c), "batch": c.batch, "layers": c.layers,
+           "context": [int(x) for x in w.ctx_lens], "tree_nodes": int(w.n_total), "vocab": c.vocab, "k": c.k,
+           "seed": int(w.seed)}
+    out.update(extra or {})
+    return out
 
 
 def step_bytes(w) -> dict:
@@ -78,70 +107,90 @@ def attention_flops(w) -> float:
 
 # ----------------------------------------------------------------------------- clocks
 class ClockSampler:
-    QUERY = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    """SM clock, power and throttle reasons of one GPU every `period_s`, through NVML (read
+    only).  summary(regions) keeps only the samples taken inside the given wall-clock
+    intervals and says "no samples" when none fell there."""
 
-    def __init__(self, index: int):
-        self.index = index
-        self.proc = None
-        self.lines = []
+    _REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+                0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, torch_index: int, period_s: float = 0.01):
+        self.period = period_s
+        self.samples = []
+        self.source = None
+        self._stop = threading.Event()
+        self._thread = None
+        self._nvml = None
+        self._h = None
+        try:
+            self._open(torch_index)
+        except Exception as e:  # reported in the line, never fatal
+            self.source = f"unavailable ({e})"[:120]
+
+    def _open(self, torch_index):
+        import torch
+
+        nv = ctypes.CDLL("libnvidia-ml.so.1")
+        if nv.nvmlInit_v2() != 0:
+            raise RuntimeError("nvmlInit failed")
+        h = ctypes.c_void_p()
+        props = torch.cuda.get_device_properties(torch_index)
+        found = False
+        try:
+            bus = b"%08X:%02X:%02X.0" % (props.pci_domain_id, props.pci_bus_id, props.pci_device_id)
+            found = nv.nvmlDeviceGetHandleByPciBusId_v2(ctypes.c_char_p(bus), ctypes.byref(h)) == 0
+        except AttributeError:
+            pass
+        if not found:
+            found = nv.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(torch_index), ctypes.byref(h)) == 0
+        if not found:
+            raise RuntimeError("no NVML handle")
+        self._nvml, self._h = nv, h
+        self._reasons_fn = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        mx = ctypes.c_uint()
+        nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx))
+        self.max_mhz = float(mx.value)
+        self.source = "nvml"
+
+    def _loop(self):
+        nv, h = self._nvml, self._h
+        mhz, mw, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        while not self._stop.is_set():
+            t = time.time()
+            if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(mhz)) == 0:
+                nv.nvmlDeviceGetPowerUsage(h, ctypes.byref(mw))
+                self._reasons_fn(h, ctypes.byref(rs))
+                self.samples.append((t, float(mhz.value), mw.value / 1000.0, int(rs.value)))
+            self._stop.wait(self.period)
 
     def start(self):
-        try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-            self.thread = threading.Thread(target=self._read, daemon=True)
-            self.thread.start()
-        except OSError:
-            self.proc = None
-
-    def _read(self):
-        for line in self.proc.stdout:
-            self.lines.append((time.time(), line.strip()))
+        if self._nvml is not None:
+            self._thread = threading.Thread(target=self._loop, daemon=True)
+            self._thread.start()
 
     def stop(self):
-        if self.proc is not None:
-            self.proc.terminate()
-            try:
-                self.proc.wait(timeout=5)
-            except subprocess.TimeoutExpired:
-                self.proc.kill()
+        self._stop.set()
+        if self._thread is not None:
+            self._thread.join(timeout=2)
 
-    def summary(self, t0: float, t1: float) -> dict:
-        rows = []
-        for ts, line in self.lines:
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) < 8:
-                continue
-            try:
-                rows.append((ts, float(parts[0]), float(parts[1]), parts[3:]))
-            except ValueError:
-                continue
-        inside = [r for r in rows if t0 <= r[0] <= t1] or rows
+    def summary(self, regions) -> dict:
+        inside = [s for s in self.samples if any(a <= s[0] <= b for a, b in regions)]
         if not inside:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = set()
-        for r in inside:
-            for n, v in zip(names, r[3][1:5]):
-                if v.lower() == "active":
-                    reasons.add(n)
-        return {"sm_mhz": float(np.median([r[1] for r in inside])), "sm_max_mhz": max(r[2] for r in inside),
-                "reasons": sorted(reasons), "samples": len(inside)}
+            return {"sm_mhz": None, "sm_max_mhz": getattr(self, "max_mhz", None), "reasons": ["no samples"],
+                    "samples": 0, "source": self.source}
+        reasons = sorted({name for s in inside for bit, name in self._REASONS.items() if s[3] & bit})
+        return {"sm_mhz": float(np.median([s[1] for s in inside])), "sm_max_mhz": self.max_mhz,
+                "reasons": reasons, "samples": len(inside), "power_w_max": round(max(s[2] for s in inside), 1),
+                "period_ms": self.period * 1e3, "source": self.source}
 
 
-def _profiled_traffic(table: dict, source: str):
+def _profiled_traffic(table: dict, source: str, key=None):
     import hashlib
 
     with open(os.path.join(ROOT, "paper_2607_10661_gb300", "csrc", source), "rb") as f:
-        return table.get(hashlib.sha256(f.read()).hexdigest()[:16])
-
-
-def _attention_traffic(layers: int):
-    t = _profiled_traffic(PROFILED_ATTENTION_TRAFFIC, "attention_tc.cu")
-    return None if t is None or layers != 32 else t
+        h = hashlib.sha256(f.read()).hexdigest()[:16]
+    return table.get(h if key is None else (key, h))
 
 
 def reduce_over_ranks(dist, values, device="cpu"):
@@ -162,12 +211,43 @@ def aggregate_rate(world: int, steps: int, ms: float) -> float:
     return world * steps / (ms * 1e-3)
 
 
-def _peak_hbm():
+def _peaks():
     try:
         with open(MEASURED_PEAKS) as f:
-            return float(json.load(f)["hbm_gbs"]), "measured"
+            m = json.load(f)
+        return float(m["hbm_gbs"]), float(m["bf16_tflops_sustained"]), "measured"
     except Exception:
-        return FALLBACK_HBM_GBS, "fallback"
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS_SUSTAINED, "fallback"
+
+
+class Regions:
+    """Repeats a timed region (K steps) until MIN_REGION_WALL_S of wall time has passed
+    (at least three times) and keeps every region's device time and wall interval."""
+
+    def __init__(self, dist, device):
+        self.dist, self.device = dist, device
+        self.ms, self.walls = [], []
+
+    def run(self, region, min_wall_s=MIN_REGION_WALL_S, min_reps=3):
+        import torch
+
+        t_start = time.time()
+        while len(self.ms) < min_reps or time.time() - t_start < min_wall_s:
+            if self.dist is not None:
+                self.dist.barrier()
+            torch.cuda.synchronize()
+            w0 = time.time()
+            ms = region()
+            torch.cuda.synchronize()
+            w1 = time.time()
+            if self.dist is not None:
+                self.dist.barrier()
+            self.ms.append(ms)
+            self.walls.append((w0, w1))
+        return self
+
+    def median(self):
+        return float(statistics.median(self.ms))
 
 
 # ----------------------------------------------------------------------------- GPU arm
@@ -180,64 +260,66 @@ def run_gpu(args, rank: int, world: int, dist):
 
     local = int(os.environ.get("LOCAL_RANK", "0"))
     torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
     import __graft_entry__
 
     if rank == 0 or not os.path.exists(ptd.LIB_PATH):
         __graft_entry__.build()
     if dist is not None:
         dist.barrier()
-    cfg = syn.CONFIGS[WORKLOAD]
+    cfg = syn.CONFIGS[args.workload]
     if args.layers:
         cfg = syn.shrink(cfg, layers=args.layers)
     w = syn.Workload(cfg, 1000 + rank)
-    dw = DeviceWorkload(w, device=f"cuda:{local}")
+    dw = DeviceWorkload(w, device=dev)
     stream = torch.cuda.current_stream()
     nb = step_bytes(w)
     sampling = args.verify == "sampling"
+    extras = args.lm_head or args.draft_update or args.ptd_step or sampling
+    if extras and (cfg.batch != 1 or cfg.dtype != "bf16"):
+        raise SystemExit("--lm-head / --draft-update / --ptd-step / --verify sampling time one-tree bf16 workloads")
+    l2 = int(torch.cuda.get_device_properties(local).L2_cache_size)
+    flush_mode = nb["roofline"] < 4 * l2
+    flush = torch.empty(2 * l2, dtype=torch.uint8, device=dev) if flush_mode else None
     if sampling:
         # Alg. 2 at temperature 1: the uniforms are inputs of the step, like the logits
-        gu = torch.Generator(device=f"cuda:{local}")
+        gu = torch.Generator(device=dev)
         gu.manual_seed(5000 + rank)
-        u_acc = torch.rand(w.n_total, device=f"cuda:{local}", generator=gu)
-        u_bon = torch.rand(cfg.batch, device=f"cuda:{local}", generator=gu)
+        u_acc = torch.rand(w.n_total, device=dev, generator=gu)
+        u_bon = torch.rand(cfg.batch, device=dev, generator=gu)
     if args.lm_head:
         # the LM head feeds top-k from the nodes' hidden states: W [vocab][d_model] bf16 and H
         # [N_tot][d_model] (synthetic, seeded; Llama-3-8B's head is 128256 x 4096)
         d_model = 4096
-        gh = torch.Generator(device=f"cuda:{local}")
+        gh = torch.Generator(device=dev)
         gh.manual_seed(7000 + rank)
-        lm_w = (torch.randn((cfg.vocab, d_model), generator=gh, device=f"cuda:{local}") / d_model ** 0.5).to(
-            torch.bfloat16)
-        lm_h = torch.randn((w.n_total, d_model), generator=gh, device=f"cuda:{local}").to(torch.bfloat16)
-        lm_ws = torch.empty(ptd.lm_head_workspace_size(w.n_total, cfg.vocab), dtype=torch.uint8,
-                            device=f"cuda:{local}")
+        lm_w = (torch.randn((cfg.vocab, d_model), generator=gh, device=dev) / d_model ** 0.5).to(torch.bfloat16)
+        lm_h = torch.randn((w.n_total, d_model), generator=gh, device=dev).to(torch.bfloat16)
+        lm_ws = torch.empty(ptd.lm_head_workspace_size(w.n_total, cfg.vocab), dtype=torch.uint8, device=dev)
         lm_evs = []
     if args.ptd_step:
         args.draft_update = True
         # the tree's own (unrotated) K and V of every layer, written by the rotary step into
         # the cache slots the attention reads; the candidate pool the draft tree feeds
-        gk = torch.Generator(device=f"cuda:{local}")
+        gk = torch.Generator(device=dev)
         gk.manual_seed(6000 + rank)
-        tree_k = torch.randn((cfg.layers, w.n_total, cfg.hkv, cfg.d), generator=gk,
-                             device=f"cuda:{local}").to(dw.tdtype)
+        tree_k = torch.randn((cfg.layers, w.n_total, cfg.hkv, cfg.d), generator=gk, device=dev).to(dw.tdtype)
         tree_v = torch.randn_like(tree_k)
-        pool = ptd.CandidatePool(1 << 20, device=f"cuda:{local}")
-        ret = [torch.zeros(1, dtype=torch.int32, device=f"cuda:{local}"),
-               torch.empty(ptd.MAX_TREE_NODES, dtype=torch.int32, device=f"cuda:{local}"),
-               torch.empty(ptd.MAX_TREE_NODES, dtype=torch.int32, device=f"cuda:{local}")]
+        pool = ptd.CandidatePool(1 << 20, device=dev)
+        ret = [torch.zeros(1, dtype=torch.int32, device=dev),
+               torch.empty(ptd.MAX_TREE_NODES, dtype=torch.int32, device=dev),
+               torch.empty(ptd.MAX_TREE_NODES, dtype=torch.int32, device=dev)]
         pool_step = [0]
     if args.draft_update:
         # the step's tree as a one-seed draft forest, grown by every node's top-1 (width 4,
         # depth 6: the paper's best setting); the output is the next step's draft tree
-        if cfg.batch != 1:
-            raise SystemExit("--draft-update times the one-tree workload only")
-        du_dev = f"cuda:{local}"
-        du_cnt = torch.tensor([w.n_total], dtype=torch.int32, device=du_dev)
-        du_out = [torch.empty((1,), dtype=torch.int32, device=du_dev)] + \
-                 [torch.empty((1, ptd.MAX_TREE_NODES), dtype=torch.int32, device=du_dev) for _ in range(3)] + \
-                 [torch.empty((1, w.n_total), dtype=torch.int32, device=du_dev)]
+        du_cnt = torch.tensor([w.n_total], dtype=torch.int32, device=dev)
+        du_out = [torch.empty((1,), dtype=torch.int32, device=dev)] + \
+                 [torch.empty((1, ptd.MAX_TREE_NODES), dtype=torch.int32, device=dev) for _ in range(3)] + \
+                 [torch.empty((1, w.n_total), dtype=torch.int32, device=dev)]
 
-    def one_step(ev=None):
+    def parts_step(ev=None):
+        """One step through the entry points one by one (events around the attention)."""
         n = 0
         if args.ptd_step:   # positions C + |pi(v)| - 1, rotary encoding, tree K/V into the cache
             n += ptd.tree_rope_append(dw.tree, dw.cache, 0, dw.q, cfg.hq, tree_k, tree_v, 500000.0, dw.dev_status)
@@ -272,135 +354,110 @@ def run_gpu(args, rank: int, world: int, dist):
             n += pool.retrieve(dw.bonus[:1], 4, 6, 64, *ret)
         return n
 
+    def call_step():
+        """One step through the one-call entry ptd_tree_verify_step (no events inside)."""
+        return ptd.tree_verify_step(dw.tree, dw.cache, dw.bufs, stream)
+
+    main_step = parts_step if extras else call_step
+    K = args.steps
+    launches = [0]
+
+    def region_of(step_fn, attn_evs=None):
+        """K steps; device ms of the region (the sum of per-step times when L2 is flushed)."""
+        def region():
+            launches[0] = 0
+            if not flush_mode:
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                for i in range(K):
+                    ev = None
+                    if attn_evs is not None:
+                        ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                        attn_evs.append(ev)
+                    launches[0] += step_fn(ev) if attn_evs is not None else step_fn()
+                b.record(stream)
+                torch.cuda.synchronize()
+                return a.elapsed_time(b)
+            pairs = []
+            for i in range(K):
+                flush.zero_()
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                ev = None
+                if attn_evs is not None:
+                    ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                    attn_evs.append(ev)
+                a.record(stream)
+                launches[0] += step_fn(ev) if attn_evs is not None else step_fn()
+                b.record(stream)
+                pairs.append((a, b))
+            torch.cuda.synchronize()
+            return float(sum(a.elapsed_time(b) for a, b in pairs))
+        return region
+
     dw.dev_status.zero_()              # sticky status word: cleared once, read after the run
     sampler = ClockSampler(local)
     sampler.start()
-    time.sleep(0.5)
     for _ in range(args.warmup):
-        one_step()
+        main_step()
     torch.cuda.synchronize()
     assert int(dw.dev_status.item()) == 0, ptd.status_string(int(dw.dev_status.item()))
 
-    K = args.steps
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    if dist is not None:
-        dist.barrier()
-    torch.cuda.synchronize()
-    t_wall0 = time.time()
-    start.record(stream)
-    launches = 0
-    for i in range(K):
-        launches += one_step(evs[i])
-    end.record(stream)
-    torch.cuda.synchronize()
-    t_wall1 = time.time()
-    if dist is not None:
-        dist.barrier()
-    ms = start.elapsed_time(end)
-    attn_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
-    lm_ms = float(np.mean([a.elapsed_time(b) for a, b in lm_evs])) if args.lm_head else None
-    clocks = sampler.summary(t_wall0, t_wall1)
-    sampler.stop()
+    # ---- value: the step through its public entry, K steps per region, repeated
+    main = Regions(dist, dev).run(region_of(main_step))
+    launches_per_region = launches[0]
     status = int(dw.dev_status.item())
 
-    # ---- the same step through its one-call entry (ptd_tree_verify_step), with no events
-    # between its launches: there the top-k may start while the attention grid drains
-    step_call_ms, Kc = None, max(10, K // 4)
-    if not (args.lm_head or args.draft_update or args.ptd_step or sampling):
-        for _ in range(3):
-            ptd.tree_verify_step(dw.tree, dw.cache, dw.bufs, stream)
-        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        if dist is not None:
-            dist.barrier()
-        torch.cuda.synchronize()
-        c0.record(stream)
-        for _ in range(Kc):
-            ptd.tree_verify_step(dw.tree, dw.cache, dw.bufs, stream)
-        c1.record(stream)
-        torch.cuda.synchronize()
-        step_call_ms = c0.elapsed_time(c1)
-        status |= int(dw.dev_status.item())
-
-    # ---- end to end: pinned host inputs and outputs through ptd_tree_verify_step_host
-    N, L = w.n_total, cfg.layers
-    C = int(w.ctx_lens[0])
-    pin = lambda t: t.contiguous().pin_memory()
-    io_t = dict(q_h=pin(dw.q.cpu()), logits_h=pin(dw.logits.cpu()), tokens_h=pin(dw.tokens.cpu()),
-                parents_h=pin(dw.parents.cpu()), node_offsets_h=pin(dw.node_offsets.cpu()),
-                ctx_lens_h=pin(dw.ctx_lens.cpu()),
-                tree_k_h=pin(dw.k[:, 0, C:C + N].cpu()), tree_v_h=pin(dw.v[:, 0, C:C + N].cpu()),
-                topk_idx_h=pin(torch.zeros((N, cfg.k), dtype=torch.int32)),
-                topk_val_h=pin(torch.zeros((N, cfg.k), dtype=torch.float32)),
-                accepted_h=pin(torch.zeros((cfg.batch, w.max_nodes), dtype=torch.int32)),
-                accept_len_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
-                bonus_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
-                new_ctx_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
-                status_h=pin(torch.zeros(1, dtype=torch.int32)))
-    io = ptd.HostIO(**io_t)
-    h2d = sum(io_t[n].numel() * io_t[n].element_size() for n in
-              ("q_h", "logits_h", "tokens_h", "parents_h", "node_offsets_h", "ctx_lens_h", "tree_k_h", "tree_v_h"))
-    d2h = sum(io_t[n].numel() * io_t[n].element_size() for n in
-              ("topk_idx_h", "topk_val_h", "accepted_h", "accept_len_h", "bonus_h", "new_ctx_h", "status_h"))
-    for _ in range(3):
-        ptd.tree_verify_step_host(dw.tree, dw.cache, dw.bufs, io)
-        stream.synchronize()
-    Ke = max(10, K // 5)
-    if dist is not None:
-        dist.barrier()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(Ke):
-        ptd.tree_verify_step_host(dw.tree, dw.cache, dw.bufs, io)
-        stream.synchronize()             # the host reads the step's result before the next step
-    e1.record(stream)
+    # ---- roofline: the same steps through the entry points one by one, with events around
+    # every attention launch (repeated the same way)
+    attn_evs = []
+    parts = Regions(dist, dev).run(region_of(parts_step, attn_evs))
     torch.cuda.synchronize()
-    sync_ms = e0.elapsed_time(e1)
-    sync_ok = int(io_t["status_h"][0]) == 0
-    # the same steps through the pipelined host-buffer API: step i + 1's uploads and step
-    # i - 1's downloads overlap step i's computation; the host reads every step's result
-    tree_b, bufs_b = dw.twin_step_buffers()
-    stage_n = 2 * L * N * cfg.hkv * cfg.d * dw.k.element_size()
-    staging = [torch.empty(stage_n, dtype=torch.uint8, device=f"cuda:{local}") for _ in range(2)]
-    pipe = ptd.Pipeline(dw.cache, (dw.tree, tree_b), (dw.bufs, bufs_b), staging)
-    io_t2 = {k: (pin(v.clone()) if k in ("topk_idx_h", "topk_val_h", "accepted_h", "accept_len_h", "bonus_h",
-                                         "new_ctx_h", "status_h") else v) for k, v in io_t.items()}
-    ios = [io, ptd.HostIO(**io_t2)]
-    outs_t = [io_t, io_t2]
+    attn_ms = float(np.mean([a.elapsed_time(b) for a, b in attn_evs]))
+    lm_ms = float(np.mean([a.elapsed_time(b) for a, b in lm_evs])) if args.lm_head else None
+    status |= int(dw.dev_status.item())
 
-    def run_pipeline(n):
-        ok, prev = True, None
-        for i in range(n):
-            tk = pipe.submit(ios[i & 1])
-            if prev is not None:
-                pipe.wait(prev)
-                ok = ok and int(outs_t[(i - 1) & 1]["status_h"][0]) == 0
-            prev = tk
-        pipe.wait(prev)
-        return ok and int(outs_t[(n - 1) & 1]["status_h"][0]) == 0
+    # ---- end to end: pinned host inputs and outputs through the pipelined host-buffer API
+    e2e = None
+    if not args.no_e2e and not extras:
+        e2e = run_e2e(args, dw, w, dist, dev, stream, K)
 
-    run_pipeline(4)
-    torch.cuda.synchronize()
-    if dist is not None:
-        dist.barrier()
-    e0.record(stream)
-    e2e_ok = run_pipeline(Ke) and sync_ok
-    e1.record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    pipe.close()
+    clocks = sampler.summary(main.walls + parts.walls + (e2e.pop("_walls") if e2e else []))
+    sampler.stop()
 
-    ms, e2e_ms, sync_ms, sc_ms = reduce_over_ranks(dist, [ms, e2e_ms, sync_ms, step_call_ms or 0.0],
-                                                   f"cuda:{local}")
-    step_call_ms = sc_ms if step_call_ms is not None else None
-
-    peak, peak_kind = _peak_hbm()
-    achieved = nb["attention"] / (attn_ms * 1e-3) / 1e9
-    ms_step = ms / K
-    value = aggregate_rate(world, K, ms)
+    ms_main, ms_parts = main.median(), parts.median()
+    ms_main, ms_parts, attn_ms = reduce_over_ranks(dist, [ms_main, ms_parts, attn_ms], dev)
+    hbm_peak, tf_peak, peak_kind = _peaks()
+    ms_step = ms_main / K
+    value = aggregate_rate(world, K, ms_main)
     flops = attention_flops(w)
+    achieved_gbs = nb["attention"] / (attn_ms * 1e-3) / 1e9
+    achieved_tf = flops / (attn_ms * 1e-3) / 1e12
+    tensor_bound = flops / nb["attention"] > 1e12 * tf_peak / (1e9 * hbm_peak)
+    if tensor_bound:
+        roof = {"bound": "tensor", "achieved": round(achieved_tf, 1), "peak": tf_peak, "unit": "TFLOP/s",
+                "frac": round(achieved_tf / tf_peak, 4), "peak_kind": f"{peak_kind} (bf16, sustained)",
+                "hbm_achieved_gbs": round(achieved_gbs, 1), "hbm_frac": round(achieved_gbs / hbm_peak, 4)}
+    else:
+        roof = {"bound": "hbm", "achieved": round(achieved_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                "frac": round(achieved_gbs / hbm_peak, 4), "peak_kind": peak_kind,
+                "tensor_tflops": round(achieved_tf, 1), "tensor_frac": round(achieved_tf / tf_peak, 4)}
+    kernel = "tree_attn_tc_kernel" if cfg.dtype == "bf16" else "tree_attn_simt_kernel"
+    roof.update({"kernel": kernel, "traffic": _profiled_traffic(PROFILED_ATTENTION_TRAFFIC, "attention_tc.cu",
+                                                                 (cfg.name, cfg.layers)),
+                 "bytes_per_launch": nb["attention"], "flops_per_launch": flops, "avg_launch_ms": round(attn_ms, 5),
+                 "launches_timed": len(attn_evs)})
+    l2_note = (f"L2 flushed before every step (a {2 * l2 >> 20} MB buffer written; each step timed alone)"
+               if flush_mode else "inputs larger than L2 (%.2f GB read per step vs %d MB L2)" % (
+                   nb["roofline"] / 1e9, l2 >> 20))
+    extra_cfg = {
+        "verify": "sampling (Alg. 2, temperature 1)" if sampling else "greedy",
+        "draft_update": "top-1 expansion, width 4, depth 6 (Alg. 1 step 3)" if args.draft_update else None,
+        "top_k_source": ("LM head from hidden states (logits not written)" if args.lm_head else "resident logits"),
+        "ptd_step": ("tree positions + rotary encoding + K/V append, attention, top-k, verification + compaction, "
+                     "draft update, pool merge, pool retrieval") if args.ptd_step else None,
+        "parallelism": f"replicas x{world}" if world > 1 else "single GPU", "l2": l2_note}
     out = {
-        "metric": "tree-verify steps/sec (HBM GB/s and fraction of ~8 TB/s alongside)",
+        "metric": METRIC,
         "value": round(value, 3),
         "unit": "steps/s",
         "n_gpus": world,
@@ -410,107 +467,180 @@ def run_gpu(args, rank: int, world: int, dist):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "bf16",
-        "data": "synthetic (seeded N(0,1) Q/K/V, N(0,2) logits with a planted +6 token, random pruned tree)",
-        "config": {"workload": _workload_desc(cfg), "batch": cfg.batch, "layers": cfg.layers,
-                   "context": cfg.ctx[0], "tree_nodes": w.n_total, "vocab": cfg.vocab, "k": cfg.k,
-                   "verify": "sampling (Alg. 2, temperature 1)" if sampling else "greedy",
-                   "draft_update": "top-1 expansion, width 4, depth 6 (Alg. 1 step 3)" if args.draft_update else None,
-                   "top_k_source": ("LM head from hidden states (63 x 4096 by 128256 x 4096 bf16, logits not "
-                                    "written)" if args.lm_head else "resident logits"),
-                   "ptd_step": ("tree positions + rotary encoding + K/V append (32 layers), attention, top-k, "
-                                "verification + compaction, draft update, pool merge, pool retrieval")
-                   if args.ptd_step else None,
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                   "l2": "inputs larger than L2 (%.2f GB read per step vs 129 MB L2)" % (nb["roofline"] / 1e9)},
+        "dtype": cfg.dtype,
+        "data": "synthetic (seeded N(0,1) Q/K/V, N(0,sigma) logits with a planted boosted token, random pruned trees)",
+        "config": bench_config(w, extra_cfg),
+        "api": ("entry points one by one (extra parts of the PTD step)" if extras else
+                "ptd_tree_verify_step (one call per step, device buffers)"),
+        "regions": {"count": len(main.ms), "ms_median": round(ms_main, 4), "ms_min": round(min(main.ms), 4),
+                    "ms_max": round(max(main.ms), 4)},
         "step_roofline_bytes": nb["roofline"],
         "hbm_gbs": round(nb["roofline"] / (ms_step * 1e-3) / 1e9, 1),
         "hbm_frac_of_8tbs": round(nb["roofline"] / (ms_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4),
-        "hbm_frac_of_measured": round(nb["roofline"] / (ms_step * 1e-3) / 1e9 / peak, 4),
-        "roofline": {"bound": "hbm", "kernel": "tree_attn_tc_kernel", "achieved": round(achieved, 1),
-                     "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
-                     "traffic": _attention_traffic(cfg.layers), "bytes_per_launch": nb["attention"],
-                     "avg_launch_ms": round(attn_ms, 5),
-                     "tensor_tflops": round(flops / (attn_ms * 1e-3) / 1e12, 1)},
+        "hbm_frac_of_measured": round(nb["roofline"] / (ms_step * 1e-3) / 1e9 / hbm_peak, 4),
+        "roofline": roof,
+        "parts": {"value": round(aggregate_rate(world, K, ms_parts), 3), "unit": "steps/s",
+                  "api": "ptd_tree_attention, ptd_topk_draft, ptd_verify_and_compact called one by one with CUDA "
+                         "events around every attention launch (the roofline's timing)",
+                  "regions": len(parts.ms),
+                  "step_minus_attention_us": round((ms_parts / K - attn_ms) * 1e3, 2)},
         "clocks": clocks,
-        "step_call": (None if step_call_ms is None else
-                      {"value": round(aggregate_rate(world, Kc, step_call_ms), 3), "unit": "steps/s", "steps": Kc,
-                       "api": "ptd_tree_verify_step (device buffers, no events between the launches)"}),
-        "e2e": {"value": round(aggregate_rate(world, Ke, e2e_ms), 3), "unit": "steps/s", "steps": Ke,
-                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "status_ok": e2e_ok,
-                "verify": "greedy",
-                "api": "ptd_pipeline_submit / ptd_pipeline_wait (uploads and downloads overlapped with compute, "
-                       "two steps in flight); every step's inputs uploaded from pinned host memory and its result "
-                       "read by the host",
-                "one_step_call_value": round(aggregate_rate(world, Ke, sync_ms), 3)},
+        "e2e": e2e,
         "lm_head": ({"kernel": "lm_head_topk_kernel", "avg_launch_ms": round(lm_ms, 5),
                      "bytes_per_launch": int(lm_w.numel() * 2 + lm_h.numel() * 2),
                      "achieved_gbs": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9, 1),
-                     "frac": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9
-                                   / _peak_hbm()[0], 4), "peak_kind": _peak_hbm()[1],
+                     "frac": round((lm_w.numel() * 2 + lm_h.numel() * 2) / (lm_ms * 1e-3) / 1e9 / hbm_peak, 4),
+                     "peak_kind": peak_kind,
                      "traffic": (_profiled_traffic(PROFILED_LM_HEAD_TRAFFIC, "lm_head.cu")
                                  if cfg.vocab == 128256 else None),
                      "note": "two launches: the product with per-CTA top-k, then the per-row merge"}
                     if args.lm_head else None),
-        "gpu_launches": int(launches),
+        "gpu_launches": int(launches_per_region),
         "status": ptd.status_string(status),
     }
     if rank == 0 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(args.cpu_seconds, sampling)
+        out["cpu_baseline"] = cpu_baseline(args.workload, args.cpu_seconds, w.seed)
     return out
 
 
-# ----------------------------------------------------------------------------- CPU oracle
-_SAMPLE_CODE = r"""
-import json, sys, time
-sys.path.insert(0, {root!r})
-import numpy as np
-import oracle
-from paper_2607_10661_gb300 import synthetic as syn
-cfg = syn.CONFIGS[{workload!r}]
-w = syn.Workload(cfg, 1000)
-G, C, L, H = cfg.hq // cfg.hkv, int(w.ctx_lens[0]), cfg.layers, cfg.hkv
-lg = syn.widen(w.logits, "bf16")
-cache = {{}}
-def layer(l):
-    if l not in cache:
-        cache.clear()
-        kl, vl = w.kv_layer(l)
-        cache[l] = (syn.widen(w.q_layer(l), "bf16"), w.seq_view(syn.widen(kl, "bf16"), 0),
-                    w.seq_view(syn.widen(vl, "bf16"), 0))
-    return cache[l]
-per_step = []
-deadline = time.time() + {budget}
-for i in range({warmup} + {steps}):
-    j = i * {workers} + {worker}          # this process's share of the samples
-    u = j % (L * H)
-    q, k, v = layer(u // H)
-    h = u % H
-    t0 = time.time()
-    oracle.tree_attention(q[:, h * G:(h + 1) * G], k[:, h:h + 1], v[:, h:h + 1], w.trees[0], C)
-    t1 = time.time()
-    idx, _ = oracle.topk(lg[j % w.n_total], cfg.k)
-    t2 = time.time()
-    if {sampling}:
-        g = np.random.default_rng(j)
-        path, n, bonus, _ = oracle.verify_sampling(w.trees[0], w.tokens, lg, 1.0, g.random(w.n_total), g.random())
-    else:
-        target = np.full(w.n_total, int(idx[0]), np.int64)
-        path, n, bonus = oracle.verify_greedy(w.trees[0], w.tokens, target)
-    t3 = time.time()
-    oracle.kv_compact(k if j % 2 == 0 else v, path, C)
-    t4 = time.time()
-    if i >= {warmup}:
-        per_step.append((t1 - t0) * L * H + (t2 - t1) * w.n_total + (t3 - t2) + (t4 - t3) * 2 * L)
-    if time.time() > deadline and len(per_step) > 0:
-        break
-print(json.dumps(dict(per_step=per_step)))
-"""
+def run_e2e(args, dw, w, dist, dev, stream, K):
+    """Pipelined host-buffer steps (ptd_pipeline_*), K per region, repeated; the one-step
+    host call (a synchronize per step) beside it for contiguous caches."""
+    import torch
 
-SAMPLE_DESC = ("per sample: one of the 256 (layer, KV head) attention units, one of the 63 top-k rows, the "
-               "whole verification and compaction of one of the 64 layer K/V tensors, timed in one process "
-               "(BLAS pinned to one thread) and scaled by those counts to one full step; one such process per "
-               "host core, each on its own share of the samples, all running at once")
+    from paper_2607_10661_gb300 import ptd
+
+    cfg = w.cfg
+    pin = lambda t: t.contiguous().pin_memory()
+    tk, tv = dw.tree_rows()
+    io_t = dict(q_h=pin(dw.q.cpu()), logits_h=pin(dw.logits.cpu()), tokens_h=pin(dw.tokens.cpu()),
+                parents_h=pin(dw.parents.cpu()), node_offsets_h=pin(dw.node_offsets.cpu()),
+                ctx_lens_h=pin(dw.ctx_lens.cpu()), tree_k_h=pin(tk.cpu()), tree_v_h=pin(tv.cpu()),
+                topk_idx_h=pin(torch.zeros((w.n_total, cfg.k), dtype=torch.int32)),
+                topk_val_h=pin(torch.zeros((w.n_total, cfg.k), dtype=torch.float32)),
+                accepted_h=pin(torch.zeros((cfg.batch, w.max_nodes), dtype=torch.int32)),
+                accept_len_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
+                bonus_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
+                new_ctx_h=pin(torch.zeros(cfg.batch, dtype=torch.int32)),
+                status_h=pin(torch.zeros(1, dtype=torch.int32)))
+    del tk, tv
+    outs = ("topk_idx_h", "topk_val_h", "accepted_h", "accept_len_h", "bonus_h", "new_ctx_h", "status_h")
+    h2d = sum(io_t[n].numel() * io_t[n].element_size() for n in io_t if n not in outs)
+    d2h = sum(io_t[n].numel() * io_t[n].element_size() for n in outs)
+    walls = []
+
+    one_step = None
+    if not cfg.page_size:
+        io = ptd.HostIO(**io_t)
+
+        def host_region():
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(K):
+                ptd.tree_verify_step_host(dw.tree, dw.cache, dw.bufs, io)
+                stream.synchronize()           # the host reads the step's result before the next step
+            b.record(stream)
+            torch.cuda.synchronize()
+            return a.elapsed_time(b)
+
+        for _ in range(3):
+            ptd.tree_verify_step_host(dw.tree, dw.cache, dw.bufs, io)
+            stream.synchronize()
+        r = Regions(dist, dev).run(host_region)
+        walls += r.walls
+        one_step = (r.median(), int(io_t["status_h"][0]) == 0)
+
+    tree_b, bufs_b = dw.twin_step_buffers()
+    es = dw.k.element_size()
+    staging = [torch.empty(2 * cfg.layers * w.n_total * cfg.hkv * cfg.d * es, dtype=torch.uint8, device=dev)
+               for _ in range(2)]
+    pipe = ptd.Pipeline(dw.cache, (dw.tree, tree_b), (dw.bufs, bufs_b), staging)
+    io_t2 = {k: (pin(v.clone()) if k in outs else v) for k, v in io_t.items()}
+    ios, outs_t = [ptd.HostIO(**io_t), ptd.HostIO(**io_t2)], [io_t, io_t2]
+    ok = [True]
+
+    def run_pipeline(n):
+        prev = None
+        for i in range(n):
+            tk_ = pipe.submit(ios[i & 1])
+            if prev is not None:
+                pipe.wait(prev)
+                ok[0] = ok[0] and int(outs_t[(i - 1) & 1]["status_h"][0]) == 0
+            prev = tk_
+        pipe.wait(prev)
+        ok[0] = ok[0] and int(outs_t[(n - 1) & 1]["status_h"][0]) == 0
+
+    def pipe_region():
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        run_pipeline(K)
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b)
+
+    run_pipeline(4)
+    r = Regions(dist, dev).run(pipe_region)
+    walls += r.walls
+    pipe.close()
+    world = dist.get_world_size() if dist is not None else 1
+    ms_pipe, ms_one = reduce_over_ranks(dist, [r.median(), one_step[0] if one_step else 0.0], dev)
+    return {"value": round(aggregate_rate(world, K, ms_pipe), 3), "unit": "steps/s", "steps": K,
+            "regions": len(r.ms), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "status_ok": ok[0] and (one_step is None or one_step[1]), "verify": "greedy",
+            "api": "ptd_pipeline_submit / ptd_pipeline_wait (uploads and downloads overlapped with compute, two "
+                   "steps in flight); every step's inputs uploaded from pinned host memory and its result read by "
+                   "the host",
+            "one_step_call_value": (round(aggregate_rate(world, K, ms_one), 3) if one_step else None),
+            "_walls": walls}
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+def _oracle_worker(conn, name, seed, units, rows):
+    """One host process of the oracle step: its share of the attention units (layer, tree,
+    KV head) and top-k rows, and the compaction of its units' K and V slices."""
+    import oracle
+    from paper_2607_10661_gb300 import synthetic as syn
+
+    try:
+        cfg = syn.CONFIGS[name]
+        w = syn.Workload(cfg, seed)
+        G = cfg.hq // cfg.hkv
+        data = {}
+        for l in sorted({u[0] for u in units}):
+            q = syn.widen(w.q_layer(l), cfg.dtype)
+            kc, vc = (syn.widen(x, cfg.dtype) for x in w.kv_layer(l))
+            for (ll, b, h) in units:
+                if ll == l:
+                    sl = w.nodes_of(b)
+                    data[(l, b, h)] = (np.ascontiguousarray(q[sl][:, h * G:(h + 1) * G]),
+                                       np.ascontiguousarray(w.seq_view(kc, b)[:, h:h + 1]),
+                                       np.ascontiguousarray(w.seq_view(vc, b)[:, h:h + 1]))
+            del q, kc, vc
+        lg = syn.widen(w.logits[rows[0]:rows[1]], cfg.dtype)
+        conn.send("ready")
+        keys = list(data)
+        while True:
+            msg = conn.recv()
+            if msg[0] == "stop":
+                break
+            if msg[0] == "attention":          # ("attention", m, j): the units u with u % m == j
+                m, j = msg[1], msg[2]
+                for u in keys[j::m]:
+                    q, k, v = data[u]
+                    oracle.tree_attention(q, k, v, w.trees[u[1]], int(w.ctx_lens[u[1]]))
+                conn.send(None)
+            elif msg[0] == "topk":
+                idx = np.array([oracle.topk(lg[r], cfg.k)[0] for r in range(len(lg))], np.int32).reshape(-1, cfg.k)
+                conn.send(idx)
+            elif msg[0] == "compact":          # ("compact", paths, m, j)
+                paths, m, j = msg[1], msg[2], msg[3]
+                for u in keys[j::m]:
+                    q, k, v = data[u]
+                    oracle.kv_compact(k, paths[u[1]], int(w.ctx_lens[u[1]]))
+                    oracle.kv_compact(v, paths[u[1]], int(w.ctx_lens[u[1]]))
+                conn.send(None)
+    except Exception as e:  # reported by the parent
+        conn.send(("error", repr(e)[-300:]))
 
 
 def host_cores() -> int:
@@ -520,86 +650,169 @@ def host_cores() -> int:
         return os.cpu_count() or 1
 
 
-def oracle_samples(steps: int, warmup: int, budget_s: float, sampling: bool = False, workers: int = 1):
-    """Per-process lists of per-sample full-step times (seconds): `workers` processes (fresh
-    interpreters, never forked from one that touched the GPU) run the oracle at once."""
-    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
-               CUDA_VISIBLE_DEVICES="")
-    per_worker = max(1, -(-int(steps) // workers))
-    procs = []
-    for wk in range(workers):
-        code = _SAMPLE_CODE.format(root=ROOT, workload=WORKLOAD, budget=float(budget_s), steps=per_worker,
-                                   warmup=int(warmup), sampling=bool(sampling), worker=wk, workers=workers)
-        procs.append(subprocess.Popen([sys.executable, "-c", code], stdout=subprocess.PIPE,
-                                      stderr=subprocess.PIPE, text=True, env=env))
-    out = []
-    for pr in procs:
-        so, se = pr.communicate(timeout=budget_s * 4 + 300)
-        if pr.returncode != 0:
-            raise RuntimeError(se[-500:])
-        out.append(json.loads(so.strip().splitlines()[-1])["per_step"])
-    return out
+class OracleStep:
+    """Whole oracle steps over the host cores: worker processes (started with spawn, BLAS
+    pinned to one thread each) hold contiguous shares of the attention units and top-k rows;
+    per step, every worker runs its attention units and top-k rows, the parent verifies
+    every tree on this step's greedy targets (top-k column 0), then every worker compacts
+    its units' K and V slices along the accepted paths."""
+
+    def __init__(self, name: str, seed: int, cores: int):
+        import multiprocessing as mp
+
+        from paper_2607_10661_gb300 import synthetic as syn
+
+        self.w = syn.Workload(syn.CONFIGS[name], seed)
+        c = self.w.cfg
+        units = [(l, b, h) for l in range(c.layers) for b in range(c.batch) for h in range(c.hkv)]
+        self.workers = max(1, min(cores, len(units)))
+        n = self.w.n_total
+        ctx = mp.get_context("spawn")
+        saved = {k: os.environ.get(k) for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS",
+                                                 "CUDA_VISIBLE_DEVICES")}
+        os.environ.update(OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+                          CUDA_VISIBLE_DEVICES="")
+        self.procs, self.conns = [], []
+        try:
+            for i in range(self.workers):
+                u = units[i * len(units) // self.workers:(i + 1) * len(units) // self.workers]
+                rows = (i * n // self.workers, (i + 1) * n // self.workers)
+                a, b = ctx.Pipe()
+                p = ctx.Process(target=_oracle_worker, args=(b, name, seed, u, rows), daemon=True)
+                p.start()
+                self.procs.append(p)
+                self.conns.append(a)
+        finally:
+            for k, v in saved.items():
+                if v is None:
+                    os.environ.pop(k, None)
+                else:
+                    os.environ[k] = v
+        for cn in self.conns:
+            self._recv(cn)
+
+    @staticmethod
+    def _recv(cn):
+        m = cn.recv()
+        if isinstance(m, tuple) and len(m) == 2 and m[0] == "error":
+            raise RuntimeError(m[1])
+        return m
+
+    def _round(self, msg):
+        for cn in self.conns:
+            cn.send(msg)
+        return [self._recv(cn) for cn in self.conns]
+
+    def step(self, m: int = 1, j: int = 0) -> float:
+        """One oracle step; returns its wall time in seconds.  With m > 1 only every m-th
+        attention unit (offset j) is run and compacted, and those two phases' times are
+        scaled by m: an estimate of the whole step from a 1/m sample of its units."""
+        import oracle
+
+        w = self.w
+        t0 = time.perf_counter()
+        self._round(("attention", m, j))
+        t1 = time.perf_counter()
+        idx = np.concatenate(self._round(("topk",)), axis=0)
+        target = idx[:, 0]
+        paths = []
+        for b, par in enumerate(w.trees):
+            sl = w.nodes_of(b)
+            paths.append(oracle.verify_greedy(par, w.tokens[sl], target[sl])[0])
+        t2 = time.perf_counter()
+        self._round(("compact", paths, m, j))
+        t3 = time.perf_counter()
+        return (t1 - t0) * m + (t2 - t1) + (t3 - t2) * m
+
+    def close(self):
+        for cn in self.conns:
+            try:
+                cn.send(("stop",))
+            except Exception:
+                pass
+        for p in self.procs:
+            p.join(timeout=10)
+            if p.is_alive():
+                p.kill()
 
 
-def oracle_rate(per_worker) -> float:
-    """Whole-host steps/s: the processes ran at the same time, each at 1 / (its mean step time)."""
-    return float(sum(1.0 / np.mean(p) for p in per_worker))
+SAMPLE_DESC = ("whole steps of the workload: every (layer, tree, KV head) attention unit, every top-k row, the "
+               "greedy verification of every tree on the step's own top-k column 0 and the compaction of every "
+               "layer's K and V, the units and rows split in contiguous shares over worker processes (BLAS pinned to "
+               "one thread each), timed on the wall clock per step")
 
 
-def cpu_baseline(budget_s: float, sampling: bool = False) -> dict:
-    """The oracle as it stands on a bounded sample of the workload (about budget_s of wall
-    time), on every host core, and on one core alone."""
+def cpu_baseline(name: str, budget_s: float, seed: int) -> dict:
+    """The oracle as it stands on whole steps of the workload: one warm-up step, then as many
+    steps as fit in about budget_s (at least one), over every host core."""
     cores = host_cores()
     try:
-        one = oracle_samples(10000, 1, budget_s / 2, sampling)[0]
-        many = oracle_samples(10000, 1, budget_s / 2, sampling, workers=cores)
+        st = OracleStep(name, seed, cores)
+        try:
+            st.step()
+            times, t0 = [], time.time()
+            while not times or time.time() - t0 < budget_s:
+                times.append(st.step())
+        finally:
+            st.close()
     except Exception as e:  # reported, never fatal for the GPU line
         return {"value": None, "unit": "steps/s", "cores": cores, "kind": "oracle", "error": str(e)[-300:]}
-    n = sum(len(p) for p in many)
-    return {"value": oracle_rate(many), "unit": "steps/s", "cores": cores, "kind": "oracle",
-            "sample": f"{n} samples over {cores} processes; " + SAMPLE_DESC,
-            "single_core": {"value": 1.0 / float(np.mean(one)), "unit": "steps/s", "cores": 1,
-                            "samples": len(one), "seconds_per_step": float(np.mean(one))}}
+    return {"value": len(times) / float(sum(times)), "unit": "steps/s", "cores": st.workers, "kind": "oracle",
+            "steps": len(times), "seconds_per_step": float(np.mean(times)),
+            "sample": f"{len(times)} {SAMPLE_DESC}"}
 
 
 def run_reference(args):
-    """--impl reference: the CPU oracle on the host cores, one bounded sample per step; the
-    run stops early (reporting the steps it timed) once about --ref-seconds of samples are taken."""
-    from paper_2607_10661_gb300 import synthetic as syn
-
-    cfg = syn.CONFIGS[WORKLOAD]
+    """--impl reference: the CPU oracle on the host cores, W untimed and K timed steps of the
+    same workload.  Steps are whole when K of them fit in --ref-seconds; otherwise every timed
+    step runs the attention and compaction of a 1/m sample of the units (a different sample
+    each step) with the top-k and verification whole, and those phases' times are scaled by
+    m, which the line states."""
     cores = host_cores()
     try:
-        per = oracle_samples(args.steps, min(args.warmup, 1), args.ref_seconds, args.verify == "sampling",
-                             workers=cores)
+        st = OracleStep(args.workload, 1000, cores)
     except Exception as e:
-        return {"impl": "reference", "unavailable": "oracle sample failed: " + str(e)[-200:]}
-    value = oracle_rate(per)
-    sec = 1.0 / value
-    n = sum(len(p) for p in per)
+        return {"impl": "reference", "unavailable": "oracle workers failed: " + str(e)[-200:]}
+    try:
+        warm = [st.step() for _ in range(args.warmup)]
+        per = float(np.mean(warm))
+        m = max(1, int(np.ceil(per * args.steps / args.ref_seconds)))
+        times = [st.step(m, i % m) for i in range(args.steps)]
+    finally:
+        st.close()
+    value = len(times) / float(sum(times))
+    sample = (f"{len(times)} {SAMPLE_DESC}" if m == 1 else
+              f"{len(times)} steps, each the top-k of every row and the verification of every tree whole, and the "
+              f"attention and compaction of every {m}-th (layer, tree, KV head) unit (a different 1/{m} each step) "
+              f"with those two phases' wall times multiplied by {m}; otherwise as for " + SAMPLE_DESC)
     return {
         "impl": "reference",
-        "metric": "tree-verify steps/sec (HBM GB/s and fraction of ~8 TB/s alongside)",
-        "value": value, "unit": "steps/s", "n_gpus": args.gpus, "steps": n, "warmup": min(args.warmup, 1),
-        "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "f64", "data": "synthetic", "config": {"workload": _workload_desc(cfg)},
-        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": cores, "kind": "oracle",
-                         "sample": f"{n} samples over {cores} processes; " + SAMPLE_DESC},
+        "metric": METRIC,
+        "value": value, "unit": "steps/s", "n_gpus": args.gpus, "steps": len(times), "warmup": args.warmup,
+        "ms_per_step": float(np.mean(times)) * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": bench_config(st.w, None),
+        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": st.workers, "kind": "oracle",
+                         "steps": len(times), "unit_sample_fraction": 1.0 / m, "sample": sample},
         "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
 
 def main():
+    from paper_2607_10661_gb300 import synthetic as syn
+
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ptd", choices=["ptd", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=list(syn.CONFIG_ORDER))
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling captures)")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
-    ap.add_argument("--ref-seconds", type=float, default=150.0,
-                    help="--impl reference: stop sampling the oracle after about this many seconds")
+    ap.add_argument("--ref-seconds", type=float, default=240.0,
+                    help="--impl reference: the most the K timed whole oracle steps may take")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--lm-head", action="store_true",
                     help="top-k from the LM head (ptd_lm_head_topk, logits never written) instead of from "
                          "resident logits")

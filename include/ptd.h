@@ -146,7 +146,9 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache,
  *     (ptd_attention_workspace_size > PTD_STATIC_SCRATCH_BYTES) the call returns
  *     PTD_ERR_WORKSPACE and enqueues nothing; use ptd_tree_attention with a workspace then.
  *   - The first call on each device resolves the array's device address on that device
- *     (make that device current); issue that first call before any stream capture.
+ *     (make that device current); issue that first call before any stream capture.  The
+ *     address is kept for the life of the process: a device reset (cudaDeviceReset) after
+ *     the first call is not supported.
  *   - Every call on a device shares the one array and it keeps the previous call's
  *     contents.  The kernels write every scratch entry they later read, so nothing needs
  *     clearing, but calls whose kernels overlap on the GPU (different streams without
@@ -330,11 +332,10 @@ ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_str
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.
  * Equivalent to ptd_tree_attention, ptd_topk_draft and ptd_verify_and_compact in that
- * order on `stream` (three launches), with one difference in timing only: the top-k grid
- * may start while the attention grid drains and read the logits then (they, like every
- * input, must be complete when the step is enqueued, which stream order guarantees for work
- * enqueued before it); it ends only after the attention grid, so the compaction, which
- * overwrites cache rows the attention reads, still follows every attention read. */
+ * order on `stream` (three launches).  Each launch after the first may be placed on the SMs
+ * while the one before it drains (programmatic dependent launch); it reads its inputs only
+ * after that one has completed, so every kernel sees the previous one's writes, as stream
+ * order would give. */
 typedef struct {
   const void* q;               /* [L][N_tot][Hq][D]                                    */
   int32_t num_q_heads;
@@ -368,6 +369,9 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
  *   slot ctx_lens_h[b] + (n - node_offsets_h[b])).
  * Host outputs: topk_idx_h, topk_val_h [N_tot][k]; accepted_h [B][max_nodes];
  *   accept_len_h, bonus_h, new_ctx_h [B]; status_h [1].
+ * The host tree layout is checked before anything is enqueued: node_offsets_h[0] = 0,
+ * node_offsets_h[B] = total_nodes, every tree has 1 .. max_nodes nodes and every
+ * ctx_lens_h[b] >= 0 with ctx_lens_h[b] + T_b <= seq_capacity (else PTD_ERR_INVALID_ARG).
  * Returns after enqueueing; the host outputs are valid after the stream synchronises. */
 typedef struct {
   const void* q_h;
@@ -394,16 +398,20 @@ ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* c
 /* Host-buffer steps with the copies overlapped (a software pipeline over two device buffer
  * sets): step i + 1's inputs go up, and step i - 1's results come down, while step i
  * computes.  Each submitted step is ptd_tree_verify_step_host's step (the same inputs,
- * outputs and rules; contiguous caches only), except that the tree's K/V rows first land
- * in a staging buffer and reach the cache slots from there at the start of the step's
- * computation, so that an upload never touches rows the previous step still reads.
+ * outputs and rules), except that the tree's K/V rows first land in a staging buffer and
+ * reach the cache slots from there at the start of the step's computation, so that an
+ * upload never touches rows the previous step still reads.  Contiguous and paged caches
+ * (for a paged cache the rows are scattered through the device block table by one extra
+ * kernel; a slot outside a sequence's pages sets PTD_ERR_INVALID_TREE in the status).
  *   trees[2], args[2]: two complete sets of device buffers (slot s serves steps
  *           s, s + 2, ...); they share `cache`.
  *   staging[2]: device buffers of at least 2 * L * N_tot * Hkv * D elements each.
  *   compute_stream: where the steps compute, in submission order.
  * The pipeline creates two streams and six events of its own (freed by destroy); the
  * device memory stays the caller's.  submit enqueues one step and returns its ticket; the
- * step's host outputs are valid once wait(ticket) returns.  A step's `io` buffers must
+ * step's host outputs are valid once wait(ticket) returns.  submit checks each step's host
+ * tree layout as ptd_tree_verify_step_host does and, on a bad one, returns
+ * PTD_ERR_INVALID_ARG with nothing enqueued and no ticket used.  A step's `io` buffers must
  * stay untouched until then; alternate two `io` sets to keep two steps in flight. */
 typedef struct ptd_pipeline ptd_pipeline;
 ptd_status ptd_pipeline_create(const ptd_kv_cache* cache, const ptd_tree* trees, const ptd_step_args* args,

@@ -543,11 +543,11 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
                           a->workspace, a->workspace_bytes, a->dev_status, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
-  // The logits are an input of the step, complete before the attention launch began: the
-  // top-k reads them while the attention grid drains, on the SMs its CTAs leave, and ends
-  // only after it (verification and compaction then wait on the top-k grid alone).
+  // The top-k's CTAs may be placed while the attention grid drains (programmatic dependent
+  // launch), but they read the logits only once the attention grid has completed: in a model
+  // step the logits come from the forward pass that this attention is part of.
   st = topk_draft(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
-                  a->topk_val, true, stream);
+                  a->topk_val, false, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
   st = ptd_verify_and_compact(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len,
@@ -578,10 +578,7 @@ ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* c
   if ((st = check_topk_args(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
                             a->topk_val)) != PTD_OK)
     return st;
-  for (int b = 0; b < tree->batch; ++b) {
-    const int T = io->node_offsets_h[b + 1] - io->node_offsets_h[b], C = io->ctx_lens_h[b];
-    if (T < 1 || C < 0 || C + T > cache->seq_capacity) return PTD_ERR_INVALID_ARG;
-  }
+  if ((st = ptd::check_host_tree_layout(tree, cache, io->node_offsets_h, io->ctx_lens_h)) != PTD_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int B = tree->batch, N = tree->total_nodes, L = cache->num_layers;
   const size_t es = dtype_size(cache->dtype);
@@ -603,7 +600,6 @@ ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* c
   const size_t layer_pitch = (size_t)B * cache->seq_capacity * slot_bytes;
   for (int b = 0; b < B && e == cudaSuccess; ++b) {
     const int off = io->node_offsets_h[b], T = io->node_offsets_h[b + 1] - off, C = io->ctx_lens_h[b];
-    if (T < 1 || C < 0 || C + T > cache->seq_capacity) return PTD_ERR_INVALID_ARG;
     const size_t dst_off = ((size_t)b * cache->seq_capacity + C) * slot_bytes;
     const size_t src_off = (size_t)off * slot_bytes;
     for (int kv = 0; kv < 2 && e == cudaSuccess; ++kv) {
@@ -634,6 +630,18 @@ ptd_status ptd_tree_verify_step_host(const ptd_tree* tree, const ptd_kv_cache* c
 }  // extern "C"
 
 namespace ptd {
+ptd_status check_host_tree_layout(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* node_offsets_h,
+                                  const int32_t* ctx_lens_h) {
+  if (!tree || !cache || !node_offsets_h || !ctx_lens_h) return PTD_ERR_INVALID_ARG;
+  if (node_offsets_h[0] != 0 || node_offsets_h[tree->batch] != tree->total_nodes) return PTD_ERR_INVALID_ARG;
+  for (int b = 0; b < tree->batch; ++b) {
+    const int64_t T = (int64_t)node_offsets_h[b + 1] - node_offsets_h[b], C = ctx_lens_h[b];
+    const int64_t cap = cache->page_size > 0 ? (int64_t)cache->max_pages * cache->page_size : cache->seq_capacity;
+    if (T < 1 || T > tree->max_nodes || C < 0 || C + T > cap) return PTD_ERR_INVALID_ARG;
+  }
+  return PTD_OK;
+}
+
 ptd_status check_step_args(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a) {
   if (!a || !a->q || !a->logits) return PTD_ERR_INVALID_ARG;
   ptd_status st = check_verify_compact_args(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes,

@@ -2,7 +2,8 @@
 // PTD_STATIC_SCRATCH_BYTES (declared in include/ptd.h).
 //
 // In host code the array's name only stands for the symbol; its device address is looked
-// up once per device with cudaGetSymbolAddress (with that device current) and cached.
+// up once per device with cudaGetSymbolAddress (with that device current) and cached for
+// the life of the process (a device reset, which reloads the module, is not supported).
 // Each call clears the piece counters at the front of the scratch before its kernel; the
 // partials written by one call are read back only by that same call, and each partial row
 // is written before it is read, so nothing else needs clearing.
@@ -43,6 +44,10 @@ extern "C" ptd_status ptd_tree_attention_noalloc(const ptd_tree* tree, const ptd
                                                  int32_t layer_begin, int32_t num_layers, const void* q,
                                                  int32_t num_q_heads, float scale, void* out, int32_t* dev_status,
                                                  void* stream) {
+  // the cheap argument checks first: an invalid call returns before the symbol lookup
+  if (!tree || !cache || !q || !out || !dev_status || num_q_heads < 1 || num_layers < 1 || layer_begin < 0 ||
+      layer_begin + num_layers > cache->num_layers)
+    return PTD_ERR_INVALID_ARG;
   const size_t need = ptd_attention_workspace_size(tree, cache, num_q_heads, num_layers);
   if (need > PTD_STATIC_SCRATCH_BYTES) return PTD_ERR_WORKSPACE;
   void* scratch = nullptr;

@@ -643,6 +643,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Output rows of one 32-row block from all pieces of its unit:
     // O = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c (pieces with l_c = 0 saw no key).
     // With `own`, this warp's piece is still in TMEM (O_t, m_own, l_own) rather than a partial.
+    // M is the maximum over the pieces, and both sums run over the pieces in CTA order with
+    // this warp's own piece at its CTA's place, so the result does not depend on which piece
+    // happened to finish last: every launch writes the same bits.
     auto merge = [&](const volatile SegRun* rec, bool own, float m_own, float l_own) {
       const int ug0 = rec->s.ug0, ug1 = ug0 + rec->s.n_kt;
       const int T = rec->s.T, mp = rec->s.mp;
@@ -656,24 +659,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto partial_of = [&](int c) {
         return c <= last && range_start(wc, c + 1) > range_start(wc, c) && !(own && c == wc.c);
       };
-      float M = -INFINITY, L = 0.f;
-      auto fold = [&](float2 ml) {
-        if (ml.y > 0.f) {
-          if (ml.x > M) {
-            L = L * ptx_exp2(M - ml.x) + ml.y;
-            M = ml.x;
-          } else {
-            L += ml.y * ptx_exp2(ml.x - M);
-          }
-        }
+      auto piece_ml = [&](int c) -> float2 {
+        if (own && c == wc.c) return make_float2(m_own, l_own);
+        return partial_of(c) ? __ldcg(pml + (size_t)piece_slot(wc, c, ug0, ug1) * 256) : make_float2(-INFINITY, 0.f);
       };
-      if (own) fold(make_float2(m_own, l_own));
-      for (int c = first; c <= last; c += 2) {   // two pieces' (m, l) loads at a time
-        const bool h0 = partial_of(c), h1 = partial_of(c + 1);
-        const float2 a0 = h0 ? __ldcg(pml + (size_t)piece_slot(wc, c, ug0, ug1) * 256) : make_float2(-INFINITY, 0.f);
-        const float2 a1 = h1 ? __ldcg(pml + (size_t)piece_slot(wc, c + 1, ug0, ug1) * 256) : make_float2(-INFINITY, 0.f);
-        fold(a0);
-        fold(a1);
+      float M = -INFINITY, L = 0.f;
+      for (int c = first; c <= last; ++c) {
+        const float2 ml = piece_ml(c);
+        if (ml.y > 0.f) M = fmaxf(M, ml.x);
+      }
+      for (int c = first; c <= last; ++c) {
+        const float2 ml = piece_ml(c);
+        if (ml.y > 0.f) L += ml.y * ptx_exp2(ml.x - M);
       }
       const float inv = (L > 0.f && !invalid) ? 1.f / L : 0.f;
       const float w_own = (own && l_own > 0.f) ? ptx_exp2(m_own - M) : 0.f;
@@ -682,16 +679,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
       for (int h = 0; h < 4; ++h) {   // 32 output columns at a time
         float acc[32];
-        if (own) {   // warp-uniform
-          tmem_ld32(tO + (uint32_t)h * 32u, r);
-          tmem_ld_wait();
 #pragma unroll
-          for (int d = 0; d < 32; ++d) acc[d] = w_own > 0.f ? __uint_as_float(r[d]) * w_own : 0.f;
-        } else {
-#pragma unroll
-          for (int d = 0; d < 32; ++d) acc[d] = 0.f;
-        }
+        for (int d = 0; d < 32; ++d) acc[d] = 0.f;
         for (int c = first; c <= last; ++c) {
+          if (own && c == wc.c) {   // warp-uniform: this warp's piece, from TMEM
+            tmem_ld32(tO + (uint32_t)h * 32u, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int d = 0; d < 32; ++d) acc[d] = w_own > 0.f ? fmaf(w_own, __uint_as_float(r[d]), acc[d]) : acc[d];
+            continue;
+          }
           if (!partial_of(c)) continue;
           const size_t q = (size_t)piece_slot(wc, c, ug0, ug1);
           const float2 ml = __ldcg(pml + q * 256);

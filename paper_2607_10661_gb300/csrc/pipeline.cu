@@ -8,8 +8,9 @@
 //            inputs_ready[s];
 //   compute: wait inputs_ready[s] and results_ready[s] (step i - 2's results are out of
 //            slot s's output buffers); clear the status word; copy the staged K/V rows into
-//            the cache slots C_b + i (device to device); the three-launch step; record
-//            compute_done[s];
+//            the cache slots C_b + i (device to device: one 2-D copy per tree and K/V for a
+//            contiguous cache, one scatter kernel through the block table for a paged one);
+//            the step; record compute_done[s];
 //   d2h:     wait compute_done[s]; copy the results to the step's host buffers; record
 //            results_ready[s].
 // So step i + 1's uploads run while step i computes, and step i's downloads while step
@@ -38,6 +39,35 @@ namespace {
 
 size_t elem_size(ptd_dtype d) { return d == PTD_BF16 ? 2 : 4; }
 
+// Staged tree rows into a paged cache: CTA (layer, node, K/V) copies staging row
+// [K/V][layer][node] (slot_bytes) to slot C_b + i of tree b, i = node - node_offsets[b],
+// through the block table.  A slot outside the sequence's pages is skipped and reported.
+__global__ void __launch_bounds__(128)
+    tree_rows_to_pages_kernel(const uint8_t* __restrict__ staging, uint8_t* __restrict__ k_cache,
+                              uint8_t* __restrict__ v_cache, int slot_bytes, int n_total, int batch,
+                              const int32_t* __restrict__ node_offsets, const int32_t* __restrict__ ctx_lens,
+                              const int32_t* __restrict__ block_table, int max_pages, int page_size, int num_pages,
+                              int32_t* __restrict__ dev_status) {
+  const int layer = blockIdx.x, n = blockIdx.y, kv = blockIdx.z;
+  int lo = 0, hi = batch;   // tree b with node_offsets[b] <= n < node_offsets[b + 1]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (node_offsets[mid] <= n) lo = mid; else hi = mid;
+  }
+  const int b = lo, i = n - node_offsets[b], slot = ctx_lens[b] + i;
+  const int pi = slot / page_size;
+  const int pg = (i >= 0 && slot >= 0 && pi < max_pages) ? block_table[(size_t)b * max_pages + pi] : -1;
+  if (pg < 0 || pg >= num_pages) {
+    if (threadIdx.x == 0) atomicMax(dev_status, (int)PTD_ERR_INVALID_TREE);
+    return;
+  }
+  const size_t L = gridDim.x;
+  const uint4* src = reinterpret_cast<const uint4*>(staging + (((size_t)kv * L + layer) * n_total + n) * slot_bytes);
+  uint4* dst = reinterpret_cast<uint4*>((kv ? v_cache : k_cache) +
+                                        (((size_t)layer * num_pages + pg) * page_size + slot % page_size) * slot_bytes);
+  for (int c = threadIdx.x; c < slot_bytes / 16; c += blockDim.x) dst[c] = src[c];
+}
+
 ptd_status cuda_st(cudaError_t e) { return e == cudaSuccess ? PTD_OK : PTD_ERR_CUDA; }
 
 }  // namespace
@@ -48,7 +78,8 @@ ptd_status ptd_pipeline_create(const ptd_kv_cache* cache, const ptd_tree* trees,
                                void* const* staging, size_t staging_bytes, void* compute_stream,
                                ptd_pipeline** out) {
   if (!cache || !trees || !args || !staging || !staging[0] || !staging[1] || !out) return PTD_ERR_INVALID_ARG;
-  if (cache->page_size != 0) return PTD_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(staging[0]) | reinterpret_cast<uintptr_t>(staging[1])) % 16 != 0)
+    return PTD_ERR_INVALID_ARG;
   for (int s = 0; s < 2; ++s) {
     if (trees[s].batch != trees[0].batch || trees[s].total_nodes != trees[0].total_nodes) return PTD_ERR_INVALID_ARG;
     // the step's own checks now, so that a bad argument never leaves uploads enqueued
@@ -98,10 +129,10 @@ ptd_status ptd_pipeline_submit(ptd_pipeline* p, const ptd_host_io* io, int64_t* 
   const size_t es = elem_size(cache.dtype);
   const size_t slot_bytes = (size_t)cache.num_kv_heads * cache.head_dim * es;
   const size_t kv_bytes = (size_t)L * N * slot_bytes;
-  for (int b = 0; b < B; ++b) {   // the tree rows must fit the cache (checked before anything is enqueued)
-    const int T = io->node_offsets_h[b + 1] - io->node_offsets_h[b], C = io->ctx_lens_h[b];
-    if (T < 1 || C < 0 || C + T > cache.seq_capacity) return PTD_ERR_INVALID_ARG;
-  }
+  // the host tree layout must describe this slot's tree and fit the cache (checked before
+  // anything is enqueued: the staged rows are read by these offsets)
+  const ptd_status layout = ptd::check_host_tree_layout(&tree, &cache, io->node_offsets_h, io->ctx_lens_h);
+  if (layout != PTD_OK) return layout;
   // ---- uploads
   cudaError_t e = cudaStreamWaitEvent(p->h2d, p->compute_done[s], 0);
   auto h2d = [&](const void* dst, const void* src, size_t n) {
@@ -120,8 +151,15 @@ ptd_status ptd_pipeline_submit(ptd_pipeline* p, const ptd_host_io* io, int64_t* 
   if (e == cudaSuccess) e = cudaStreamWaitEvent(p->compute, p->inputs_ready[s], 0);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(p->compute, p->results_ready[s], 0);
   if (e == cudaSuccess) e = cudaMemsetAsync(a.dev_status, 0, 4, p->compute);
+  if (cache.page_size > 0 && e == cudaSuccess) {
+    tree_rows_to_pages_kernel<<<dim3((unsigned)L, (unsigned)N, 2), 128, 0, p->compute>>>(
+        static_cast<const uint8_t*>(p->staging[s]), static_cast<uint8_t*>(cache.k), static_cast<uint8_t*>(cache.v),
+        (int)slot_bytes, N, B, tree.node_offsets, tree.ctx_lens, cache.block_table, cache.max_pages,
+        cache.page_size, cache.num_pages, a.dev_status);
+    e = cudaGetLastError();
+  }
   const size_t layer_pitch = (size_t)B * cache.seq_capacity * slot_bytes;
-  for (int b = 0; b < B && e == cudaSuccess; ++b) {
+  for (int b = 0; b < B && cache.page_size == 0 && e == cudaSuccess; ++b) {
     const int off = io->node_offsets_h[b], T = io->node_offsets_h[b + 1] - off, C = io->ctx_lens_h[b];
     const size_t dst_off = ((size_t)b * cache.seq_capacity + C) * slot_bytes;
     for (int kv = 0; kv < 2 && e == cudaSuccess; ++kv) {

@@ -97,3 +97,17 @@ class DeviceWorkload:
                                torch.zeros((c.batch,), **i32), torch.zeros((c.batch,), **i32),
                                torch.zeros(1, **i32), ws)
         return tree, bufs
+
+    def tree_rows(self):
+        """The tree's own K and V rows of every layer as they sit in the cache (slots C_b + i),
+        [L][N_tot][Hkv][D] each: the `tree_k_h` / `tree_v_h` inputs of a host-buffer step."""
+        w = self.w
+        outer, inner = [], []
+        for b in range(w.cfg.batch):
+            o, i = w.slot_rows(b)
+            C = int(w.ctx_lens[b])
+            outer.append(o[C:])
+            inner.append(i[C:])
+        o = torch.tensor(np.concatenate(outer), dtype=torch.long, device=self.device)
+        i = torch.tensor(np.concatenate(inner), dtype=torch.long, device=self.device)
+        return self.k[:, o, i].contiguous(), self.v[:, o, i].contiguous()

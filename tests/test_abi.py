@@ -217,3 +217,39 @@ def test_pipeline_create_checks_the_step_arguments(lib, bad):
     args = (ptd._StepArgs * 2)(a0, a0)
     st = lib.ptd_pipeline_create(ctypes.byref(c), trees, args, staging, 1 << 40, None, ctypes.byref(out))
     assert st == ptd.CUDA_ERROR and not out.value
+
+
+@host_only
+@pytest.mark.parametrize("offs,ctx", [([1, 63], [8192]), ([0, 62], [8192]), ([0, 64], [8192]), ([0, 63], [-1]),
+                                      ([0, 0], [8192])])
+def test_host_step_rejects_a_bad_host_tree_layout(lib, offs, ctx):
+    """A host offset array that does not describe the tree (not starting at 0, not ending at
+    total_nodes, an empty tree) or a negative context is rejected before any copy: the host
+    step would otherwise read the tree K/V rows past the host buffers."""
+    import numpy as np
+    from paper_2607_10661_gb300 import ptd
+
+    o = np.array(offs, np.int32)
+    cx = np.array(ctx, np.int32)
+    fake = 1 << 24
+    io = ptd._HostIO(*([fake] * 4 + [o.ctypes.data, cx.ctypes.data] + [fake] * 9))
+    t, c, a = _step_structs(ptd)
+    assert lib.ptd_tree_verify_step_host(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a), ctypes.byref(io),
+                                         None) == ptd.INVALID_ARG
+
+
+@host_only
+def test_host_step_rejects_a_tree_above_max_nodes(lib):
+    """Two trees whose offsets add up to total_nodes but one of which exceeds max_nodes."""
+    import numpy as np
+    from paper_2607_10661_gb300 import ptd
+
+    o = np.array([0, 40, 63], np.int32)
+    cx = np.array([100, 100], np.int32)
+    fake = 1 << 24
+    io = ptd._HostIO(*([fake] * 4 + [o.ctypes.data, cx.ctypes.data] + [fake] * 9))
+    A = 1 << 20
+    t = ptd._Tree(2, 63, 32, 100, A, A + 1024, A + 2048)           # max_nodes 32 < 40
+    _, c, a = _step_structs(ptd)
+    assert lib.ptd_tree_verify_step_host(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a), ctypes.byref(io),
+                                         None) == ptd.INVALID_ARG

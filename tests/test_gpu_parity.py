@@ -144,34 +144,70 @@ def test_attention_peaked_context_exposes_mask():
     assert np.abs(flat - ref).max() > 0.1
 
 
-def test_attention_full_size_llama3_sampled():
-    """32 layers, context 8192, 63 nodes, the launch the benchmark times; oracle on a sample
-    of (layer, KV group) pairs."""
+def _check_every_unit(w, got, what, layers=None):
+    """Oracle attention of every (layer, tree, KV head) unit of a workload, each unit checked
+    on its own (a per-unit tolerance, so that one wrong unit cannot hide in a mean over the
+    others).  `got` is the kernel's [L][N_tot][Hq][D] output."""
+    c = w.cfg
+    G = c.hq // c.hkv
+    for l in (range(c.layers) if layers is None else layers):
+        q_all = syn.widen(w.q_layer(l), c.dtype)
+        kc, vc = (syn.widen(x, c.dtype) for x in w.kv_layer(l))
+        for b in range(c.batch):
+            sl = w.nodes_of(b)
+            ref = oracle.tree_attention(q_all[sl], w.seq_view(kc, b), w.seq_view(vc, b), w.trees[b],
+                                        int(w.ctx_lens[b]))
+            for kvh in range(c.hkv):
+                hs = slice(kvh * G, (kvh + 1) * G)
+                _check_attn(got[l][sl][:, hs], ref[:, hs], c.dtype, f"{what} l{l} b{b} kv{kvh}")
+
+
+def test_attention_full_size_llama2_layer():
+    """The Llama-2-7B-shaped layer at its own size: 32 MHA heads (M = 31 rows per unit, one
+    128-row tcgen05 tile mostly padding), context 2048 (17 key tiles), every head."""
+    w = syn.Workload(syn.CONFIGS["llama2-7b-layer"], 2000)
+    assert (w.cfg.hq, w.cfg.hkv, int(w.ctx_lens[0]), w.n_total) == (32, 32, 2048, 31)
+    dw, got = _run_attention(w)
+    _check_every_unit(w, got, "llama2")
+
+
+def test_attention_full_size_llama3_every_unit():
+    """32 layers, context 8192, 63 nodes, the launch the benchmark times: all 256 (layer, KV
+    head) units against the oracle.  With 152 persistent CTAs over 256 x 65 key tiles most
+    units are cut between two CTAs and finished by the merge of their pieces."""
     w = syn.Workload(syn.CONFIGS["llama3-8b-gqa"], 1000)
     dw, got = _run_attention(w)
-    G = w.cfg.hq // w.cfg.hkv
-    for l, kvh in ((0, 0), (13, 5), (31, 7)):
-        ref = _attn_ref(w, l, 0, heads=kvh * G)
-        _check_attn(got[l][:, kvh * G:(kvh + 1) * G], ref, "bf16", f"l{l} kv{kvh}")
+    _check_every_unit(w, got, "llama3")
 
 
-def test_attention_full_size_long_context_sampled():
+def test_attention_full_size_long_context_every_head():
+    """Context 32768, 128 nodes, 64 query / 8 KV heads: every KV head (each unit spans
+    several CTAs' ranges)."""
     w = syn.Workload(syn.CONFIGS["long-context"], 5000)
     dw, got = _run_attention(w)
-    G = w.cfg.hq // w.cfg.hkv
-    for kvh in (0, 6):
-        ref = _attn_ref(w, 0, 0, heads=kvh * G)
-        _check_attn(got[0][:, kvh * G:(kvh + 1) * G], ref, "bf16", f"kv{kvh}")
+    _check_every_unit(w, got, "long")
 
 
-def test_attention_full_size_batched_paged():
+def test_attention_full_size_batched_paged_every_unit():
+    """Eight ragged sequences over a paged cache: every sequence and every KV head."""
     w = syn.Workload(syn.CONFIGS["batched-paged"], 4000)
     dw, got = _run_attention(w)
-    for b in range(w.cfg.batch):
-        ref = _attn_ref(w, 0, b, heads=(b % w.cfg.hkv) * (w.cfg.hq // w.cfg.hkv))
-        G = w.cfg.hq // w.cfg.hkv
-        kvh = b % w.cfg.hkv
-        _check_attn(got[0][w.nodes_of(b)][:, kvh * G:(kvh + 1) * G], ref, "bf16", f"b{b}")
+    _check_every_unit(w, got, "paged")
+
+
+def test_attention_is_bit_reproducible():
+    """Two launches on the same inputs write the same bits: the merge of a unit's pieces runs
+    in a fixed order whatever piece finishes last."""
+    w = syn.Workload(syn.shrink(syn.CONFIGS["long-context"], ctx=(6000, 6000), vocab=100), 17)
+    dw = DeviceWorkload(w, with_step_buffers=False)
+    outs = []
+    for _ in range(3):
+        dw.attn_out.zero_()
+        dw.attention()
+        torch.cuda.synchronize()
+        outs.append(dw.attn_out.clone())
+    assert int(dw.dev_status.item()) == 0
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
 
 
 def test_attention_invalid_tree_reports_and_zeroes():
@@ -512,10 +548,7 @@ def test_full_size_step_compaction_after_attention():
     assert int(dw.accept_len[0]) == nacc and int(dw.bonus[0]) == bonus
     assert dw.accepted[0, :nacc].cpu().tolist() == path
     got = dw.attn_out.float().cpu().numpy()
-    G = cfg.hq // cfg.hkv
-    for l, kvh in ((0, 1), (17, 4), (31, 6)):
-        ref = _attn_ref(w, l, 0, heads=kvh * G)
-        _check_attn(got[l][:, kvh * G:(kvh + 1) * G], ref, "bf16", f"step l{l} kv{kvh}")
+    _check_every_unit(w, got, "step", layers=range(0, cfg.layers, 3))
     ka = dw.k.cpu().view(torch.int16).numpy()
     for l in range(cfg.layers):
         ref, new_ctx = oracle.kv_compact(w.seq_view(k_before[l], 0), path, int(w.ctx_lens[0]))

@@ -93,3 +93,30 @@ def test_pipeline_argument_checks():
     with pytest.raises(ptd.PtdError) as e:
         ptd.Pipeline(dw_a.cache, (dw_a.tree, tree_b), (dw_a.bufs, bufs_b), small)
     assert e.value.status == ptd.WORKSPACE
+
+
+def test_pipeline_submit_rejects_a_bad_host_tree_layout():
+    """A host offset array that does not describe the slot's tree is refused with nothing
+    enqueued and no ticket used: the next good submission gets ticket 0 and the right result."""
+    w = syn.Workload(syn.shrink(syn.CONFIGS["llama3-8b-gqa"], layers=2, ctx=(200, 200), vocab=3000), 93)
+    dw_a, dw_ref = DeviceWorkload(w), DeviceWorkload(w)
+    tree_b, bufs_b = dw_a.twin_step_buffers()
+    c = w.cfg
+    n = 2 * c.layers * w.n_total * c.hkv * c.d * 2
+    staging = [torch.empty(n, dtype=torch.uint8, device="cuda") for _ in range(2)]
+    pipe = ptd.Pipeline(dw_a.cache, (dw_a.tree, tree_b), (dw_a.bufs, bufs_b), staging)
+    good = _io(w, dw_ref, 0)
+    for bad_offs in ([1, w.n_total], [0, w.n_total + 5], [0, w.n_total - 1]):
+        bad = dict(good)
+        bad["node_offsets_h"] = torch.tensor(bad_offs, dtype=torch.int32).pin_memory()
+        with pytest.raises(ptd.PtdError) as e:
+            pipe.submit(ptd.HostIO(**bad))
+        assert e.value.status == ptd.INVALID_ARG
+    ref = {k: (v.clone().pin_memory() if k in OUT else v) for k, v in good.items()}
+    ptd.tree_verify_step_host(dw_ref.tree, dw_ref.cache, dw_ref.bufs, ptd.HostIO(**ref))
+    torch.cuda.synchronize()
+    assert pipe.submit(ptd.HostIO(**good)) == 0
+    pipe.wait(0)
+    pipe.close()
+    for k in OUT:
+        assert torch.equal(good[k], ref[k]), k

@@ -61,8 +61,6 @@ def test_single_process_reduction_is_identity():
 
     assert bench.reduce_over_ranks(None, [1, 2.5]) == [1.0, 2.5]
     assert bench.aggregate_rate(1, 50, 20.0) == pytest.approx(2500.0)
-    # processes running the oracle at once add their rates: two at 2 s and 4 s per step
-    assert bench.oracle_rate([[2.0, 2.0], [4.0]]) == pytest.approx(0.5 + 0.25)
     assert bench.host_cores() >= 1
 
 
@@ -72,7 +70,7 @@ def test_reference_arm_under_torchrun_prints_once():
     port = _free_port()
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2", "--master-addr",
            "127.0.0.1", "--master-port", str(port), os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus",
-           "2", "--steps", "2", "--warmup", "1", "--ref-seconds", "5"]
+           "2", "--steps", "4", "--warmup", "3", "--workload", "tiny-fp32"]
     r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=300,
                        env=dict(os.environ, CUDA_VISIBLE_DEVICES="", OMP_NUM_THREADS="1"))
     assert r.returncode == 0, r.stderr[-2000:]
@@ -83,6 +81,50 @@ def test_reference_arm_under_torchrun_prints_once():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    # the steps and warm-up the driver asked for, whole steps, and the GPU arm's config
+    assert d["steps"] == 4 and d["warmup"] == 3 and cb["steps"] == 4 and cb["unit_sample_fraction"] == 1.0
+    assert d["ms_per_step"] == pytest.approx(1e3 / d["value"])
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2607_10661_gb300 import synthetic as syn
+
+    assert d["config"] == bench.bench_config(syn.Workload(syn.CONFIGS["tiny-fp32"], 1000), None)
+
+
+def test_oracle_step_runs_whole_and_sampled_steps():
+    """The CPU baseline's whole oracle step (worker processes started with spawn): whole steps
+    and 1/m unit samples both complete, and the sampled estimate scales the sampled phases."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    st = bench.OracleStep("tiny-fp32", 1000, 2)
+    try:
+        assert st.workers == 2                 # 8 (layer, tree, KV head) units over 2 workers
+        assert st.step() > 0
+        assert st.step(2, 1) > 0               # every 2nd unit of each share, from offset 1
+    finally:
+        st.close()
+    st = bench.OracleStep("llama2-7b-layer", 1000, 3)
+    try:
+        assert st.workers == 3
+        assert st.step() > 0 and st.step(4, 0) > 0
+    finally:
+        st.close()
+
+
+def test_clock_summary_keeps_only_samples_inside_the_regions():
+    sys.path.insert(0, ROOT)
+    import bench
+
+    cs = bench.ClockSampler.__new__(bench.ClockSampler)
+    cs.samples = [(1.0, 2070.0, 900.0, 0), (2.0, 1500.0, 1400.0, 0x4), (3.0, 1800.0, 1000.0, 0x40)]
+    cs.max_mhz, cs.source, cs.period = 2070.0, "test", 0.01
+    s = cs.summary([(1.5, 2.5)])
+    assert s["samples"] == 1 and s["sm_mhz"] == 1500.0 and s["reasons"] == ["sw_power_cap"]
+    s = cs.summary([(0.5, 1.5), (2.5, 3.5)])
+    assert s["samples"] == 2 and s["reasons"] == ["hw_thermal_slowdown"]
+    s = cs.summary([(5.0, 6.0)])
+    assert s["samples"] == 0 and s["reasons"] == ["no samples"] and s["sm_mhz"] is None
 
 
 def test_bench_algorithmic_bytes_and_flops_closed_forms():

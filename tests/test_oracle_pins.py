@@ -8,8 +8,8 @@ operand, an unsafe overlapping copy) fails at least one of them:
     the ancestor sets (chain = causal chunk, single node = plain decode, star),
     np.lexsort for top-k;
   * closed forms (identical keys -> mean of the visible values);
-  * brute force: every root path of every recursive tree with <= 6 nodes (and a
-    sample at 7 nodes) under every binary token/target assignment;
+  * brute force: every root path of every recursive tree with <= 7 nodes under
+    every binary token/target assignment;
   * invariants and metamorphic relabelling.
 """
 import itertools
@@ -276,14 +276,38 @@ def test_verify_brute_force_exhaustive(n):
                 assert oracle.verify_greedy(parents, tokens, target) == _brute_force(parents, tokens, list(target))
 
 
-def test_verify_brute_force_seven_nodes_sampled():
-    g = np.random.default_rng(7)
-    trees = list(_recursive_trees(7))
-    for parents in trees:
-        for _ in range(24):
-            tokens = [0] + g.integers(0, 2, size=6).tolist()
-            target = g.integers(0, 2, size=7).tolist()
-            assert oracle.verify_greedy(parents, tokens, target) == _brute_force(parents, tokens, target)
+def test_verify_brute_force_seven_nodes_exhaustive():
+    """Every root path of every one of the 720 recursive trees with 7 nodes, under every
+    binary token / target assignment (2^6 x 2^7 per tree, 5.9 million oracle calls): the
+    brute force is vectorised over the assignments, and the trees are spread over worker
+    processes started with spawn."""
+    import multiprocessing as mp
+
+    import _verify_brute_force as bf
+
+    trees = list(bf.recursive_trees(7))
+    assert len(trees) == 720
+    workers = max(1, min(8, os.cpu_count() or 1))
+    chunks = [trees[i::workers] for i in range(workers)]
+    with mp.get_context("spawn").Pool(workers) as pool:
+        counts = pool.map(bf.check_trees, chunks)
+    assert sum(counts) == 720 * 2 ** 6 * 2 ** 7
+
+
+def test_verify_brute_force_helper_catches_a_planted_mistake():
+    """The vectorised brute force above is itself exercised against the plain one of this
+    file on 6-node trees, and it rejects an oracle that prefers the largest sequence."""
+    import _verify_brute_force as bf
+
+    for parents in list(bf.recursive_trees(6))[::7]:
+        tokens, target, best, lengths, paths = bf.brute_force_all_assignments(parents)
+        for a in range(0, len(tokens), 97):
+            want = _brute_force(parents, tokens[a].tolist(), target[a].tolist())
+            assert (paths[int(best[a])], int(lengths[a]), int(target[a, int(best[a])])) == want
+    parents = [-1, 0, 0]
+    tokens, target, best, lengths, paths = bf.brute_force_all_assignments(parents)
+    a = [i for i in range(len(tokens)) if tokens[i].tolist() == [0, 1, 1] and target[i, 0] == 1][0]
+    assert paths[int(best[a])] == [0, 1]               # both children eligible: the smaller wins
 
 
 @pytest.mark.parametrize("name", syn.CONFIG_ORDER)
