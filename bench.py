@@ -11,14 +11,15 @@ KV heads, head dim 128, 32 layers, committed context 8192, 63-node draft tree, v
 
 Prints one JSON line (rank 0).
   value      whole-job steps/s through the one-call entry ptd_tree_verify_step, inputs
-             resident in HBM.  A timed region is K steps bracketed by a barrier, a device
-             synchronize and CUDA events; it is repeated until at least one second of wall
-             time has passed and the median region is reported.  Workloads whose step reads
-             less than four times the L2 size get the L2 flushed (a buffer twice its size
-             written) before every step, and every step is then timed on its own.
+             resident in HBM: K steps captured in a CUDA graph (so that the host's launch
+             cost is not what is timed) and replayed between CUDA events, the region repeated
+             until at least one second of wall time has passed, the median region reported.
+             Workloads whose step reads less than three times the L2 size get that many copies
+             of every buffer, used in turn, so that no step finds its inputs in L2.  `eager`
+             is the same steps called from Python one by one.
   roofline   the attention kernel's algorithmic bytes (or FLOPs) over its mean launch time,
-             from CUDA events around every attention launch of a second, equally repeated
-             loop that calls the step's entry points one by one.
+             from timing events (graph nodes) around every attention launch of a second,
+             equally repeated loop that calls the step's entry points one by one.
   e2e        the same metric through the pipelined host-buffer API (ptd_pipeline_*): every
              step's inputs uploaded from pinned host memory and its results read back.
   clocks     SM clock and throttle reasons sampled every 10 ms through NVML, only inside
@@ -251,6 +252,41 @@ class Regions:
 
 
 # ----------------------------------------------------------------------------- GPU arm
+def _external_record(ev, stream):
+    """Record a timing event as a node of the CUDA graph being captured on `stream` (a plain
+    cudaEventRecord during capture only orders streams).  Driver API, read-only on settings."""
+    r = _libcuda().cuEventRecordWithFlags(ctypes.c_void_p(ev.cuda_event), ctypes.c_void_p(stream.cuda_stream),
+                                         ctypes.c_uint(1))   # CU_EVENT_RECORD_EXTERNAL
+    if r != 0:
+        raise RuntimeError(f"cuEventRecordWithFlags failed ({r})")
+
+
+_CUDA = []
+
+
+def _libcuda():
+    if not _CUDA:
+        _CUDA.append(ctypes.CDLL("libcuda.so.1"))
+    return _CUDA[0]
+
+
+def _capture(fn):
+    """A CUDA graph of fn's launches (fn runs once eagerly on a side stream first)."""
+    import torch
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        fn()
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn()
+    torch.cuda.synchronize()
+    return g
+
+
 def run_gpu(args, rank: int, world: int, dist):
     import torch
 
@@ -272,15 +308,19 @@ def run_gpu(args, rank: int, world: int, dist):
         cfg = syn.shrink(cfg, layers=args.layers)
     w = syn.Workload(cfg, 1000 + rank)
     dw = DeviceWorkload(w, device=dev)
-    stream = torch.cuda.current_stream()
     nb = step_bytes(w)
     sampling = args.verify == "sampling"
     extras = args.lm_head or args.draft_update or args.ptd_step or sampling
     if extras and (cfg.batch != 1 or cfg.dtype != "bf16"):
         raise SystemExit("--lm-head / --draft-update / --ptd-step / --verify sampling time one-tree bf16 workloads")
     l2 = int(torch.cuda.get_device_properties(local).L2_cache_size)
-    flush_mode = nb["roofline"] < 4 * l2
-    flush = torch.empty(2 * l2, dtype=torch.uint8, device=dev) if flush_mode else None
+    # rotating copies of every buffer: consecutive steps use different copies and the copies
+    # together are at least three times the L2 size, so no step finds its inputs in L2
+    R = 1 if nb["roofline"] >= 3 * l2 or extras else min(512, -(-3 * l2 // nb["roofline"]))
+    copies = [dw] + [dw.clone() for _ in range(R - 1)]
+    K = args.steps
+    n_graphs = -(-R // K)                     # graph j runs steps j*K .. j*K + K - 1 (mod R)
+    plan = [[copies[(j * K + i) % R] for i in range(K)] for j in range(n_graphs)]
     if sampling:
         # Alg. 2 at temperature 1: the uniforms are inputs of the step, like the logits
         gu = torch.Generator(device=dev)
@@ -318,114 +358,170 @@ def run_gpu(args, rank: int, world: int, dist):
                  [torch.empty((1, ptd.MAX_TREE_NODES), dtype=torch.int32, device=dev) for _ in range(3)] + \
                  [torch.empty((1, w.n_total), dtype=torch.int32, device=dev)]
 
-    def parts_step(ev=None):
-        """One step through the entry points one by one (events around the attention)."""
+    def parts_step(d, ev=None, record=None):
+        """One step of copy d through the entry points one by one; `record(event)` around the
+        attention when timing it."""
         n = 0
         if args.ptd_step:   # positions C + |pi(v)| - 1, rotary encoding, tree K/V into the cache
-            n += ptd.tree_rope_append(dw.tree, dw.cache, 0, dw.q, cfg.hq, tree_k, tree_v, 500000.0, dw.dev_status)
+            n += ptd.tree_rope_append(d.tree, d.cache, 0, d.q, cfg.hq, tree_k, tree_v, 500000.0, d.dev_status)
         if ev is not None:
-            ev[0].record(stream)
-        n += dw.attention()
+            record(ev[0])
+        n += d.attention()
         if ev is not None:
-            ev[1].record(stream)
+            record(ev[1])
         if args.lm_head:
+            e2 = None
             if ev is not None:
                 e2 = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                e2[0].record(stream)
-            n += ptd.lm_head_topk(lm_h, lm_w, cfg.k, dw.topk_idx, dw.topk_val, lm_ws, dw.dev_status)
-            if ev is not None:
-                e2[1].record(stream)
+                e2[0].record()
+            n += ptd.lm_head_topk(lm_h, lm_w, cfg.k, d.topk_idx, d.topk_val, lm_ws, d.dev_status)
+            if e2 is not None:
+                e2[1].record()
                 lm_evs.append(e2)
         else:
-            n += dw.topk()
+            n += d.topk()
         if args.draft_update:
-            n += ptd.draft_tree_update(du_cnt, dw.parents.view(1, -1), dw.tokens.view(1, -1), dw.topk_idx, 1, 4, 6,
-                                       ptd.MAX_TREE_NODES, *du_out, dw.dev_status)
+            n += ptd.draft_tree_update(du_cnt, d.parents.view(1, -1), d.tokens.view(1, -1), d.topk_idx, 1, 4, 6,
+                                       ptd.MAX_TREE_NODES, *du_out, d.dev_status)
         if args.ptd_step:   # the grown draft tree joins the pool; C_X for the next step
             pool_step[0] += 1
-            n += pool.merge(pool_step[0], du_out[0], du_out[1][0], du_out[2][0], dw.dev_status, max_load=1 << 19)
+            n += pool.merge(pool_step[0], du_out[0], du_out[1][0], du_out[2][0], d.dev_status, max_load=1 << 19)
         if sampling:
-            n += ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, 1.0, u_acc, u_bon, dw.accepted, dw.accept_len,
-                                     dw.bonus, dw.dev_status)
-            n += dw.compact()
+            n += ptd.verify_sampling(d.tree, d.tokens, d.logits, 1.0, u_acc, u_bon, d.accepted, d.accept_len,
+                                     d.bonus, d.dev_status)
+            n += d.compact()
         else:
-            n += dw.verify_and_compact()
+            n += d.verify_and_compact()
         if args.ptd_step:
-            n += pool.retrieve(dw.bonus[:1], 4, 6, 64, *ret)
+            n += pool.retrieve(d.bonus[:1], 4, 6, 64, *ret)
         return n
 
-    def call_step():
-        """One step through the one-call entry ptd_tree_verify_step (no events inside)."""
-        return ptd.tree_verify_step(dw.tree, dw.cache, dw.bufs, stream)
+    def call_step(d):
+        """One step of copy d through the one-call entry ptd_tree_verify_step (the current stream)."""
+        return ptd.tree_verify_step(d.tree, d.cache, d.bufs)
 
-    main_step = parts_step if extras else call_step
-    K = args.steps
     launches = [0]
 
-    def region_of(step_fn, attn_evs=None):
-        """K steps; device ms of the region (the sum of per-step times when L2 is flushed)."""
-        def region():
-            launches[0] = 0
-            if not flush_mode:
-                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                a.record(stream)
-                for i in range(K):
-                    ev = None
-                    if attn_evs is not None:
-                        ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                        attn_evs.append(ev)
-                    launches[0] += step_fn(ev) if attn_evs is not None else step_fn()
-                b.record(stream)
-                torch.cuda.synchronize()
-                return a.elapsed_time(b)
-            pairs = []
-            for i in range(K):
-                flush.zero_()
-                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                ev = None
-                if attn_evs is not None:
-                    ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                    attn_evs.append(ev)
-                a.record(stream)
-                launches[0] += step_fn(ev) if attn_evs is not None else step_fn()
-                b.record(stream)
-                pairs.append((a, b))
-            torch.cuda.synchronize()
-            return float(sum(a.elapsed_time(b) for a, b in pairs))
-        return region
+    def k_steps(j, step_fn):
+        n = 0
+        for d in plan[j]:
+            n += step_fn(d)
+        launches[0] = n
+        return n
 
-    dw.dev_status.zero_()              # sticky status word: cleared once, read after the run
+    for d in copies:
+        d.dev_status.zero_()            # sticky status words: cleared once, read after the run
     sampler = ClockSampler(local)
     sampler.start()
-    for _ in range(args.warmup):
-        main_step()
+    for i in range(max(args.warmup, R)):
+        (parts_step if extras else call_step)(copies[i % R])
     torch.cuda.synchronize()
-    assert int(dw.dev_status.item()) == 0, ptd.status_string(int(dw.dev_status.item()))
+    bad = [int(d.dev_status.item()) for d in copies if int(d.dev_status.item())]
+    assert not bad, ptd.status_string(bad[0])
 
-    # ---- value: the step through its public entry, K steps per region, repeated
-    main = Regions(dist, dev).run(region_of(main_step))
-    launches_per_region = launches[0]
-    status = int(dw.dev_status.item())
+    # ---- value: K steps through the public one-call entry, captured as CUDA graphs and replayed
+    # (so that the host's launch overhead is not in the timed region), repeated, median region
+    graph_note = None
+    graphs = None
+    if not extras:
+        try:
+            graphs = [_capture(lambda j=j: k_steps(j, call_step)) for j in range(n_graphs)]
+        except Exception as e:   # reported; the eager loop then gives the value
+            graph_note = f"graph capture failed: {e}"[:200]
+            graphs = None
+    turn = [0]
 
-    # ---- roofline: the same steps through the entry points one by one, with events around
-    # every attention launch (repeated the same way)
-    attn_evs = []
-    parts = Regions(dist, dev).run(region_of(parts_step, attn_evs))
-    torch.cuda.synchronize()
-    attn_ms = float(np.mean([a.elapsed_time(b) for a, b in attn_evs]))
+    def graph_region():
+        j = turn[0] % n_graphs
+        turn[0] += 1
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        graphs[j].replay()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b)
+
+    def eager_region():
+        j = turn[0] % n_graphs
+        turn[0] += 1
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        k_steps(j, parts_step if extras else call_step)
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b)
+
+    main = Regions(dist, dev).run(graph_region if graphs is not None else eager_region)
+    launches_per_region = launches[0] if graphs is None else K * 3
+    eager = Regions(dist, dev).run(eager_region) if graphs is not None else main
+    status = 0
+    for d in copies:
+        status |= int(d.dev_status.item())
+
+    # ---- roofline: the same steps through the entry points one by one with timing events
+    # around every attention launch (graph nodes when captured), repeated the same way
+    attn_pairs = []
+    parts_graphs, parts_events = None, None
+    if not extras:
+        try:
+            parts_events = []
+            for j in range(n_graphs):
+                evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+                for e in evs:          # create the events before the capture
+                    e[0].record()
+                    e[1].record()
+                parts_events.append(evs)
+            torch.cuda.synchronize()
+
+            def parts_k(j):
+                evs = iter(parts_events[j])
+                capturing = torch.cuda.is_current_stream_capturing()
+                rec = ((lambda e: _external_record(e, torch.cuda.current_stream())) if capturing else
+                       (lambda e: e.record()))
+                for d in plan[j]:
+                    parts_step(d, next(evs), rec)
+
+            parts_graphs = [_capture(lambda j=j: parts_k(j)) for j in range(n_graphs)]
+        except Exception as e:
+            graph_note = (graph_note or "") + f" parts graph capture failed: {e}"[:200]
+            parts_graphs = None
+
+    def parts_region():
+        j = turn[0] % n_graphs
+        turn[0] += 1
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if parts_graphs is not None:
+            a.record()
+            parts_graphs[j].replay()
+            b.record()
+            torch.cuda.synchronize()
+            attn_pairs.extend(x.elapsed_time(y) for x, y in parts_events[j])
+        else:
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+            a.record()
+            for d, ev in zip(plan[j], evs):
+                parts_step(d, ev, lambda e: e.record())
+            b.record()
+            torch.cuda.synchronize()
+            attn_pairs.extend(x.elapsed_time(y) for x, y in evs)
+        return a.elapsed_time(b)
+
+    parts = Regions(dist, dev).run(parts_region)
+    attn_ms = float(np.mean(attn_pairs))
     lm_ms = float(np.mean([a.elapsed_time(b) for a, b in lm_evs])) if args.lm_head else None
-    status |= int(dw.dev_status.item())
+    for d in copies:
+        status |= int(d.dev_status.item())
 
     # ---- end to end: pinned host inputs and outputs through the pipelined host-buffer API
     e2e = None
     if not args.no_e2e and not extras:
-        e2e = run_e2e(args, dw, w, dist, dev, stream, K)
+        e2e = run_e2e(args, dw, w, dist, dev, torch.cuda.current_stream(), K)
 
     clocks = sampler.summary(main.walls + parts.walls + (e2e.pop("_walls") if e2e else []))
     sampler.stop()
 
-    ms_main, ms_parts = main.median(), parts.median()
-    ms_main, ms_parts, attn_ms = reduce_over_ranks(dist, [ms_main, ms_parts, attn_ms], dev)
+    ms_main, ms_eager, ms_parts = main.median(), eager.median(), parts.median()
+    ms_main, ms_eager, ms_parts, attn_ms = reduce_over_ranks(dist, [ms_main, ms_eager, ms_parts, attn_ms], dev)
     hbm_peak, tf_peak, peak_kind = _peaks()
     ms_step = ms_main / K
     value = aggregate_rate(world, K, ms_main)
@@ -445,10 +541,13 @@ def run_gpu(args, rank: int, world: int, dist):
     roof.update({"kernel": kernel, "traffic": _profiled_traffic(PROFILED_ATTENTION_TRAFFIC, "attention_tc.cu",
                                                                  (cfg.name, cfg.layers)),
                  "bytes_per_launch": nb["attention"], "flops_per_launch": flops, "avg_launch_ms": round(attn_ms, 5),
-                 "launches_timed": len(attn_evs)})
-    l2_note = (f"L2 flushed before every step (a {2 * l2 >> 20} MB buffer written; each step timed alone)"
-               if flush_mode else "inputs larger than L2 (%.2f GB read per step vs %d MB L2)" % (
-                   nb["roofline"] / 1e9, l2 >> 20))
+                 "launches_timed": len(attn_pairs),
+                 "timing": ("CUDA events recorded as graph nodes around every attention launch of the replayed "
+                            "parts loop" if parts_graphs is not None else
+                            "CUDA events around every attention launch of the eager parts loop")})
+    l2_note = (f"inputs larger than L2 ({nb['roofline'] / 1e9:.2f} GB read per step vs {l2 >> 20} MB L2)" if R == 1
+               else f"{R} copies of every input rotated step by step ({R * nb['roofline'] / 1e6:.0f} MB in all vs "
+                    f"{l2 >> 20} MB L2): no step finds its inputs in L2")
     extra_cfg = {
         "verify": "sampling (Alg. 2, temperature 1)" if sampling else "greedy",
         "draft_update": "top-1 expansion, width 4, depth 6 (Alg. 1 step 3)" if args.draft_update else None,
@@ -470,17 +569,21 @@ def run_gpu(args, rank: int, world: int, dist):
         "dtype": cfg.dtype,
         "data": "synthetic (seeded N(0,1) Q/K/V, N(0,sigma) logits with a planted boosted token, random pruned trees)",
         "config": bench_config(w, extra_cfg),
-        "api": ("entry points one by one (extra parts of the PTD step)" if extras else
-                "ptd_tree_verify_step (one call per step, device buffers)"),
+        "api": ("entry points one by one (extra parts of the PTD step), eager" if extras else
+                "ptd_tree_verify_step (one call per step, device buffers), K steps captured in one CUDA graph and "
+                "replayed"),
+        "graph_note": graph_note,
         "regions": {"count": len(main.ms), "ms_median": round(ms_main, 4), "ms_min": round(min(main.ms), 4),
                     "ms_max": round(max(main.ms), 4)},
+        "eager": {"value": round(aggregate_rate(world, K, ms_eager), 3), "unit": "steps/s",
+                  "api": "the same steps called from Python one by one (host launch overhead included)"},
         "step_roofline_bytes": nb["roofline"],
         "hbm_gbs": round(nb["roofline"] / (ms_step * 1e-3) / 1e9, 1),
         "hbm_frac_of_8tbs": round(nb["roofline"] / (ms_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4),
         "hbm_frac_of_measured": round(nb["roofline"] / (ms_step * 1e-3) / 1e9 / hbm_peak, 4),
         "roofline": roof,
         "parts": {"value": round(aggregate_rate(world, K, ms_parts), 3), "unit": "steps/s",
-                  "api": "ptd_tree_attention, ptd_topk_draft, ptd_verify_and_compact called one by one with CUDA "
+                  "api": "ptd_tree_attention, ptd_topk_draft, ptd_verify_and_compact called one by one with timing "
                          "events around every attention launch (the roofline's timing)",
                   "regions": len(parts.ms),
                   "step_minus_attention_us": round((ms_parts / K - attn_ms) * 1e3, 2)},

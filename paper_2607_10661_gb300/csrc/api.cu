@@ -9,6 +9,7 @@
 #include <cstddef>
 #include <cstdint>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 
 #include "../../include/ptd.h"
@@ -109,7 +110,17 @@ int persistent_ctas(int units, int n_kt, int sms) {
   return (int)(w < sms ? w : sms);
 }
 
-size_t counters_bytes(int units) { return (((size_t)units * 8 * sizeof(int32_t)) + 255) / 256 * 256; }
+size_t counters_bytes(int units) { return (((size_t)units * 8 * sizeof(unsigned long long)) + 255) / 256 * 256; }
+
+// Epoch of an attention launch: the kernel's piece counters hold (epoch << 32) | count, so a
+// counter left by another launch reads as zero and the scratch needs no clearing.  Unique
+// per launch in the process (never 0).
+uint32_t next_epoch() {
+  static std::atomic<uint32_t> epoch{0};
+  uint32_t e = epoch.fetch_add(1u) + 1u;
+  if (e == 0) e = epoch.fetch_add(1u) + 1u;
+  return e;
+}
 
 size_t persistent_workspace_bytes(int units, int ctas, int head_dim) {
   return counters_bytes(units) + (size_t)2 * ctas * 256 * ((size_t)head_dim + 2) * sizeof(float);
@@ -221,7 +232,8 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
   dim3 grid;
   if (persistent) {
     p.persistent = 1;
-    p.counters = static_cast<int32_t*>(workspace);
+    p.counters = static_cast<unsigned long long*>(workspace);
+    p.epoch = next_epoch();
     p.part_o = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + counters_bytes(units));
     p.part_ml = p.part_o + (size_t)2 * ctas * 256 * D;
     grid = dim3((unsigned)ctas, 1, 1);
@@ -262,10 +274,8 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS)
       p.q_tma = 1;
   }
-  if (persistent && cudaMemsetAsync(p.counters, 0, (size_t)units * 8 * sizeof(int32_t), s) != cudaSuccess)
-    return PTD_ERR_CUDA;
   if ((st = cuda_status(ptd::launch_tree_attn_tc(map_k, map_v, map_q, p, grid, s))) != PTD_OK) return st;
-  g_last_launches = 1;   // (the counter clear before it is a memset, not a kernel of this library)
+  g_last_launches = 1;
   return PTD_OK;
 }
 
@@ -281,19 +291,19 @@ static ptd_status check_topk_args(const void* logits, ptd_dtype dtype, int64_t r
 }
 
 static ptd_status topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab, int64_t row_stride,
-                             int32_t k, int32_t* out_idx, float* out_val, bool early, void* stream) {
+                             int32_t k, int32_t* out_idx, float* out_val, void* stream) {
   g_last_launches = 0;
   ptd_status st0 = check_topk_args(logits, dtype, rows, vocab, row_stride, k, out_idx, out_val);
   if (st0 != PTD_OK) return st0;
   const ptd_status st = cuda_status(ptd::launch_topk(logits, dtype == PTD_BF16, rows, vocab, row_stride, k, out_idx,
-                                                     out_val, nullptr, early, static_cast<cudaStream_t>(stream)));
+                                                     out_val, nullptr, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }
 
 ptd_status ptd_topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab, int64_t row_stride,
                           int32_t k, int32_t* out_idx, float* out_val, void* stream) {
-  return topk_draft(logits, dtype, rows, vocab, row_stride, k, out_idx, out_val, false, stream);
+  return topk_draft(logits, dtype, rows, vocab, row_stride, k, out_idx, out_val, stream);
 }
 
 ptd_status ptd_verify_greedy(const ptd_tree* tree, const int32_t* tokens, const int32_t* target,
@@ -365,10 +375,10 @@ static ptd_status check_verify_compact_args(const ptd_tree* tree, const ptd_kv_c
   return PTD_OK;
 }
 
-ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
-                                  const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
-                                  int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
-                                  int32_t* dev_status, void* stream) {
+static ptd_status verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
+                                     const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
+                                     int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
+                                     int32_t* dev_status, bool early_inputs, void* stream) {
   g_last_launches = 0;
   ptd_status st = check_verify_compact_args(tree, cache, tokens, target, target_stride, accepted_nodes, accept_len,
                                             bonus_token, new_ctx_lens, dev_status);
@@ -378,9 +388,17 @@ ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cach
       tree->node_offsets, tree->parents, tokens, target, target_stride, tree->total_nodes, tree->max_nodes,
       accepted_nodes, accept_len, bonus_token, dev_status, cache->k, cache->v, row_bytes, cache->num_layers,
       tree->batch, cache->page_size, cache->seq_capacity, cache->num_pages, cache->block_table, cache->max_pages,
-      tree->ctx_lens, new_ctx_lens, static_cast<cudaStream_t>(stream)));
+      tree->ctx_lens, new_ctx_lens, early_inputs, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
+}
+
+ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
+                                  const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
+                                  int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
+                                  int32_t* dev_status, void* stream) {
+  return verify_and_compact(tree, cache, tokens, target, target_stride, accepted_nodes, accept_len, bonus_token,
+                            new_ctx_lens, dev_status, false, stream);
 }
 
 ptd_status ptd_draft_tree_update(int32_t batch, int32_t in_stride, const int32_t* in_count, const int32_t* in_parents,
@@ -547,11 +565,13 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
   // launch), but they read the logits only once the attention grid has completed: in a model
   // step the logits come from the forward pass that this attention is part of.
   st = topk_draft(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
-                  a->topk_val, false, stream);
+                  a->topk_val, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
-  st = ptd_verify_and_compact(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len,
-                              a->bonus_token, a->new_ctx_lens, a->dev_status, stream);
+  // the tree arrays and context lengths are inputs of the step, complete before its
+  // attention (a plain launch) began: the verification reads them before its wait
+  st = verify_and_compact(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len,
+                          a->bonus_token, a->new_ctx_lens, a->dev_status, true, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
   g_last_launches = total;

@@ -14,7 +14,9 @@ struct AttnParams {
   void* out;                   // [layers][n_total][hq][D]
   float* part_o;               // piece partials: [slot][M tile][D][128 rows] fp32 (O unnormalised)
   float* part_ml;              // [slot][256 rows][2] (running max in log2 units, row sum)
-  int32_t* counters;           // persistent schedule: pieces finished per (unit, 32-row block)
+  unsigned long long* counters;   // persistent schedule: pieces finished per (unit, 32-row block):
+                                  // (epoch << 32) | count, a value of another epoch counting as 0
+  uint32_t epoch;                 // this launch's epoch (never 0)
   const int32_t* node_offsets;
   const int32_t* parents;
   const int32_t* ctx_lens;
@@ -34,6 +36,9 @@ struct AttnParams {
 };
 
 size_t tc_smem_bytes();
+// Launched with programmatic stream serialization: the kernel's set-up (barriers, tensor
+// memory, descriptor prefetch) may overlap the stream's previous grid; it waits for that grid
+// before its first global access.
 cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const CUtensorMap& map_q,
                                 const AttnParams& p, dim3 grid, cudaStream_t stream);
 cudaError_t launch_tree_attn_simt(const AttnParams& p, cudaStream_t stream);

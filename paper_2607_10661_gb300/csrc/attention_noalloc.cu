@@ -4,9 +4,9 @@
 // In host code the array's name only stands for the symbol; its device address is looked
 // up once per device with cudaGetSymbolAddress (with that device current) and cached for
 // the life of the process (a device reset, which reloads the module, is not supported).
-// Each call clears the piece counters at the front of the scratch before its kernel; the
-// partials written by one call are read back only by that same call, and each partial row
-// is written before it is read, so nothing else needs clearing.
+// The piece counters at the front of the scratch carry the launch's epoch, so a value left by
+// an earlier call counts as zero; the partials written by one call are read back only by that
+// same call, and each partial row is written before it is read, so nothing needs clearing.
 #include <cuda_runtime.h>
 
 #include <cstdint>

@@ -114,7 +114,15 @@ struct WarpArea {
   int tree_invalid;            // that tree failed the parent check
   int mask_mp;                 // M-tile pair the ancestor masks in registers were built for
 };
-constexpr uint32_t kSmemUsed = kOffWarp + 8 * sizeof(WarpArea);
+// Geometry of every tree of the call, read from global memory once per CTA at the start (the
+// schedule walkers decode it at every segment boundary); calls with more trees read it from
+// global memory each time instead.
+struct TreeInfo {
+  int node0, T, C, n_kt, pairs, wb;
+};
+constexpr int kMaxCachedTrees = 256;
+constexpr uint32_t kOffTrees = kOffWarp + 8 * sizeof(WarpArea);
+constexpr uint32_t kSmemUsed = kOffTrees + kMaxCachedTrees * sizeof(TreeInfo);
 constexpr uint32_t kSmemBytes = kSmemUsed + 1024;   // slack to align the base to 1024 B
 static_assert(kSmemBytes <= 232448, "shared memory budget");
 
@@ -124,9 +132,19 @@ struct WalkConst {
 };
 
 // Tree b: first node, size, context, key tiles and M-tile pairs; returns the key tiles of all
-// its units in one layer (0 for a malformed entry, which is skipped and reported).
-__device__ __forceinline__ int seq_info(const AttnParams& p, int b, int& node0, int& T, int& C, int& n_kt,
-                                        int& pairs) {
+// its units in one layer (0 for a malformed entry, which is skipped and reported).  From the
+// CTA's shared copy `ti` when there is one.
+__device__ __forceinline__ int seq_info(const AttnParams& p, const TreeInfo* ti, int b, int& node0, int& T, int& C,
+                                        int& n_kt, int& pairs) {
+  if (ti != nullptr) {
+    const TreeInfo x = ti[b];
+    node0 = x.node0;
+    T = x.T;
+    C = x.C;
+    n_kt = x.n_kt;
+    pairs = x.pairs;
+    return x.wb;
+  }
   node0 = p.node_offsets[b];
   T = p.node_offsets[b + 1] - node0;
   C = p.ctx_lens[b];
@@ -162,12 +180,12 @@ __device__ __forceinline__ int owner_cta(const WalkConst& wc, int g) {
 }
 
 // Returns false (schedule inconsistent with the tree arrays) if g maps to no tree.
-__device__ __noinline__ bool decode_tile(const AttnParams& p, int Wl, int g, Seg& s) {
+__device__ __noinline__ bool decode_tile(const AttnParams& p, const TreeInfo* ti, int Wl, int g, Seg& s) {
   s.lq = g / Wl;
   int r = g - s.lq * Wl;
   for (int b = 0; b < p.batch; ++b) {
     int node0, T, C, n_kt, pairs;
-    const int wb = seq_info(p, b, node0, T, C, n_kt, pairs);
+    const int wb = seq_info(p, ti, b, node0, T, C, n_kt, pairs);
     if (r < wb) {
       const int idx = r / n_kt;
       const int tile = r - idx * n_kt;
@@ -182,13 +200,13 @@ __device__ __noinline__ bool decode_tile(const AttnParams& p, int Wl, int g, Seg
   return false;
 }
 
-__device__ __noinline__ void make_walk_const(const AttnParams& p, WalkConst& wc) {
+__device__ __noinline__ void make_walk_const(const AttnParams& p, const TreeInfo* ti, WalkConst& wc) {
   wc.persistent = p.persistent;
   if (!p.persistent) return;
   int wl = 0;
   for (int b = 0; b < p.batch; ++b) {
     int node0, T, C, n_kt, pairs;
-    const int w = seq_info(p, b, node0, T, C, n_kt, pairs);
+    const int w = seq_info(p, ti, b, node0, T, C, n_kt, pairs);
     if (w == 0 && blockIdx.x == 0) atomicMax(p.dev_status, (int)PTD_ERR_INVALID_TREE);   // malformed sizes
     wl += w;
   }
@@ -204,7 +222,8 @@ __device__ __noinline__ void make_walk_const(const AttnParams& p, WalkConst& wc)
 constexpr int kWalkStart = INT_MIN;
 
 // Next segment of this CTA for one walker (cursor starts at kWalkStart); s.valid = 0 when done.
-__device__ __noinline__ void next_segment(const AttnParams& p, const WalkConst& wc, int& cursor, Seg& s) {
+__device__ __noinline__ void next_segment(const AttnParams& p, const TreeInfo* ti, const WalkConst& wc, int& cursor,
+                                          Seg& s) {
   s.valid = 0;
   if (!wc.persistent) {
     // grid schedule: CTA u computes unit u whole
@@ -218,7 +237,7 @@ __device__ __noinline__ void next_segment(const AttnParams& p, const WalkConst& 
     const int b = u % p.batch;
     s.lq = u / p.batch;
     int node0, T, C, n_kt, pairs;
-    if (seq_info(p, b, node0, T, C, n_kt, pairs) == 0) {
+    if (seq_info(p, ti, b, node0, T, C, n_kt, pairs) == 0) {
       atomicMax(p.dev_status, (int)PTD_ERR_INVALID_TREE);   // malformed sizes
       return;
     }
@@ -235,7 +254,7 @@ __device__ __noinline__ void next_segment(const AttnParams& p, const WalkConst& 
   if (cursor == kWalkStart) cursor = wc.r0;
   if (cursor >= wc.r1) return;
   // self-check: every step must decode and move the cursor forward (the walk then ends)
-  if (!decode_tile(p, wc.Wl, cursor, s) || s.ug0 + s.n_kt <= cursor || s.ug0 > cursor) {
+  if (!decode_tile(p, ti, wc.Wl, cursor, s) || s.ug0 + s.n_kt <= cursor || s.ug0 > cursor) {
     atomicMax(p.dev_status, (int)PTD_ERR_TIMEOUT);
     cursor = wc.r1;
     return;
@@ -251,6 +270,29 @@ __device__ __noinline__ void next_segment(const AttnParams& p, const WalkConst& 
     s.slot = wc.c * 2 + ((wc.r0 >= s.ug0 && wc.r0 < s.ug0 + s.n_kt) ? 0 : 1);
   }
   s.valid = 1;
+}
+
+// Pieces counted on a (unit, 32-row block) counter in this launch: the counter holds
+// (epoch << 32) | count, and a value left by another launch counts as 0, so no launch needs
+// the counters cleared before it.
+__device__ __forceinline__ int epoch_count(unsigned long long v, uint32_t epoch) {
+  return (uint32_t)(v >> 32) == epoch ? (int)(uint32_t)v : 0;
+}
+__device__ __forceinline__ int epoch_read(unsigned long long* ctr, uint32_t epoch) {
+  return epoch_count(atomicAdd(ctr, 0ull), epoch);
+}
+// Adds one piece; returns the count after it, or -1 if the compare-and-swap never settled
+// (bounded: a handful of pieces contend at most).
+__device__ __forceinline__ int epoch_increment(unsigned long long* ctr, uint32_t epoch) {
+  unsigned long long cur = atomicAdd(ctr, 0ull);
+  for (int it = 0; it < 4096; ++it) {
+    const unsigned long long want =
+        epoch_count(cur, epoch) > 0 ? cur + 1ull : (((unsigned long long)epoch << 32) | 1ull);
+    const unsigned long long prev = atomicCAS(ctr, cur, want);
+    if (prev == cur) return (int)(uint32_t)want;
+    cur = prev;
+  }
+  return -1;
 }
 
 // Partial slot of CTA c's piece of the unit starting at global tile ug0 (c owns a piece).
@@ -319,6 +361,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // A grid launched after this one with programmatic stream serialization (the step's top-k)
   // may be scheduled now; its CTAs take the SMs this grid's CTAs leave at its end.
   if (threadIdx.x == 0) grid_launch_dependents();
+  // set-up that reads no global memory: it may overlap the stream's previous grid
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(fullk_bar(s), 1);
@@ -335,14 +378,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
-    make_walk_const(p, *wc_s);
     fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&map_k);
+    prefetch_tensormap(&map_v);
   }
   if (warp == 1) {
     tmem_alloc(base + kOffTmemPtr, kTmemCols);
     tmem_relinquish();
     tc_fence_before();
   }
+  // every input (trees, Q, the cache) and output belongs to the stream's previous work
+  grid_dependency_wait();
+  TreeInfo* const trees_s = reinterpret_cast<TreeInfo*>(smem + kOffTrees);
+  const TreeInfo* const ti = p.batch <= kMaxCachedTrees ? trees_s : nullptr;
+  if (ti != nullptr) {
+    for (int b = threadIdx.x; b < p.batch; b += kThreads) {
+      TreeInfo x;
+      x.wb = seq_info(p, nullptr, b, x.node0, x.T, x.C, x.n_kt, x.pairs);
+      trees_s[b] = x;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) make_walk_const(p, ti, *wc_s);
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + kOffTmemPtr);
@@ -351,17 +410,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile Seg* sgv = my_seg;
   auto advance = [&]() -> bool {
     __syncwarp();
-    if (lane == 0) next_segment(p, wc, cursor, *my_seg);
+    if (lane == 0) next_segment(p, ti, wc, cursor, *my_seg);
     __syncwarp();
     return sgv->valid != 0;
   };
 
   if (warp == 0) {
     // ================================================================ TMA producer
-    if (lane == 0) {
-      prefetch_tensormap(&map_k);
-      prefetch_tensormap(&map_v);
-    }
     bool ok = true;
     int gt = 0;                    // key tiles issued by this CTA (ring position)
     int vloads[kStages] = {0, 0};  // v_load completions per stage (waited on here only)
@@ -795,6 +850,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
+      // A piece: how many of its unit's pieces have left their partials, read now so that the
+      // load overlaps the drain of this segment's last PV (the count only grows; a stale one
+      // sends this warp down the partial path, which counts again).
+      int seen = -1;
+      if (cur->s.slot >= 0 && lane == 0)
+        seen = epoch_read(p.counters + (size_t)cur->s.unit * 8 + t * 4 + (warp & 3), p.epoch);
       // Every S_t GEMM of this segment has completed (its last s_full was seen), so the next
       // segment's Q can go in now: the tensor core starts on it while this epilogue runs.
       const bool have_next = next_mine();
@@ -850,11 +911,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int ug1 = ug0 + cur->s.n_kt;
         const int first = owner_cta(wc, ug0);
         const int last = owner_cta(wc, ug1 - 1);
-        int* counter = p.counters + (size_t)cur->s.unit * 8 + t * 4 + (warp & 3);
+        unsigned long long* counter = p.counters + (size_t)cur->s.unit * 8 + t * 4 + (warp & 3);
         int pieces = 0, done = 0;
         if (lane == 0) {
           for (int c = first; c <= last; ++c) pieces += range_start(wc, c + 1) > range_start(wc, c) ? 1 : 0;
-          done = atomicAdd(counter, 0) == pieces - 1;
+          done = seen == pieces - 1;
         }
         done = __shfl_sync(0xffffffffu, done, 0);
         if (done) {
@@ -876,7 +937,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           __threadfence();
           __syncwarp();
           int is_last = 0;
-          if (lane == 0) is_last = atomicAdd(counter, 1) == pieces - 1;
+          if (lane == 0) {
+            const int now = epoch_increment(counter, p.epoch);
+            if (now < 0) atomicMax(p.dev_status, (int)PTD_ERR_TIMEOUT);
+            is_last = now == pieces;
+          }
           is_last = __shfl_sync(0xffffffffu, is_last, 0);
           if (is_last) {
             __threadfence();
@@ -904,13 +969,22 @@ size_t tc_smem_bytes() { return tc::kSmemBytes; }
 
 cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const CUtensorMap& map_q,
                                 const AttnParams& p, dim3 grid, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(tc::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = tc::kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // set-up overlaps the previous kernel
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
 #define PTD_TC_LAUNCH(PAGED, QTMA)                                                                            \
   do {                                                                                                       \
     cudaError_t e = cudaFuncSetAttribute(tc::tree_attn_tc_kernel<PAGED, QTMA>,                               \
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc::kSmemBytes);  \
     if (e != cudaSuccess) return e;                                                                          \
-    tc::tree_attn_tc_kernel<PAGED, QTMA><<<grid, tc::kThreads, tc::kSmemBytes, stream>>>(map_k, map_v, map_q, \
-                                                                                          p);               \
+    return cudaLaunchKernelEx(&cfg, tc::tree_attn_tc_kernel<PAGED, QTMA>, map_k, map_v, map_q, p);           \
   } while (0)
   if (p.page_size > 0) {
     if (p.q_tma)
@@ -924,7 +998,6 @@ cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map
       PTD_TC_LAUNCH(false, false);
   }
 #undef PTD_TC_LAUNCH
-  return cudaGetLastError();
 }
 
 

@@ -143,7 +143,7 @@ template <int KM, typename T>
 __global__ void __launch_bounds__(kThreads) topk_cluster_kernel(const T* __restrict__ logits, int64_t rows,
                                                                 int vocab, int64_t row_stride, int k,
                                                                 int32_t* __restrict__ out_idx,
-                                                                float* __restrict__ out_val, int early) {
+                                                                float* __restrict__ out_val) {
   constexpr int VN = Vec<T>::kN;
   __shared__ uint64_t warp_keys[kWarps][KM];
   __shared__ uint64_t cta_keys[KM];
@@ -153,7 +153,8 @@ __global__ void __launch_bounds__(kThreads) topk_cluster_kernel(const T* __restr
   const int csize = (int)cluster.num_blocks();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  if (!early) grid_dependency_wait();   // the logits and outputs belong to the stream's previous work
+  if (threadIdx.x == 0) grid_launch_dependents();   // the next grid may be placed now; it waits for this one
+  grid_dependency_wait();   // the logits and outputs belong to the stream's previous work
   for (int64_t r = blockIdx.y; r < rows; r += gridDim.y) {
     const T* row = logits + r * row_stride;
     // vector body [a0, a1): 16-byte aligned; head [0, a0) and tail [a1, vocab) scalar
@@ -231,10 +232,6 @@ __global__ void __launch_bounds__(kThreads) topk_cluster_kernel(const T* __restr
     }
     cluster.sync();   // keep every CTA's shared memory alive until rank 0 has read it
   }
-  // Early start: the logits were complete before the previous grid began, so the rows were
-  // read without waiting; the grid still ends only after the previous grid has, so work
-  // ordered after this launch also finds the previous grid's writes.
-  if (early) grid_dependency_wait();
 }
 
 // ------------------------------------------------------------------ bf16 fast path
@@ -271,8 +268,7 @@ template <int KM>
 __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16* __restrict__ logits,
                                                              int64_t rows, int vocab, int64_t row_stride, int k,
                                                              int32_t* __restrict__ out_idx,
-                                                             float* __restrict__ out_val, int32_t* dev_status,
-                                                             int early) {
+                                                             float* __restrict__ out_val, int32_t* dev_status) {
   extern __shared__ __align__(128) uint4 slice[];
   __shared__ uint64_t warp_keys[kWarps][KM];
   __shared__ uint64_t cta_keys[KM];
@@ -295,7 +291,8 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
     fence_mbar_init();
   }
   __syncthreads();
-  if (!early) grid_dependency_wait();   // the logits and outputs belong to the stream's previous work
+  if (tid == 0) grid_launch_dependents();   // the next grid may be placed now; it waits for this one
+  grid_dependency_wait();   // the logits and outputs belong to the stream's previous work
   uint32_t phase = 0;
 
   for (int64_t r = blockIdx.y; r < rows; r += gridDim.y, phase ^= 1u) {
@@ -498,12 +495,11 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
     }
     cluster.sync();
   }
-  if (early) grid_dependency_wait();   // as in topk_cluster_kernel
 }
 
 template <int KM, typename T, bool kFast>
 cudaError_t launch_km(const T* logits, int64_t rows, int vocab, int64_t row_stride, int k, int32_t* out_idx,
-                      float* out_val, int cluster, int32_t* dev_status, int early, cudaStream_t stream) {
+                      float* out_val, int cluster, int32_t* dev_status, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   const int64_t gy = rows < 65535 ? rows : 65535;
   cfg.gridDim = dim3((unsigned)cluster, (unsigned)gy, 1);
@@ -526,17 +522,17 @@ cudaError_t launch_km(const T* logits, int64_t rows, int vocab, int64_t row_stri
                                          kSliceVec * 16);
     if (e != cudaSuccess) return e;
     return cudaLaunchKernelEx(&cfg, topk_bf16_kernel<KM>, logits, rows, vocab, row_stride, k, out_idx, out_val,
-                              dev_status, early);
+                              dev_status);
   } else {
     cfg.dynamicSmemBytes = 0;
     return cudaLaunchKernelEx(&cfg, topk_cluster_kernel<KM, T>, logits, rows, vocab, row_stride, k, out_idx,
-                              out_val, early);
+                              out_val);
   }
 }
 
 template <typename T, bool kFast>
 cudaError_t launch_t(const T* logits, int64_t rows, int vocab, int64_t row_stride, int k, int32_t* out_idx,
-                     float* out_val, int32_t* dev_status, int early, cudaStream_t stream) {
+                     float* out_val, int32_t* dev_status, cudaStream_t stream) {
   int cluster;
   if (kFast) {
     const int nvec = vocab / 8 + 1;
@@ -547,8 +543,7 @@ cudaError_t launch_t(const T* logits, int64_t rows, int vocab, int64_t row_strid
   }
   cluster = cluster < 1 ? 1 : (cluster > kMaxCluster ? kMaxCluster : cluster);
 #define PTD_TOPK_LAUNCH(KMV) \
-  return launch_km<KMV, T, kFast>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, dev_status, early, \
-                                  stream)
+  return launch_km<KMV, T, kFast>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, dev_status, stream)
   if (k <= 1) PTD_TOPK_LAUNCH(1);
   if (k <= 2) PTD_TOPK_LAUNCH(2);
   if (k <= 4) PTD_TOPK_LAUNCH(4);
@@ -560,18 +555,17 @@ cudaError_t launch_t(const T* logits, int64_t rows, int vocab, int64_t row_strid
 }  // namespace topk
 
 cudaError_t launch_topk(const void* logits, bool bf16, int64_t rows, int vocab, int64_t row_stride, int k,
-                        int32_t* out_idx, float* out_val, int32_t* dev_status, bool early, cudaStream_t stream) {
-  const int e = early ? 1 : 0;
+                        int32_t* out_idx, float* out_val, int32_t* dev_status, cudaStream_t stream) {
   if (bf16) {
     // the shared-memory path covers rows up to kMaxCluster slices of kSliceVec vectors
     if ((int64_t)vocab / 8 + 1 <= (int64_t)topk::kMaxCluster * topk::kSliceVec)
       return topk::launch_t<__nv_bfloat16, true>(static_cast<const __nv_bfloat16*>(logits), rows, vocab,
-                                                 row_stride, k, out_idx, out_val, dev_status, e, stream);
+                                                 row_stride, k, out_idx, out_val, dev_status, stream);
     return topk::launch_t<__nv_bfloat16, false>(static_cast<const __nv_bfloat16*>(logits), rows, vocab, row_stride,
-                                                k, out_idx, out_val, dev_status, e, stream);
+                                                k, out_idx, out_val, dev_status, stream);
   }
   return topk::launch_t<float, false>(static_cast<const float*>(logits), rows, vocab, row_stride, k, out_idx,
-                                      out_val, dev_status, e, stream);
+                                      out_val, dev_status, stream);
 }
 
 }  // namespace ptd

@@ -189,27 +189,48 @@ struct TreeVerdict {
   int invalid;
 };
 
-__device__ void verify_tree_warp(const int32_t* __restrict__ node_offsets, const int32_t* __restrict__ parents,
-                                 const int32_t* __restrict__ tokens, const int32_t* __restrict__ target,
-                                 int target_stride, int n_total, int max_nodes, int b, int* par_s, int* jump_s,
-                                 int* reach_s, int* depth_s, int* onpath_s, int* tgt_s, TreeVerdict* out) {
-  const int lane = threadIdx.x & 31;
-  const int node0 = node_offsets[b];
-  const int T = node_offsets[b + 1] - node0;
-  const bool bad_shape = T < 1 || T > max_nodes || T > kVerifyThreads || node0 < 0 || node0 + T > n_total;
-  bool bad = false;
+// The tree inputs of one verification (warp-collective): first node, size, and the parent
+// and token of nodes lane + 32 q.
+struct TreeInputs {
+  int node0, T, bad_shape;
   int par[4], tok[4];
-  // every node's parent, token and own greedy token V_i at once (no load waits on another)
+};
+
+__device__ __forceinline__ void load_tree_warp(const int32_t* __restrict__ node_offsets,
+                                               const int32_t* __restrict__ parents,
+                                               const int32_t* __restrict__ tokens, int n_total, int max_nodes, int b,
+                                               TreeInputs& in) {
+  const int lane = threadIdx.x & 31;
+  in.node0 = node_offsets[b];
+  in.T = node_offsets[b + 1] - in.node0;
+  in.bad_shape = in.T < 1 || in.T > max_nodes || in.T > kVerifyThreads || in.node0 < 0 || in.node0 + in.T > n_total;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const int i = lane + 32 * q;
-    par[q] = -1;
-    tok[q] = 0;
-    if (!bad_shape && i < T) {
-      par[q] = parents[node0 + i];
-      tok[q] = tokens[node0 + i];
-      tgt_s[i] = target[(size_t)(node0 + i) * target_stride];
+    in.par[q] = -1;
+    in.tok[q] = 0;
+    if (!in.bad_shape && i < in.T) {
+      in.par[q] = parents[in.node0 + i];
+      in.tok[q] = tokens[in.node0 + i];
     }
+  }
+}
+
+__device__ void verify_tree_warp(const TreeInputs& in, const int32_t* __restrict__ target, int target_stride,
+                                 int* par_s, int* jump_s, int* reach_s, int* depth_s, int* onpath_s, int* tgt_s,
+                                 TreeVerdict* out) {
+  const int lane = threadIdx.x & 31;
+  const int node0 = in.node0, T = in.T;
+  const bool bad_shape = in.bad_shape != 0;
+  bool bad = false;
+  int par[4], tok[4];
+  // every node's own greedy token V_i (the parents and tokens are already in registers)
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = lane + 32 * q;
+    par[q] = in.par[q];
+    tok[q] = in.tok[q];
+    if (!bad_shape && i < T) tgt_s[i] = target[(size_t)(node0 + i) * target_stride];
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -307,16 +328,21 @@ __global__ void __launch_bounds__(kCompactThreads)
                           int32_t* __restrict__ bonus, int32_t* __restrict__ dev_status, uint8_t* __restrict__ k_cache,
                           uint8_t* __restrict__ v_cache, int row_bytes, int batch, int page_size, int seq_capacity,
                           int num_pages, const int32_t* __restrict__ block_table, int max_pages,
-                          const int32_t* __restrict__ ctx_lens, int32_t* __restrict__ new_ctx) {
+                          const int32_t* __restrict__ ctx_lens, int32_t* __restrict__ new_ctx, int early_inputs) {
   __shared__ int par_s[kVerifyThreads], jump_s[kVerifyThreads], reach_s[kVerifyThreads];
   __shared__ int depth_s[kVerifyThreads], onpath_s[kVerifyThreads], tgt_s[kVerifyThreads];
   __shared__ TreeVerdict verdict;
   const int layer = blockIdx.x, b = blockIdx.y;
-  grid_dependency_wait();   // the targets and the cache belong to the stream's previous work
-  const int C = ctx_lens[b];   // in flight while warp 0 verifies
+  // early_inputs: the tree arrays and context lengths were written before the previous grids
+  // of the step began (the step's first kernel waits for all earlier work), so they are read
+  // before the wait; the targets and the cache are read only after it
+  if (!early_inputs) grid_dependency_wait();
+  TreeInputs in;
+  if (threadIdx.x < 32) load_tree_warp(node_offsets, parents, tokens, n_total, max_nodes, b, in);
+  const int C = ctx_lens[b];
+  if (early_inputs) grid_dependency_wait();
   if (threadIdx.x < 32)
-    verify_tree_warp(node_offsets, parents, tokens, target, target_stride, n_total, max_nodes, b, par_s, jump_s,
-                     reach_s, depth_s, onpath_s, tgt_s, &verdict);
+    verify_tree_warp(in, target, target_stride, par_s, jump_s, reach_s, depth_s, onpath_s, tgt_s, &verdict);
   __syncthreads();
   int len = verdict.len;
   if (len > max_nodes) len = max_nodes;
@@ -390,7 +416,7 @@ cudaError_t launch_verify_compact(const int32_t* node_offsets, const int32_t* pa
                                   int32_t* accepted, int32_t* accept_len, int32_t* bonus, int32_t* dev_status, void* k,
                                   void* v, int row_bytes, int layers, int batch, int page_size, int seq_capacity,
                                   int num_pages, const int32_t* block_table, int max_pages, const int32_t* ctx_lens,
-                                  int32_t* new_ctx, cudaStream_t stream) {
+                                  int32_t* new_ctx, bool early_inputs, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(layers, batch, 2);
   cfg.blockDim = dim3(vc::kCompactThreads, 1, 1);
@@ -404,7 +430,7 @@ cudaError_t launch_verify_compact(const int32_t* node_offsets, const int32_t* pa
   return cudaLaunchKernelEx(&cfg, vc::verify_compact_kernel, node_offsets, parents, tokens, target, target_stride,
                             n_total, max_nodes, accepted, accept_len, bonus, dev_status, static_cast<uint8_t*>(k),
                             static_cast<uint8_t*>(v), row_bytes, batch, page_size, seq_capacity, num_pages,
-                            block_table, max_pages, ctx_lens, new_ctx);
+                            block_table, max_pages, ctx_lens, new_ctx, early_inputs ? 1 : 0);
 }
 
 cudaError_t launch_compact(void* k, void* v, int row_bytes, int layers, int batch, int page_size, int seq_capacity,

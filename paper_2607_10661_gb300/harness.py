@@ -59,6 +59,25 @@ class DeviceWorkload:
                                     self.topk_val, self.accepted, self.accept_len, self.bonus, self.new_ctx,
                                     self.dev_status, self.workspace) if with_step_buffers else None
 
+    def clone(self) -> "DeviceWorkload":
+        """An independent copy of every device buffer (inputs, cache, outputs, workspace) with
+        its own Tree / KVCache / StepBuffers descriptions: consecutive benchmark steps can
+        alternate between copies so that no step finds the previous one's inputs in L2."""
+        new = DeviceWorkload.__new__(DeviceWorkload)
+        new.w, new.device, new.tdtype = self.w, self.device, self.tdtype
+        c, w = self.w.cfg, self.w
+        for name in ("node_offsets", "parents", "ctx_lens", "k", "v", "q", "logits", "tokens", "attn_out", "topk_idx",
+                     "topk_val", "accepted", "accept_len", "bonus", "new_ctx", "dev_status"):
+            setattr(new, name, getattr(self, name).clone())
+        new.block_table = self.block_table.clone() if self.block_table is not None else None
+        new.workspace = torch.empty_like(self.workspace) if self.workspace is not None else None
+        new.tree = ptd.Tree(new.node_offsets, new.parents, new.ctx_lens, w.max_nodes, w.max_ctx)
+        new.cache = ptd.KVCache(new.k, new.v, c.hkv, c.d, c.page_size, new.block_table)
+        new.bufs = (ptd.StepBuffers(new.q, c.hq, new.attn_out, new.logits, c.k, new.tokens, new.topk_idx,
+                                    new.topk_val, new.accepted, new.accept_len, new.bonus, new.new_ctx,
+                                    new.dev_status, new.workspace) if self.bufs is not None else None)
+        return new
+
     # ---- the whole step, or one call at a time ------------------------------------
     def step(self, stream=None) -> int:
         self.dev_status.zero_()
