@@ -112,6 +112,16 @@ typedef struct {
 size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache,
                                     int32_t num_q_heads, int32_t num_layers);
 
+/* Bytes of scratch the one-call step (ptd_tree_verify_step and the host-buffer and pipelined
+ * steps built on it) wants as ptd_step_args.workspace: the attention's scratch
+ * (ptd_attention_workspace_size, rounded up to 256 bytes) followed by one 4-byte counter per
+ * tree (rounded up to 256 bytes).  With that much (and a bf16 cache), the top-k's CTAs also
+ * verify every tree (the cluster that writes a tree's last row does it) and a copy kernel
+ * compacts; with less, the top-k is followed by ptd_verify_and_compact, every CTA of which
+ * verifies its tree before copying.  The scratch needs no clearing: the attention kernel
+ * clears the tail's counters and tags its own with the launch.  0 for invalid arguments. */
+size_t ptd_step_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t num_q_heads);
+
 /* Tree-masked attention (Sec. 3.1 ancestor-only visibility; Sec. 3.2 one pass over
  * [X; T; C_X]).  For every layer l in [layer_begin, layer_begin + num_layers), tree b,
  * node i and query head h (KV head h / (Hq / Hkv)):
@@ -332,10 +342,15 @@ ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_str
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.
  * Equivalent to ptd_tree_attention, ptd_topk_draft and ptd_verify_and_compact in that
- * order on `stream` (three launches).  Each launch after the first may be placed on the SMs
- * while the one before it drains (programmatic dependent launch); it reads its inputs only
- * after that one has completed, so every kernel sees the previous one's writes, as stream
- * order would give. */
+ * order on `stream` (three launches); when the workspace holds ptd_step_workspace_size
+ * bytes and the logits are bf16 with vocab <= 262143, the top-k's CTAs verify the trees
+ * instead and the third launch only copies the accepted rows (node_offsets must then run
+ * from 0 to total_nodes without decreasing, as ptd_tree states; a tree with an empty or
+ * out-of-range node range is reported as PTD_ERR_INVALID_TREE with accept_len 0, and when
+ * the offsets decrease the outputs of the other trees are unspecified).  Each launch may be
+ * placed on the SMs while the one before it drains (programmatic dependent launch); it reads
+ * its inputs only after that one has completed, so every kernel sees the previous one's
+ * writes, as stream order would give. */
 typedef struct {
   const void* q;               /* [L][N_tot][Hq][D]                                    */
   int32_t num_q_heads;

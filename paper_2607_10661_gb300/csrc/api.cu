@@ -126,6 +126,9 @@ size_t persistent_workspace_bytes(int units, int ctas, int head_dim) {
   return counters_bytes(units) + (size_t)2 * ctas * 256 * ((size_t)head_dim + 2) * sizeof(float);
 }
 
+// The step's tail counters (rows done per tree, epoch-tagged), after the attention's scratch.
+size_t tail_counters_bytes(int batch) { return ((size_t)batch * sizeof(unsigned int) + 255) / 256 * 256; }
+
 // Tile indices of the persistent schedule are 32-bit.
 bool persistent_fits(int units, int n_kt) { return (long long)units * n_kt < (1ll << 30); }
 
@@ -172,9 +175,18 @@ size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* ca
   return persistent_workspace_bytes(units, persistent_ctas(units, n_kt, sms), cache->head_dim);
 }
 
-ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
-                              int32_t num_layers, const void* q, int32_t num_q_heads, float scale, void* out,
-                              void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream) {
+size_t ptd_step_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t num_q_heads) {
+  if (check_tree(tree) != PTD_OK || check_cache(cache) != PTD_OK) return 0;
+  const size_t attn = ptd_attention_workspace_size(tree, cache, num_q_heads, cache->num_layers);
+  return (attn + 255) / 256 * 256 + tail_counters_bytes(tree->batch);
+}
+
+// ptd_tree_attention, and besides: the tensor-core kernel's CTA 0 clears zero_count words at
+// zero_ptr after its dependency wait (the step's tail counters).
+static ptd_status tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
+                                 int32_t num_layers, const void* q, int32_t num_q_heads, float scale, void* out,
+                                 void* workspace, size_t workspace_bytes, int32_t* dev_status, unsigned int* zero_ptr,
+                                 int zero_count, void* stream) {
   g_last_launches = 0;
   ptd_status st = check_tree(tree);
   if (st != PTD_OK) return st;
@@ -210,6 +222,8 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
   const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)D);
   p.scale = sc;
   p.scale_log2 = sc * 1.4426950408889634f;
+  p.zero_ptr = zero_ptr;
+  p.zero_count = zero_ptr != nullptr ? zero_count : 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
 
   if (cache->dtype == PTD_F32) {
@@ -279,6 +293,13 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, i
   return PTD_OK;
 }
 
+ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
+                              int32_t num_layers, const void* q, int32_t num_q_heads, float scale, void* out,
+                              void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream) {
+  return tree_attention(tree, cache, layer_begin, num_layers, q, num_q_heads, scale, out, workspace, workspace_bytes,
+                        dev_status, nullptr, 0, stream);
+}
+
 // Host checks of ptd_topk_draft's arguments (no launch).
 static ptd_status check_topk_args(const void* logits, ptd_dtype dtype, int64_t rows, int32_t vocab,
                                   int64_t row_stride, int32_t k, const int32_t* out_idx, const float* out_val) {
@@ -296,7 +317,7 @@ static ptd_status topk_draft(const void* logits, ptd_dtype dtype, int64_t rows, 
   ptd_status st0 = check_topk_args(logits, dtype, rows, vocab, row_stride, k, out_idx, out_val);
   if (st0 != PTD_OK) return st0;
   const ptd_status st = cuda_status(ptd::launch_topk(logits, dtype == PTD_BF16, rows, vocab, row_stride, k, out_idx,
-                                                     out_val, nullptr, static_cast<cudaStream_t>(stream)));
+                                                     out_val, nullptr, nullptr, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }
@@ -378,7 +399,7 @@ static ptd_status check_verify_compact_args(const ptd_tree* tree, const ptd_kv_c
 static ptd_status verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cache, const int32_t* tokens,
                                      const int32_t* target, int32_t target_stride, int32_t* accepted_nodes,
                                      int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
-                                     int32_t* dev_status, bool early_inputs, void* stream) {
+                                     int32_t* dev_status, void* stream) {
   g_last_launches = 0;
   ptd_status st = check_verify_compact_args(tree, cache, tokens, target, target_stride, accepted_nodes, accept_len,
                                             bonus_token, new_ctx_lens, dev_status);
@@ -388,7 +409,7 @@ static ptd_status verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* c
       tree->node_offsets, tree->parents, tokens, target, target_stride, tree->total_nodes, tree->max_nodes,
       accepted_nodes, accept_len, bonus_token, dev_status, cache->k, cache->v, row_bytes, cache->num_layers,
       tree->batch, cache->page_size, cache->seq_capacity, cache->num_pages, cache->block_table, cache->max_pages,
-      tree->ctx_lens, new_ctx_lens, early_inputs, static_cast<cudaStream_t>(stream)));
+      tree->ctx_lens, new_ctx_lens, static_cast<cudaStream_t>(stream)));
   if (st == PTD_OK) g_last_launches = 1;
   return st;
 }
@@ -398,7 +419,7 @@ ptd_status ptd_verify_and_compact(const ptd_tree* tree, const ptd_kv_cache* cach
                                   int32_t* accept_len, int32_t* bonus_token, int32_t* new_ctx_lens,
                                   int32_t* dev_status, void* stream) {
   return verify_and_compact(tree, cache, tokens, target, target_stride, accepted_nodes, accept_len, bonus_token,
-                            new_ctx_lens, dev_status, false, stream);
+                            new_ctx_lens, dev_status, stream);
 }
 
 ptd_status ptd_draft_tree_update(int32_t batch, int32_t in_stride, const int32_t* in_count, const int32_t* in_parents,
@@ -556,22 +577,58 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
   if ((st = check_topk_args(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
                             a->topk_val)) != PTD_OK)
     return st;
+  // The tail: with room for its counters after the attention's scratch (the size given by
+  // ptd_step_workspace_size), the tensor-core attention (which clears those counters) and bf16
+  // logits on the clustered path, the top-k kernel also verifies every tree (the cluster that
+  // writes a tree's last row does it) and a copy kernel compacts.  Otherwise the top-k, then
+  // verification + compaction in one launch.  Each launch may be placed while the previous one
+  // drains; it reads its inputs only after that one has completed (the top-k's logits come from
+  // the step's forward pass).
+  const size_t attn_ws = (ptd_attention_workspace_size(tree, cache, a->num_q_heads, cache->num_layers) + 255) /
+                         256 * 256;
+  const bool fused = use_tensor_cores(cache) && a->logits_dtype == PTD_BF16 &&
+                     ptd::topk_can_verify(true, a->vocab) && a->workspace && aligned16(a->workspace) &&
+                     a->workspace_bytes >= attn_ws + tail_counters_bytes(tree->batch);
+  unsigned int* tail_counters =
+      fused ? reinterpret_cast<unsigned int*>(static_cast<uint8_t*>(a->workspace) + attn_ws) : nullptr;
   int total = 0;
-  st = ptd_tree_attention(tree, cache, 0, cache->num_layers, a->q, a->num_q_heads, a->scale, a->attn_out,
-                          a->workspace, a->workspace_bytes, a->dev_status, stream);
+  st = tree_attention(tree, cache, 0, cache->num_layers, a->q, a->num_q_heads, a->scale, a->attn_out, a->workspace,
+                      a->workspace_bytes, a->dev_status, tail_counters, tree->batch, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
-  // The top-k's CTAs may be placed while the attention grid drains (programmatic dependent
-  // launch), but they read the logits only once the attention grid has completed: in a model
-  // step the logits come from the forward pass that this attention is part of.
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (fused) {
+    ptd::VerifyArgs va = {};
+    va.node_offsets = tree->node_offsets;
+    va.parents = tree->parents;
+    va.tokens = a->tokens;
+    va.ctx_lens = tree->ctx_lens;
+    va.counters = tail_counters;
+    va.batch = tree->batch;
+    va.n_total = tree->total_nodes;
+    va.max_nodes = tree->max_nodes;
+    va.accepted = a->accepted_nodes;
+    va.accept_len = a->accept_len;
+    va.bonus = a->bonus_token;
+    va.dev_status = a->dev_status;
+    if ((st = cuda_status(ptd::launch_topk(a->logits, true, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
+                                           a->topk_val, a->dev_status, &va, s))) != PTD_OK)
+      return st;
+    const int row_bytes = cache->num_kv_heads * cache->head_dim * (int)dtype_size(cache->dtype);
+    if ((st = cuda_status(ptd::launch_compact(cache->k, cache->v, row_bytes, cache->num_layers, tree->batch,
+                                              cache->page_size, cache->seq_capacity, cache->num_pages,
+                                              cache->block_table, cache->max_pages, tree->ctx_lens, a->accepted_nodes,
+                                              a->accept_len, tree->max_nodes, a->new_ctx_lens, s))) != PTD_OK)
+      return st;
+    g_last_launches = total + 2;
+    return PTD_OK;
+  }
   st = topk_draft(a->logits, a->logits_dtype, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
                   a->topk_val, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
-  // the tree arrays and context lengths are inputs of the step, complete before its
-  // attention (a plain launch) began: the verification reads them before its wait
   st = verify_and_compact(tree, cache, a->tokens, a->topk_idx, a->k, a->accepted_nodes, a->accept_len,
-                          a->bonus_token, a->new_ctx_lens, a->dev_status, true, stream);
+                          a->bonus_token, a->new_ctx_lens, a->dev_status, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
   g_last_launches = total;

@@ -17,6 +17,8 @@ struct AttnParams {
   unsigned long long* counters;   // persistent schedule: pieces finished per (unit, 32-row block):
                                   // (epoch << 32) | count, a value of another epoch counting as 0
   uint32_t epoch;                 // this launch's epoch (never 0)
+  unsigned int* zero_ptr;         // zero_count words that CTA 0 clears after its dependency wait:
+  int zero_count;                 // the step's tail counters, read by the kernels after this one
   const int32_t* node_offsets;
   const int32_t* parents;
   const int32_t* ctx_lens;

@@ -272,29 +272,6 @@ __device__ __noinline__ void next_segment(const AttnParams& p, const TreeInfo* t
   s.valid = 1;
 }
 
-// Pieces counted on a (unit, 32-row block) counter in this launch: the counter holds
-// (epoch << 32) | count, and a value left by another launch counts as 0, so no launch needs
-// the counters cleared before it.
-__device__ __forceinline__ int epoch_count(unsigned long long v, uint32_t epoch) {
-  return (uint32_t)(v >> 32) == epoch ? (int)(uint32_t)v : 0;
-}
-__device__ __forceinline__ int epoch_read(unsigned long long* ctr, uint32_t epoch) {
-  return epoch_count(atomicAdd(ctr, 0ull), epoch);
-}
-// Adds one piece; returns the count after it, or -1 if the compare-and-swap never settled
-// (bounded: a handful of pieces contend at most).
-__device__ __forceinline__ int epoch_increment(unsigned long long* ctr, uint32_t epoch) {
-  unsigned long long cur = atomicAdd(ctr, 0ull);
-  for (int it = 0; it < 4096; ++it) {
-    const unsigned long long want =
-        epoch_count(cur, epoch) > 0 ? cur + 1ull : (((unsigned long long)epoch << 32) | 1ull);
-    const unsigned long long prev = atomicCAS(ctr, cur, want);
-    if (prev == cur) return (int)(uint32_t)want;
-    cur = prev;
-  }
-  return -1;
-}
-
 // Partial slot of CTA c's piece of the unit starting at global tile ug0 (c owns a piece).
 __device__ __forceinline__ int piece_slot(const WalkConst& wc, int c, int ug0, int ug1) {
   const int rs = range_start(wc, c);
@@ -391,6 +368,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   // every input (trees, Q, the cache) and output belongs to the stream's previous work
   grid_dependency_wait();
+  if (blockIdx.x == 0)   // counters of the work that follows this kernel in the step (see AttnParams)
+    for (int i = threadIdx.x; i < p.zero_count; i += kThreads) p.zero_ptr[i] = 0u;
   TreeInfo* const trees_s = reinterpret_cast<TreeInfo*>(smem + kOffTrees);
   const TreeInfo* const ti = p.batch <= kMaxCachedTrees ? trees_s : nullptr;
   if (ti != nullptr) {
@@ -419,6 +398,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ================================================================ TMA producer
     bool ok = true;
     int gt = 0;                    // key tiles issued by this CTA (ring position)
+    // K and V are read once: their lines leave L2 first, so that the stream of them does not
+    // push out what the step's next kernels read (their code, the trees, the top-k rows)
+    const uint64_t kv_policy = l2_policy_evict_first();
     int vloads[kStages] = {0, 0};  // v_load completions per stage (waited on here only)
     while (ok && advance()) {
       const int layer = p.layer_begin + sgv->lq;
@@ -440,8 +422,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (!kPaged) {
                 const int row0 = (layer * p.batch + b) * p.seq_capacity + t0;
                 mbar_arrive_expect_tx(fb, kTileBytes);
-                tma_load_3d(d, map, fb, 0, hkv, row0);
-                tma_load_3d(d + kHalfBytes, map, fb, 64, hkv, row0);
+                tma_load_3d_hint(d, map, fb, 0, hkv, row0, kv_policy);
+                tma_load_3d_hint(d + kHalfBytes, map, fb, 64, hkv, row0, kv_policy);
               } else {
                 const int ps = p.page_size;
                 const int first_page = t0 / ps;
@@ -452,8 +434,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                   const int phys = p.block_table[(size_t)b * p.max_pages + first_page + pg];
                   const int row0 = (layer * p.num_pages + phys) * ps;
                   const uint32_t off = (uint32_t)(pg * ps * 128);
-                  tma_load_3d(d + off, map, fb, 0, hkv, row0);
-                  tma_load_3d(d + kHalfBytes + off, map, fb, 64, hkv, row0);
+                  tma_load_3d_hint(d + off, map, fb, 0, hkv, row0, kv_policy);
+                  tma_load_3d_hint(d + kHalfBytes + off, map, fb, 64, hkv, row0, kv_policy);
                 }
               }
             }

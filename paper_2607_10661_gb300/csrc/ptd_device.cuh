@@ -107,6 +107,29 @@ __device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity, unsign
   }
 }
 
+// ---------------------------------------------------------------- epoch-tagged counters
+// A counter that needs no clearing between launches: it holds (epoch << 32) | count, where the
+// epoch is unique to the launch (never 0), and a value left by another launch counts as 0.
+__device__ __forceinline__ int epoch_count(unsigned long long v, uint32_t epoch) {
+  return (uint32_t)(v >> 32) == epoch ? (int)(uint32_t)v : 0;
+}
+__device__ __forceinline__ int epoch_read(unsigned long long* ctr, uint32_t epoch) {
+  return epoch_count(atomicAdd(ctr, 0ull), epoch);
+}
+// Adds one; returns the count after it, or -1 if the compare-and-swap never settled (bounded:
+// a handful of CTAs contend at most).
+__device__ __forceinline__ int epoch_increment(unsigned long long* ctr, uint32_t epoch) {
+  unsigned long long cur = atomicAdd(ctr, 0ull);
+  for (int it = 0; it < 4096; ++it) {
+    const unsigned long long want =
+        epoch_count(cur, epoch) > 0 ? cur + 1ull : (((unsigned long long)epoch << 32) | 1ull);
+    const unsigned long long prev = atomicCAS(ctr, cur, want);
+    if (prev == cur) return (int)(uint32_t)want;
+    cur = prev;
+  }
+  return -1;
+}
+
 // ---------------------------------------------------------------- programmatic dependent launch
 // Block until the preceding grid in the stream has completed and its writes are visible.
 // With a launch that allows programmatic stream serialization, the code before this call
@@ -134,6 +157,23 @@ __device__ __forceinline__ void tc_fence_after() {
 }
 
 // ---------------------------------------------------------------- TMA
+// An L2 cache policy that evicts the lines it covers before any other (for data read once).
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t policy;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
+  return policy;
+}
+
+// As tma_load_3d, with an L2 cache policy for the lines it brings in.
+__device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap* map, uint32_t bar, int c0, int c1,
+                                                 int c2, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], "
+      "[%1, {%3, %4, %5}], [%2], %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "l"(policy)
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int c0, int c1,
                                             int c2) {
   asm volatile(

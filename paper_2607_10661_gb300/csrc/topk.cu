@@ -19,6 +19,7 @@
 
 #include "ptd_device.cuh"
 #include "topk.cuh"
+#include "verify_tree.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -236,46 +237,35 @@ __global__ void __launch_bounds__(kThreads) topk_cluster_kernel(const T* __restr
 
 // ------------------------------------------------------------------ bf16 fast path
 // Each CTA stages its contiguous slice of the row (up to kSliceVec 16-byte vectors) into
-// shared memory with bulk asynchronous copies, so the row is read from HBM exactly once,
-// then makes three passes over shared memory:
-//   1. every thread's maximum (four vectors in flight per thread);
-//   2. T = the k-th largest warp maximum (k <= 8 warps), else the k-th largest thread
-//      maximum.  The k warps (threads) holding those maxima own k distinct elements >= T,
-//      so every element of the CTA's top-k is >= T;
-//   3. elements >= T become candidates (exact 64-bit keys); warp 0 selects the CTA's top-k
-//      among them.
-// A slice with more than kCandCap candidates (many ties at the threshold, e.g. a constant
-// row) is selected exactly with per-thread sorted lists instead.
+// shared memory with bulk asynchronous copies, so the row is read from HBM exactly once.
+// Then every warp works on its own share of the slice (vectors lane + 32 w + 256 j) without
+// waiting for the others:
+//   1. every lane's maximum;
+//   2. T_w = the k-th largest lane maximum of the warp (k rounds of "largest wins"): the k
+//      lanes holding those maxima own k distinct elements >= T_w, so the warp's top-k is
+//      among its elements >= T_w;
+//   3. each lane keeps its elements >= T_w in an exact sorted list of KM (value, index)
+//      pairs (elements arrive in increasing index order, so ties keep the lower index), and
+//      the warp selects its top-k from the lists' heads.
+// One CTA barrier, then warp 0 merges the 8 warps' lists and the CTAs of the cluster merge
+// theirs over distributed shared memory.  With verification (the step's tail), the cluster
+// that writes the last row of a tree then verifies that tree (greedy, on one warp), so no
+// separate verification launch follows.
 constexpr int kSliceVec = 4096;            // 64 KB of bf16 logits per CTA
-constexpr int kCandCap = 1024;
 constexpr uint32_t kChunkBytes = 16384;    // bytes per bulk copy
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// k rounds of "largest key wins" over one key per lane; lane s < k ends with the s-th largest.
-__device__ __forceinline__ uint64_t warp_topk_of_one(uint64_t key, int k, int lane) {
-  uint64_t mine = key, out = 0ull;
-  for (int s = 0; s < k; ++s) {
-    const uint64_t best = warp_max_u64(mine);
-    if (mine == best) mine = 0ull;
-    if (lane == s) out = best;
-  }
-  return out;
-}
-
-template <int KM>
+template <int KM, bool kVerify>
 __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16* __restrict__ logits,
                                                              int64_t rows, int vocab, int64_t row_stride, int k,
                                                              int32_t* __restrict__ out_idx,
-                                                             float* __restrict__ out_val, int32_t* dev_status) {
+                                                             float* __restrict__ out_val, int32_t* dev_status,
+                                                             const VerifyArgs va) {
   extern __shared__ __align__(128) uint4 slice[];
   __shared__ uint64_t warp_keys[kWarps][KM];
   __shared__ uint64_t cta_keys[KM];
-  __shared__ uint64_t cand[kCandCap];
-  __shared__ int ncand;
-  __shared__ float thr_s;
-  __shared__ float wmax_s[kWarps];
   __shared__ __align__(8) uint64_t bar_s;
   __shared__ int abort_s;
 
@@ -292,7 +282,35 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
   }
   __syncthreads();
   if (tid == 0) grid_launch_dependents();   // the next grid may be placed now; it waits for this one
-  grid_dependency_wait();   // the logits and outputs belong to the stream's previous work
+  // the tree of a row (rank 0's thread 0 looks it up while the row's copy is in flight)
+  auto tree_of = [&](int64_t r) {
+    int lo = 0, hi = va.batch;
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (va.node_offsets[mid] <= r) lo = mid; else hi = mid;
+    }
+    return lo;
+  };
+  int row_tree = 0;
+  grid_dependency_wait();   // the logits, the trees and the outputs belong to the stream's previous work
+  if constexpr (kVerify) {
+    // Trees that no row completes (an empty or out-of-range node range, or offsets that do not
+    // run from 0 to n_total): their outputs and the status are written here, by warp 1 of the
+    // first CTA, while its copy is in flight; a tree whose rows all arrive is verified below.
+    if (blockIdx.x == 0 && blockIdx.y == 0 && warp == 1) {
+      for (int b = lane; b < va.batch; b += 32) {
+        const int n0 = va.node_offsets[b], n1 = va.node_offsets[b + 1];
+        const bool bad = n1 - n0 < 1 || n1 - n0 > va.max_nodes || n0 < 0 || n1 > va.n_total ||
+                         (b == 0 && n0 != 0) || (b == va.batch - 1 && n1 != va.n_total);
+        if (bad) {
+          for (int j = 0; j < va.max_nodes; ++j) va.accepted[(size_t)b * va.max_nodes + j] = -1;
+          va.accept_len[b] = 0;
+          va.bonus[b] = -1;
+          atomicMax(va.dev_status, (int)PTD_ERR_INVALID_TREE);
+        }
+      }
+    }
+  }
   uint32_t phase = 0;
 
   for (int64_t r = blockIdx.y; r < rows; r += gridDim.y, phase ^= 1u) {
@@ -317,6 +335,9 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
         const uint32_t n = total - off < kChunkBytes ? total - off : kChunkBytes;
         bulk_load(smem_u32(slice) + off, reinterpret_cast<const uint8_t*>(vrow) + off, n, bar);
       }
+      if constexpr (kVerify) {
+        if (rank == 0) row_tree = tree_of(r);
+      }
     }
     // head / tail scalars while the copy is in flight
     float tmax = -INFINITY;
@@ -326,7 +347,7 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
       for (int i = a1; i < vocab; ++i) tmax = fmaxf(tmax, Vec<__nv_bfloat16>::scalar(row + i));
     mbar_wait(bar, phase, &abort_s, dev_status);   // bounded: a lost copy only flags PTD_ERR_TIMEOUT
 
-    // pass 1: thread maximum (four vectors in flight, two chains)
+    // 1. lane maximum (four vectors in flight, two chains)
     {
       float t1 = -INFINITY;
       int v = tid;
@@ -353,57 +374,29 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
     }
     const bool has_elems = tid < nv || (own_head && a0 > 0) || (own_tail && a1 < vocab);
 
-    // pass 2: T = k-th largest warp maximum (k <= kWarps: the k warps holding those maxima
-    // own k distinct elements >= T), else the k-th largest thread maximum
-    if (k <= kWarps) {
-      float wm = has_elems ? tmax : -INFINITY;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
-      if (lane == 0) wmax_s[warp] = wm;
-      if (tid == 0) ncand = 0;
-      __syncthreads();
-      float t_k = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < kWarps; ++i) {
-        const float wi = wmax_s[i];
-        int above = 0;
-#pragma unroll
-        for (int j = 0; j < kWarps; ++j) {
-          const float wj = wmax_s[j];
-          above += (wj > wi || (wj == wi && j < i)) ? 1 : 0;
-        }
-        if (above == k - 1) t_k = wi;
+    // 2. T_w: the k-th largest lane maximum of this warp (-inf when fewer lanes hold elements)
+    float thr;
+    {
+      uint64_t mine = has_elems ? make_key(ordered_bits(tmax), (uint32_t)lane) : 0ull;
+      uint64_t kth = 0ull;
+      for (int s = 0; s < k; ++s) {
+        const uint64_t best = warp_max_u64(mine);
+        if (mine == best) mine = 0ull;
+        kth = best;
       }
-      if (tid == 0) thr_s = t_k;
-    } else {
-      const uint64_t key = has_elems ? make_key(ordered_bits(tmax), (uint32_t)tid) : 0ull;
-      const uint64_t wk = warp_topk_of_one(key, k, lane);
-      if (lane < k) warp_keys[warp][lane] = wk;
-      if (tid == 0) ncand = 0;
-      __syncthreads();
-      if (warp == 0) {
-        int cur = 0;
-        uint64_t kth = 0ull;
-        for (int s = 0; s < k; ++s) {
-          const uint64_t mine = (lane < kWarps && cur < k) ? warp_keys[lane][cur] : 0ull;
-          const uint64_t best = warp_max_u64(mine);
-          if (lane < kWarps && mine == best && best != 0ull) ++cur;
-          kth = best;
-        }
-        if (lane == 0) thr_s = kth != 0ull ? from_ordered((uint32_t)(kth >> 32)) : -INFINITY;
-      }
+      thr = kth != 0ull ? from_ordered((uint32_t)(kth >> 32)) : -INFINITY;
     }
-    __syncthreads();
-    const float thr = thr_s;
 
-    // pass 3: candidates >= T
-    auto offer = [&](float f, uint32_t gidx) {
-      if (f >= thr) {
-        const int pos = atomicAdd(&ncand, 1);
-        if (pos < kCandCap) cand[pos] = make_key(ordered_bits(f), gidx);
+    // 3. every lane's exact list of its elements >= T_w, then the warp's top-k
+    ThreadList<KM> list;
+    list.init();
+    if (own_head)
+      for (int i = 0; i < a0; ++i) {
+        const float f = Vec<__nv_bfloat16>::scalar(row + i);
+        if (f >= thr) list.push(ordered_bits(f), (uint32_t)i);
       }
-    };
-    auto scan = [&](const uint4& x, int v) {
+    for (int v = tid; v < nv; v += kThreads) {
+      const uint4 x = slice[v];
       float vm = fmax3(bf16_lo(x.x), bf16_hi(x.x), bf16_lo(x.y));
       vm = fmax3(vm, bf16_hi(x.y), bf16_lo(x.z));
       vm = fmax3(vm, bf16_hi(x.z), bf16_lo(x.w));
@@ -413,93 +406,97 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
         const uint32_t w[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          offer(bf16_lo(w[q]), gi + 2 * q);
-          offer(bf16_hi(w[q]), gi + 2 * q + 1);
+          const float f0 = bf16_lo(w[q]), f1 = bf16_hi(w[q]);
+          if (f0 >= thr) list.push(ordered_bits(f0), gi + 2 * q);
+          if (f1 >= thr) list.push(ordered_bits(f1), gi + 2 * q + 1);
         }
       }
-    };
-    {
-      int v = tid;
-      for (; v + 3 * kThreads < nv; v += 4 * kThreads) {   // four vectors in flight
-        uint4 x[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) x[u] = slice[v + u * kThreads];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) scan(x[u], v + u * kThreads);
-      }
-      for (; v < nv; v += kThreads) scan(slice[v], v);
     }
-    if (own_head)
-      for (int i = 0; i < a0; ++i) offer(Vec<__nv_bfloat16>::scalar(row + i), (uint32_t)i);
     if (own_tail)
-      for (int i = a1; i < vocab; ++i) offer(Vec<__nv_bfloat16>::scalar(row + i), (uint32_t)i);
-    __syncthreads();
-    const int nc = ncand;
-
-    // CTA top-k: from the candidates, or exactly from every element on overflow
-    ThreadList<KM> list;
-    list.init();
-    if (nc <= kCandCap) {
-      // few candidates: warp 0 selects the CTA's top-k by itself (no cross-warp merge)
-      if (warp == 0) {
-        for (int i = lane; i < nc; i += 32) list.push_key(cand[i]);
-        for (int s = 0; s < k; ++s) {
-          const uint64_t mine = list.head();
-          const uint64_t best = warp_max_u64(mine);
-          if (mine == best) list.pop();
-          if (lane == 0) cta_keys[s] = best;
-        }
+      for (int i = a1; i < vocab; ++i) {
+        const float f = Vec<__nv_bfloat16>::scalar(row + i);
+        if (f >= thr) list.push(ordered_bits(f), (uint32_t)i);
       }
-      __syncthreads();   // every thread is done reading the slice
-    } else {
-      if (own_head)
-        for (int i = 0; i < a0; ++i) list.push(ordered_bits(Vec<__nv_bfloat16>::scalar(row + i)), (uint32_t)i);
-      for (int v = tid; v < nv; v += kThreads) {
-        float f[8];
-        Vec<__nv_bfloat16>::unpack(slice[v], f);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) list.push(ordered_bits(f[e]), (uint32_t)(a0 + (v_begin + v) * 8 + e));
-      }
-      if (own_tail)
-        for (int i = a1; i < vocab; ++i) list.push(ordered_bits(Vec<__nv_bfloat16>::scalar(row + i)), (uint32_t)i);
-      for (int s = 0; s < k; ++s) {
-        const uint64_t mine = list.head();
-        const uint64_t best = warp_max_u64(mine);
-        if (mine == best) list.pop();
-        if (lane == 0) warp_keys[warp][s] = best;
-      }
-      __syncthreads();   // also: every thread is done reading the slice
-      if (warp == 0) {
-        int cur = 0;
-        for (int s = 0; s < k; ++s) {
-          const uint64_t mine = (lane < kWarps && cur < k) ? warp_keys[lane][cur] : 0ull;
-          const uint64_t best = warp_max_u64(mine);
-          if (lane < kWarps && mine == best && best != 0ull) ++cur;
-          if (lane == 0) cta_keys[s] = best;
-        }
-      }
+    for (int s = 0; s < k; ++s) {
+      const uint64_t mine = list.head();
+      const uint64_t best = warp_max_u64(mine);
+      if (mine == best) list.pop();
+      if (lane == 0) warp_keys[warp][s] = best;
     }
-    cluster.sync();
-    if (rank == 0 && warp == 0) {
-      const uint64_t* remote = lane < csize ? cluster.map_shared_rank(cta_keys, lane) : nullptr;
+    __syncthreads();   // also: every thread is done reading the slice
+    if (warp == 0) {   // CTA merge across warps (lane w owns warp w's list)
       int cur = 0;
       for (int s = 0; s < k; ++s) {
-        const uint64_t mine = (lane < csize && cur < k) ? remote[cur] : 0ull;
+        const uint64_t mine = (lane < kWarps && cur < k) ? warp_keys[lane][cur] : 0ull;
         const uint64_t best = warp_max_u64(mine);
-        if (lane < csize && mine == best && best != 0ull) ++cur;
-        if (lane == 0) {
-          out_idx[r * k + s] = (int32_t)(~(uint32_t)(best & 0xFFFFFFFFull));
-          out_val[r * k + s] = from_ordered((uint32_t)(best >> 32));
-        }
+        if (lane < kWarps && mine == best && best != 0ull) ++cur;
+        if (lane == 0) cta_keys[s] = best;
       }
     }
     cluster.sync();
+    // cluster merge: lane c of rank 0's warp 0 reads CTA c's sorted list at once, then k rounds
+    // of "largest head wins"; lane s writes entry s
+    if (rank == 0 && warp == 0) {
+      ThreadList<KM> ml;
+      ml.init();
+      if (lane < csize) {
+        const uint64_t* remote = cluster.map_shared_rank(cta_keys, lane);
+        uint64_t got[KM];
+#pragma unroll
+        for (int s = 0; s < KM; ++s) got[s] = s < k ? remote[s] : 0ull;
+#pragma unroll
+        for (int s = 0; s < KM; ++s)
+          if (got[s] != 0ull) ml.push_key(got[s]);
+      }
+      uint64_t out = 0ull;
+      for (int s = 0; s < k; ++s) {
+        const uint64_t mine = ml.head();
+        const uint64_t best = warp_max_u64(mine);
+        if (mine == best && best != 0ull) ml.pop();
+        if (lane == s) out = best;
+      }
+      if (lane < k) {
+        out_idx[r * k + lane] = (int32_t)(~(uint32_t)(out & 0xFFFFFFFFull));
+        out_val[r * k + lane] = from_ordered((uint32_t)(out >> 32));
+      }
+      if constexpr (kVerify) {
+        // the last row of a tree to be written: this cluster verifies the tree
+        int vb = -1;
+        if (lane == 0) {
+          const int b = row_tree;
+          __threadfence();   // this row's top-k is visible before it is counted
+          const int node0 = va.node_offsets[b], T = va.node_offsets[b + 1] - node0;
+          const int done = (int)atomicAdd(va.counters + b, 1u) + 1;
+          if (done == T) vb = b;
+        }
+        vb = __shfl_sync(0xffffffffu, vb, 0);
+        if (vb >= 0) {
+          __shared__ vt::VerifyScratch vsc[1];
+          __shared__ vt::TreeVerdict verdict[1];
+          __threadfence();   // every other row's top-k of the tree was counted after it was written
+          vt::TreeInputs in;
+          vt::load_tree_warp(va.node_offsets, va.parents, va.tokens, va.n_total, va.max_nodes, vb, in);
+          vt::verify_tree_warp(in, out_idx, k, vsc[0], &verdict[0]);
+          __syncwarp();
+          int len = verdict[0].len;
+          if (len > va.max_nodes) len = va.max_nodes;
+          int32_t* acc_row = va.accepted + (size_t)vb * va.max_nodes;
+          for (int j = lane; j < va.max_nodes; j += 32) acc_row[j] = j < len ? verdict[0].path[j] : -1;
+          if (lane == 0) {
+            va.accept_len[vb] = len;
+            va.bonus[vb] = verdict[0].bonus;
+            if (verdict[0].invalid) atomicMax(va.dev_status, (int)PTD_ERR_INVALID_TREE);
+          }
+        }
+      }
+    }
+    cluster.sync();   // keep every CTA's shared memory alive until rank 0 has read it
   }
 }
 
-template <int KM, typename T, bool kFast>
+template <int KM, typename T, bool kFast, bool kVerify>
 cudaError_t launch_km(const T* logits, int64_t rows, int vocab, int64_t row_stride, int k, int32_t* out_idx,
-                      float* out_val, int cluster, int32_t* dev_status, cudaStream_t stream) {
+                      float* out_val, int cluster, int32_t* dev_status, const VerifyArgs& va, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   const int64_t gy = rows < 65535 ? rows : 65535;
   cfg.gridDim = dim3((unsigned)cluster, (unsigned)gy, 1);
@@ -518,11 +515,11 @@ cudaError_t launch_km(const T* logits, int64_t rows, int vocab, int64_t row_stri
     const int nvec = vocab / 8 + 1;
     const int per = (nvec + cluster - 1) / cluster;
     cfg.dynamicSmemBytes = (size_t)per * 16;
-    cudaError_t e = cudaFuncSetAttribute(topk_bf16_kernel<KM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(topk_bf16_kernel<KM, kVerify>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          kSliceVec * 16);
     if (e != cudaSuccess) return e;
-    return cudaLaunchKernelEx(&cfg, topk_bf16_kernel<KM>, logits, rows, vocab, row_stride, k, out_idx, out_val,
-                              dev_status);
+    return cudaLaunchKernelEx(&cfg, topk_bf16_kernel<KM, kVerify>, logits, rows, vocab, row_stride, k, out_idx,
+                              out_val, dev_status, va);
   } else {
     cfg.dynamicSmemBytes = 0;
     return cudaLaunchKernelEx(&cfg, topk_cluster_kernel<KM, T>, logits, rows, vocab, row_stride, k, out_idx,
@@ -530,9 +527,9 @@ cudaError_t launch_km(const T* logits, int64_t rows, int vocab, int64_t row_stri
   }
 }
 
-template <typename T, bool kFast>
+template <typename T, bool kFast, bool kVerify>
 cudaError_t launch_t(const T* logits, int64_t rows, int vocab, int64_t row_stride, int k, int32_t* out_idx,
-                     float* out_val, int32_t* dev_status, cudaStream_t stream) {
+                     float* out_val, int32_t* dev_status, const VerifyArgs& va, cudaStream_t stream) {
   int cluster;
   if (kFast) {
     const int nvec = vocab / 8 + 1;
@@ -543,7 +540,8 @@ cudaError_t launch_t(const T* logits, int64_t rows, int vocab, int64_t row_strid
   }
   cluster = cluster < 1 ? 1 : (cluster > kMaxCluster ? kMaxCluster : cluster);
 #define PTD_TOPK_LAUNCH(KMV) \
-  return launch_km<KMV, T, kFast>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, dev_status, stream)
+  return launch_km<KMV, T, kFast, kVerify>(logits, rows, vocab, row_stride, k, out_idx, out_val, cluster, dev_status, \
+                                           va, stream)
   if (k <= 1) PTD_TOPK_LAUNCH(1);
   if (k <= 2) PTD_TOPK_LAUNCH(2);
   if (k <= 4) PTD_TOPK_LAUNCH(4);
@@ -554,18 +552,30 @@ cudaError_t launch_t(const T* logits, int64_t rows, int vocab, int64_t row_strid
 
 }  // namespace topk
 
+bool topk_can_verify(bool bf16, int vocab) {
+  return bf16 && (int64_t)vocab / 8 + 1 <= (int64_t)topk::kMaxCluster * topk::kSliceVec;
+}
+
 cudaError_t launch_topk(const void* logits, bool bf16, int64_t rows, int vocab, int64_t row_stride, int k,
-                        int32_t* out_idx, float* out_val, int32_t* dev_status, cudaStream_t stream) {
+                        int32_t* out_idx, float* out_val, int32_t* dev_status, const VerifyArgs* va,
+                        cudaStream_t stream) {
+  const VerifyArgs none = {};
   if (bf16) {
     // the shared-memory path covers rows up to kMaxCluster slices of kSliceVec vectors
-    if ((int64_t)vocab / 8 + 1 <= (int64_t)topk::kMaxCluster * topk::kSliceVec)
-      return topk::launch_t<__nv_bfloat16, true>(static_cast<const __nv_bfloat16*>(logits), rows, vocab,
-                                                 row_stride, k, out_idx, out_val, dev_status, stream);
-    return topk::launch_t<__nv_bfloat16, false>(static_cast<const __nv_bfloat16*>(logits), rows, vocab, row_stride,
-                                                k, out_idx, out_val, dev_status, stream);
+    if (topk_can_verify(true, vocab)) {
+      if (va != nullptr)
+        return topk::launch_t<__nv_bfloat16, true, true>(static_cast<const __nv_bfloat16*>(logits), rows, vocab,
+                                                         row_stride, k, out_idx, out_val, dev_status, *va, stream);
+      return topk::launch_t<__nv_bfloat16, true, false>(static_cast<const __nv_bfloat16*>(logits), rows, vocab,
+                                                        row_stride, k, out_idx, out_val, dev_status, none, stream);
+    }
+    if (va != nullptr) return cudaErrorInvalidValue;
+    return topk::launch_t<__nv_bfloat16, false, false>(static_cast<const __nv_bfloat16*>(logits), rows, vocab,
+                                                       row_stride, k, out_idx, out_val, dev_status, none, stream);
   }
-  return topk::launch_t<float, false>(static_cast<const float*>(logits), rows, vocab, row_stride, k, out_idx,
-                                      out_val, dev_status, stream);
+  if (va != nullptr) return cudaErrorInvalidValue;
+  return topk::launch_t<float, false, false>(static_cast<const float*>(logits), rows, vocab, row_stride, k, out_idx,
+                                             out_val, dev_status, none, stream);
 }
 
 }  // namespace ptd

@@ -21,6 +21,7 @@
 
 #include "ptd_device.cuh"
 #include "verify_compact.cuh"
+#include "verify_tree.cuh"
 
 namespace ptd {
 namespace vc {
@@ -127,6 +128,7 @@ __global__ void __launch_bounds__(kCompactThreads)
                       const int32_t* __restrict__ accept_len, int max_nodes, int32_t* __restrict__ new_ctx) {
   const int layer = blockIdx.x, b = blockIdx.y;
   uint8_t* base = blockIdx.z == 0 ? k_cache : v_cache;
+  grid_dependency_wait();   // the path, its length and the cache belong to the stream's previous work
   const int C = ctx_lens[b];
   int len = accept_len[b];
   if (len < 0) len = 0;
@@ -182,145 +184,6 @@ __global__ void __launch_bounds__(kCompactThreads)
 // lane, pointer jumping with warp barriers only), so the path is in shared memory before
 // the copy; CTA (0, b, K) writes the verification outputs.  The computation is that of
 // verify_greedy_kernel followed by kv_compact_kernel.
-struct TreeVerdict {
-  int path[kVerifyThreads];
-  int len;      // accepted length (0: the tree failed the checks)
-  int bonus;
-  int invalid;
-};
-
-// The tree inputs of one verification (warp-collective): first node, size, and the parent
-// and token of nodes lane + 32 q.
-struct TreeInputs {
-  int node0, T, bad_shape;
-  int par[4], tok[4];
-};
-
-__device__ __forceinline__ void load_tree_warp(const int32_t* __restrict__ node_offsets,
-                                               const int32_t* __restrict__ parents,
-                                               const int32_t* __restrict__ tokens, int n_total, int max_nodes, int b,
-                                               TreeInputs& in) {
-  const int lane = threadIdx.x & 31;
-  in.node0 = node_offsets[b];
-  in.T = node_offsets[b + 1] - in.node0;
-  in.bad_shape = in.T < 1 || in.T > max_nodes || in.T > kVerifyThreads || in.node0 < 0 || in.node0 + in.T > n_total;
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int i = lane + 32 * q;
-    in.par[q] = -1;
-    in.tok[q] = 0;
-    if (!in.bad_shape && i < in.T) {
-      in.par[q] = parents[in.node0 + i];
-      in.tok[q] = tokens[in.node0 + i];
-    }
-  }
-}
-
-__device__ void verify_tree_warp(const TreeInputs& in, const int32_t* __restrict__ target, int target_stride,
-                                 int* par_s, int* jump_s, int* reach_s, int* depth_s, int* onpath_s, int* tgt_s,
-                                 TreeVerdict* out) {
-  const int lane = threadIdx.x & 31;
-  const int node0 = in.node0, T = in.T;
-  const bool bad_shape = in.bad_shape != 0;
-  bool bad = false;
-  int par[4], tok[4];
-  // every node's own greedy token V_i (the parents and tokens are already in registers)
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int i = lane + 32 * q;
-    par[q] = in.par[q];
-    tok[q] = in.tok[q];
-    if (!bad_shape && i < T) tgt_s[i] = target[(size_t)(node0 + i) * target_stride];
-  }
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int i = lane + 32 * q;
-    if (!bad_shape && i < T) bad = bad || (i == 0 ? (par[q] != -1) : (par[q] < 0 || par[q] >= i));
-  }
-  if (__any_sync(0xffffffffu, bad) || bad_shape) {
-    if (lane == 0) {
-      out->len = 0;
-      out->bonus = -1;
-      out->invalid = 1;
-    }
-    return;
-  }
-  __syncwarp();   // tgt_s complete
-  // eligible edge into node i: tokens[i] == V_{parent}
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int i = lane + 32 * q;
-    if (i < T) {
-      const int elig = i == 0 ? 1 : (tok[q] == tgt_s[par[q]]);
-      par_s[i] = par[q];
-      jump_s[i] = i == 0 ? 0 : par[q];
-      reach_s[i] = elig;
-      depth_s[i] = i == 0 ? 0 : 1;
-      onpath_s[i] = 0;
-    }
-  }
-  __syncwarp();
-  // pointer jumping: after round r, jump[i] is the 2^r-th ancestor (clamped at the root)
-  for (int r = 0; (1 << r) < T; ++r) {
-    int j[4], rj[4], dj[4], jj[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int i = lane + 32 * q;
-      j[q] = 0;
-      if (i < T) {
-        j[q] = jump_s[i];
-        rj[q] = reach_s[j[q]];
-        dj[q] = depth_s[j[q]];
-        jj[q] = jump_s[j[q]];
-      }
-    }
-    __syncwarp();
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int i = lane + 32 * q;
-      if (i < T && j[q] != 0) {
-        reach_s[i] &= rj[q];
-        depth_s[i] += dj[q];
-        jump_s[i] = jj[q];
-      }
-    }
-    __syncwarp();
-  }
-  int dmax = 0;
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int i = lane + 32 * q;
-    if (i < T && reach_s[i]) dmax = max(dmax, depth_s[i]);
-  }
-  const int D = __reduce_max_sync(0xffffffffu, dmax);
-  // mark every node on a root path that reaches depth D through eligible edges
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int i = lane + 32 * q;
-    if (i < T && reach_s[i] && depth_s[i] == D)
-      for (int a = i; a >= 0 && !onpath_s[a]; a = par_s[a]) onpath_s[a] = 1;
-  }
-  __syncwarp();
-  // the lexicographically smallest longest path, one level per step
-  int cur = 0;
-  if (lane == 0) out->path[0] = 0;
-  for (int d = 1; d <= D; ++d) {
-    int best = 0x7FFFFFFF;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int i = lane + 32 * q;
-      if (i < T && par_s[i] == cur && onpath_s[i]) best = min(best, i);
-    }
-    cur = __reduce_min_sync(0xffffffffu, best);
-    if (lane == 0) out->path[d] = cur;
-  }
-  if (lane == 0) {
-    out->len = D + 1;
-    out->bonus = tgt_s[cur];
-    out->invalid = 0;
-  }
-}
-
 __global__ void __launch_bounds__(kCompactThreads)
     verify_compact_kernel(const int32_t* __restrict__ node_offsets, const int32_t* __restrict__ parents,
                           const int32_t* __restrict__ tokens, const int32_t* __restrict__ target, int target_stride,
@@ -328,21 +191,16 @@ __global__ void __launch_bounds__(kCompactThreads)
                           int32_t* __restrict__ bonus, int32_t* __restrict__ dev_status, uint8_t* __restrict__ k_cache,
                           uint8_t* __restrict__ v_cache, int row_bytes, int batch, int page_size, int seq_capacity,
                           int num_pages, const int32_t* __restrict__ block_table, int max_pages,
-                          const int32_t* __restrict__ ctx_lens, int32_t* __restrict__ new_ctx, int early_inputs) {
-  __shared__ int par_s[kVerifyThreads], jump_s[kVerifyThreads], reach_s[kVerifyThreads];
-  __shared__ int depth_s[kVerifyThreads], onpath_s[kVerifyThreads], tgt_s[kVerifyThreads];
-  __shared__ TreeVerdict verdict;
+                          const int32_t* __restrict__ ctx_lens, int32_t* __restrict__ new_ctx) {
+  __shared__ vt::VerifyScratch vsc;
+  __shared__ vt::TreeVerdict verdict;
   const int layer = blockIdx.x, b = blockIdx.y;
-  // early_inputs: the tree arrays and context lengths were written before the previous grids
-  // of the step began (the step's first kernel waits for all earlier work), so they are read
-  // before the wait; the targets and the cache are read only after it
-  if (!early_inputs) grid_dependency_wait();
-  TreeInputs in;
-  if (threadIdx.x < 32) load_tree_warp(node_offsets, parents, tokens, n_total, max_nodes, b, in);
+  grid_dependency_wait();   // the targets, the trees and the cache belong to the stream's previous work
+  vt::TreeInputs in;
+  if (threadIdx.x < 32) vt::load_tree_warp(node_offsets, parents, tokens, n_total, max_nodes, b, in);
   const int C = ctx_lens[b];
-  if (early_inputs) grid_dependency_wait();
   if (threadIdx.x < 32)
-    verify_tree_warp(in, target, target_stride, par_s, jump_s, reach_s, depth_s, onpath_s, tgt_s, &verdict);
+    vt::verify_tree_warp(in, target, target_stride, vsc, &verdict);
   __syncthreads();
   int len = verdict.len;
   if (len > max_nodes) len = max_nodes;
@@ -416,7 +274,7 @@ cudaError_t launch_verify_compact(const int32_t* node_offsets, const int32_t* pa
                                   int32_t* accepted, int32_t* accept_len, int32_t* bonus, int32_t* dev_status, void* k,
                                   void* v, int row_bytes, int layers, int batch, int page_size, int seq_capacity,
                                   int num_pages, const int32_t* block_table, int max_pages, const int32_t* ctx_lens,
-                                  int32_t* new_ctx, bool early_inputs, cudaStream_t stream) {
+                                  int32_t* new_ctx, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(layers, batch, 2);
   cfg.blockDim = dim3(vc::kCompactThreads, 1, 1);
@@ -430,17 +288,26 @@ cudaError_t launch_verify_compact(const int32_t* node_offsets, const int32_t* pa
   return cudaLaunchKernelEx(&cfg, vc::verify_compact_kernel, node_offsets, parents, tokens, target, target_stride,
                             n_total, max_nodes, accepted, accept_len, bonus, dev_status, static_cast<uint8_t*>(k),
                             static_cast<uint8_t*>(v), row_bytes, batch, page_size, seq_capacity, num_pages,
-                            block_table, max_pages, ctx_lens, new_ctx, early_inputs ? 1 : 0);
+                            block_table, max_pages, ctx_lens, new_ctx);
 }
 
 cudaError_t launch_compact(void* k, void* v, int row_bytes, int layers, int batch, int page_size, int seq_capacity,
                            int num_pages, const int32_t* block_table, int max_pages, const int32_t* ctx_lens,
                            const int32_t* accepted, const int32_t* accept_len, int max_nodes, int32_t* new_ctx,
                            cudaStream_t stream) {
-  vc::kv_compact_kernel<<<dim3(layers, batch, 2), vc::kCompactThreads, 0, stream>>>(
-      static_cast<uint8_t*>(k), static_cast<uint8_t*>(v), row_bytes, batch, page_size, seq_capacity, num_pages,
-      block_table, max_pages, ctx_lens, accepted, accept_len, max_nodes, new_ctx);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(layers, batch, 2);
+  cfg.blockDim = dim3(vc::kCompactThreads, 1, 1);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // placed while the previous kernel drains
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, vc::kv_compact_kernel, static_cast<uint8_t*>(k), static_cast<uint8_t*>(v), row_bytes,
+                            batch, page_size, seq_capacity, num_pages, block_table, max_pages, ctx_lens, accepted,
+                            accept_len, max_nodes, new_ctx);
 }
 
 }  // namespace ptd

@@ -19,5 +19,5 @@ cudaError_t launch_verify_compact(const int32_t* node_offsets, const int32_t* pa
                                   int32_t* accepted, int32_t* accept_len, int32_t* bonus, int32_t* dev_status, void* k,
                                   void* v, int row_bytes, int layers, int batch, int page_size, int seq_capacity,
                                   int num_pages, const int32_t* block_table, int max_pages, const int32_t* ctx_lens,
-                                  int32_t* new_ctx, bool early_inputs, cudaStream_t stream);
+                                  int32_t* new_ctx, cudaStream_t stream);
 }  // namespace ptd

@@ -53,7 +53,10 @@ class DeviceWorkload:
         self.bonus = torch.zeros(c.batch, **i32)
         self.new_ctx = torch.zeros(c.batch, **i32)
         self.dev_status = torch.zeros(1, **i32)
-        nbytes = ptd.attention_workspace_size(self.tree, self.cache, c.hq)
+        # the step's scratch (the attention's, then the tail's per-tree counters), or the
+        # attention's alone for the attention-only workloads
+        nbytes = (ptd.step_workspace_size(self.tree, self.cache, c.hq) if with_step_buffers else
+                  ptd.attention_workspace_size(self.tree, self.cache, c.hq))
         self.workspace = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=dev) if nbytes else None
         self.bufs = ptd.StepBuffers(self.q, c.hq, self.attn_out, self.logits, c.k, self.tokens, self.topk_idx,
                                     self.topk_val, self.accepted, self.accept_len, self.bonus, self.new_ctx,

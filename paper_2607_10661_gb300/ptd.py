@@ -31,6 +31,7 @@ EXPORTED = (
     "ptd_draft_tree_update", "ptd_pool_bytes", "ptd_pool_init", "ptd_pool_merge", "ptd_pool_retrieve",
     "ptd_tree_rope_append", "ptd_lm_head_topk_workspace_size", "ptd_lm_head_topk", "ptd_pipeline_create",
     "ptd_pipeline_submit", "ptd_pipeline_wait", "ptd_pipeline_destroy", "ptd_check_bounded_wait",
+    "ptd_step_workspace_size",
 )
 
 
@@ -87,6 +88,8 @@ def lib() -> ctypes.CDLL:
         L.ptd_last_launch_count.argtypes = []
         L.ptd_attention_workspace_size.restype = sz
         L.ptd_attention_workspace_size.argtypes = [P(_Tree), P(_Cache), i32, i32]
+        L.ptd_step_workspace_size.restype = sz
+        L.ptd_step_workspace_size.argtypes = [P(_Tree), P(_Cache), i32]
         L.ptd_tree_attention.restype = ctypes.c_int
         L.ptd_tree_attention.argtypes = [P(_Tree), P(_Cache), i32, i32, vp, i32, f32, vp, vp, sz, vp, vp]
         L.ptd_tree_attention_noalloc.restype = ctypes.c_int
@@ -224,6 +227,11 @@ class KVCache:
 def attention_workspace_size(tree: Tree, cache: KVCache, num_q_heads: int, num_layers: Optional[int] = None) -> int:
     n = cache.num_layers if num_layers is None else num_layers
     return int(lib().ptd_attention_workspace_size(ctypes.byref(tree.c), ctypes.byref(cache.c), num_q_heads, n))
+
+
+def step_workspace_size(tree: Tree, cache: KVCache, num_q_heads: int) -> int:
+    """ptd_step_workspace_size: the one-call step's scratch (attention's, then the tail's counters)."""
+    return int(lib().ptd_step_workspace_size(ctypes.byref(tree.c), ctypes.byref(cache.c), num_q_heads))
 
 
 def tree_attention(tree: Tree, cache: KVCache, q: torch.Tensor, out: torch.Tensor, num_q_heads: int,

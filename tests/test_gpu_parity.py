@@ -730,3 +730,74 @@ def test_verify_sampling_invalid_tree_and_argument_checks():
     with pytest.raises(RuntimeError):
         ptd.verify_sampling(dw.tree, dw.tokens, dw.logits, 0.0, ua, ub, dw.accepted, dw.accept_len, dw.bonus,
                             dw.dev_status)
+
+
+# ------------------------------------------------------------------ the step's two tails
+
+def _step_outputs(dw):
+    kk = dw.k.cpu()
+    kk = kk.view(torch.int16) if kk.dtype == torch.bfloat16 else kk.view(torch.int32)
+    vv = dw.v.cpu()
+    vv = vv.view(torch.int16) if vv.dtype == torch.bfloat16 else vv.view(torch.int32)
+    return dict(idx=dw.topk_idx.cpu(), val=dw.topk_val.cpu(), acc=dw.accepted.cpu(), alen=dw.accept_len.cpu(),
+                bonus=dw.bonus.cpu(), new_ctx=dw.new_ctx.cpu(), status=int(dw.dev_status.item()), k=kk, v=vv,
+                out=dw.attn_out.cpu())
+
+
+@pytest.mark.parametrize("base,over,seed", [
+    ("llama3-8b-gqa", dict(layers=2, ctx=(300, 300), vocab=50000), 81),
+    ("batched-paged", dict(ctx=(64, 400), vocab=3000), 82),
+    # forty ragged trees of 1-16 nodes: several clusters finish rows of the same tree at once
+    ("batched-paged", dict(batch=40, ctx=(16, 200), nodes=(1, 16), depth_range=(1, 4), vocab=700, hq=8, hkv=2), 83),
+])
+def test_step_fused_tail_equals_three_launch_tail(base, over, seed):
+    """With the step's workspace (ptd_step_workspace_size) the top-k's CTAs verify the trees and
+    a copy kernel compacts; with the attention's workspace alone the step runs the top-k and
+    ptd_verify_and_compact (whose every CTA verifies its tree before copying).  Every output and the cache must be identical,
+    on trees whose draft tokens mostly match their parent's greedy token (long tied paths), with
+    one tree made invalid, and on two steps in a row (the counters' tags change per launch)."""
+    cfg = syn.shrink(syn.CONFIGS[base], **over)
+    outs = []
+    for fused in (True, False):
+        w = syn.Workload(cfg, seed)
+        dw = DeviceWorkload(w)
+        if not fused:
+            small = ptd.attention_workspace_size(dw.tree, dw.cache, cfg.hq)
+            ws = torch.empty(max(small, 16), dtype=torch.uint8, device="cuda")
+            dw.bufs = ptd.StepBuffers(dw.q, cfg.hq, dw.attn_out, dw.logits, cfg.k, dw.tokens, dw.topk_idx,
+                                      dw.topk_val, dw.accepted, dw.accept_len, dw.bonus, dw.new_ctx, dw.dev_status,
+                                      ws if small else None)
+        idx_ref, _ = oracle.topk_rows(syn.widen(w.logits, cfg.dtype), cfg.k)
+        rng = np.random.default_rng(seed)
+        tokens = w.tokens.copy()
+        for b, par in enumerate(w.trees):
+            o = int(w.node_offsets[b])
+            for i in range(1, len(par)):
+                tokens[o + i] = idx_ref[o + par[i], 0] if rng.random() < 0.85 else int(rng.integers(cfg.vocab))
+        dw.tokens.copy_(torch.tensor(tokens, dtype=torch.int32))
+        if cfg.batch > 2:
+            bad = w.parents.copy()
+            o = int(w.node_offsets[1])
+            if int(w.node_offsets[2]) - o > 2:
+                bad[o + 2] = 5 if int(w.node_offsets[2]) - o > 5 else -3    # tree 1: not a tree
+                dw.parents.copy_(torch.tensor(bad))
+        launches = []
+        for _ in range(2):
+            launches.append(dw.step())
+        torch.cuda.synchronize()
+        assert launches == [3, 3]                      # attention, top-k, compaction (+ verification)
+        outs.append(_step_outputs(dw))
+        if cfg.batch <= 2:
+            # and against the oracle: path, length and bonus of every tree
+            for b, par in enumerate(w.trees):
+                sl = w.nodes_of(b)
+                path, n, bo = oracle.verify_greedy(par, tokens[sl], idx_ref[sl, 0])
+                assert int(dw.accept_len[b]) == n and int(dw.bonus[b]) == bo
+                assert dw.accepted[b, :n].cpu().tolist() == path
+    a, b = outs
+    for key in a:
+        if isinstance(a[key], int):
+            assert a[key] == b[key], key
+        else:
+            assert torch.equal(a[key], b[key]), key
+    assert int(a["alen"].max()) > 2
