@@ -105,10 +105,12 @@ typedef struct {
 
 /* Bytes of scratch `ptd_tree_attention` wants for these shapes (0 if it needs none):
  * per-block counters and the fp32 partials of the units that the balanced schedule splits
- * between neighbouring SMs.  Passing less (even 0 with a NULL pointer) is allowed: the
- * call then computes each (layer, tree, KV head, 256-row block) in one CTA, which needs no
- * scratch but leaves SMs idle when such units are few or their count is not a multiple of
- * the SM count. */
+ * between neighbouring SMs (one CTA per SM, two partial slots each: about 266 KB per SM).
+ * Passing less (even 0 with a NULL pointer) is allowed: the call then computes each (layer,
+ * tree, KV head, 256-row block) in one CTA, which needs no scratch but leaves SMs idle when
+ * such units are few or their count is not a multiple of the SM count.  With the scratch, the
+ * call still takes one CTA per unit when an estimate from the shapes favours it (few, short
+ * units, where the balanced cut would split each unit into many pieces to merge). */
 size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache,
                                     int32_t num_q_heads, int32_t num_layers);
 
@@ -148,9 +150,10 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache,
  * loop may not tolerate cudaMalloc, whose implicit device synchronisation stalls every
  * stream.  This variant computes exactly what ptd_tree_attention computes, with the same
  * schedule, but takes its scratch from a fixed array that the library
- * holds in device memory (PTD_STATIC_SCRATCH_BYTES; every GPU that loads the library keeps
- * it until the process exits) instead of from a caller workspace.  The paper has no
- * counterpart of this entry point.
+ * holds in device memory (PTD_STATIC_SCRATCH_BYTES = 48 MiB, enough for the partials of one
+ * CTA per SM on a 152-SM GPU plus the counters of ~100k units; every GPU that loads the
+ * library keeps it until the process exits) instead of from a caller workspace.  The paper
+ * has no counterpart of this entry point.
  *   - Arguments are those of ptd_tree_attention without workspace / workspace_bytes.
  *   - If these shapes need more than PTD_STATIC_SCRATCH_BYTES of scratch
  *     (ptd_attention_workspace_size > PTD_STATIC_SCRATCH_BYTES) the call returns
@@ -164,7 +167,7 @@ ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache,
  *     clearing, but calls whose kernels overlap on the GPU (different streams without
  *     ordering between them) race on the array: serialise them.
  *   - Calls no allocator (no cudaMalloc/cudaFree, no allocating library routine). */
-#define PTD_STATIC_SCRATCH_BYTES ((size_t)8 << 20)
+#define PTD_STATIC_SCRATCH_BYTES ((size_t)48 << 20)
 ptd_status ptd_tree_attention_noalloc(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t layer_begin,
                                       int32_t num_layers, const void* q, int32_t num_q_heads, float scale,
                                       void* out, int32_t* dev_status, void* stream);

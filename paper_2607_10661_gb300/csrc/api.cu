@@ -129,6 +129,24 @@ size_t persistent_workspace_bytes(int units, int ctas, int head_dim) {
 // The step's tail counters (rows done per tree, epoch-tagged), after the attention's scratch.
 size_t tail_counters_bytes(int batch) { return ((size_t)batch * sizeof(unsigned int) + 255) / 256 * 256; }
 
+// Which schedule the shapes favour, from the host-known maxima (estimates in microseconds
+// measured on GB300 with these kernels): a key tile costs ~1.75 us for a unit of two 128-row
+// M tiles (~1.2 us for one), a CTA needs ~6.5 us to its first tile, and under the balanced
+// cut the last piece of a unit merges the others' partials, ~9 us plus ~4 us per partial.
+// One CTA per unit (no pieces, no merges) wins when units are few and short, e.g. a single
+// MHA layer over a short context; the balanced cut wins as soon as units are long or outnumber
+// the SMs.
+bool grid_schedule_cheaper(int units, int n_kt, int m_tiles, int sms) {
+  const double t_tile = m_tiles >= 2 ? 1.75 : 1.2;
+  const double waves = (double)((units + sms - 1) / sms);
+  const double t_grid = 6.5 + waves * n_kt * t_tile;
+  const double W = (double)units * n_kt;
+  const double w = W / (W < sms ? W : sms);
+  const int pieces = (int)((n_kt + w - 1e-9) / w);   // pieces of a unit, about
+  const double t_pers = 6.5 + w * t_tile + (pieces > 1 ? 9.0 + 4.0 * (pieces - 1) : 1.5);
+  return t_grid < t_pers;
+}
+
 // Tile indices of the persistent schedule are 32-bit.
 bool persistent_fits(int units, int n_kt) { return (long long)units * n_kt < (1ll << 30); }
 
@@ -241,8 +259,10 @@ static ptd_status tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache
   p.pairs = pairs;
   const int sms = num_sms_of_current_device();
   const int ctas = persistent_ctas(units, n_kt, sms);
+  const int m_tiles = (tree->max_nodes * (num_q_heads / cache->num_kv_heads) + 127) / 128;
   const bool persistent = persistent_fits(units, n_kt) && workspace != nullptr && aligned16(workspace) &&
-                          workspace_bytes >= persistent_workspace_bytes(units, ctas, D);
+                          workspace_bytes >= persistent_workspace_bytes(units, ctas, D) &&
+                          !grid_schedule_cheaper(units, n_kt, m_tiles, sms);
   dim3 grid;
   if (persistent) {
     p.persistent = 1;

@@ -12,7 +12,7 @@ namespace ptd {
 struct AttnParams {
   const void* q;               // [layers][n_total][hq][D]
   void* out;                   // [layers][n_total][hq][D]
-  float* part_o;               // piece partials: [slot][M tile][D][128 rows] fp32 (O unnormalised)
+  float* part_o;               // piece partials: [slot][M tile][D / 4][128 rows][4] fp32 (O unnormalised)
   float* part_ml;              // [slot][256 rows][2] (running max in log2 units, row sum)
   unsigned long long* counters;   // persistent schedule: pieces finished per (unit, 32-row block):
                                   // (epoch << 32) | count, a value of another epoch counting as 0

@@ -398,8 +398,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ================================================================ TMA producer
     bool ok = true;
     int gt = 0;                    // key tiles issued by this CTA (ring position)
-    // K and V are read once: their lines leave L2 first, so that the stream of them does not
-    // push out what the step's next kernels read (their code, the trees, the top-k rows)
+    // K and V lines leave L2 first: the stream of them (read once per M-tile pair) does not push
+    // out what the step's next kernels read (their code, the trees, the top-k rows)
     const uint64_t kv_policy = l2_policy_evict_first();
     int vloads[kStages] = {0, 0};  // v_load completions per stage (waited on here only)
     while (ok && advance()) {
@@ -729,10 +729,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!partial_of(c)) continue;
           const size_t q = (size_t)piece_slot(wc, c, ug0, ug1);
           const float2 ml = __ldcg(pml + q * 256);
-          const float* po = p.part_o + (q * 2 + t) * (128 * 128) + (size_t)(h * 32) * 128 + row;
+          // partial layout [slot][M tile][column / 4][128 rows][4]: four columns of a row in 16 bytes
+          const float4* po = reinterpret_cast<const float4*>(p.part_o + (q * 2 + t) * (128 * 128)) +
+                             (size_t)(h * 8) * 128 + row;
           float o[32];
 #pragma unroll
-          for (int d = 0; d < 32; ++d) o[d] = __ldcg(po + (size_t)d * 128);
+          for (int g = 0; g < 8; ++g) {
+            const float4 v4 = __ldcg(po + (size_t)g * 128);
+            o[4 * g] = v4.x;
+            o[4 * g + 1] = v4.y;
+            o[4 * g + 2] = v4.z;
+            o[4 * g + 3] = v4.w;
+          }
           // rows of a piece that saw no key were not written: weight 0 and never read into acc
           const float wgt = ml.y > 0.f ? ptx_exp2(ml.x - M) : 0.f;
 #pragma unroll
@@ -885,9 +893,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       } else {
         // A piece.  If every other piece of this 32-row block has left its partial, this warp
         // finishes the block from its own O in TMEM.  Otherwise it leaves a partial (O
-        // unnormalised, running max in log2 units, row sum; column-major per M tile, so each
-        // store of the warp is one 128-byte line) and counts itself in; if that makes it the
-        // last, it merges the partials.  (Ranges are walked forward, so the piece at the start
+        // unnormalised, running max in log2 units, row sum; four columns of a row per 16 bytes,
+        // rows consecutive, so each store of the warp is 512 contiguous bytes) and counts
+        // itself in; if that makes it the last, it merges the partials.  (Ranges are walked forward, so the piece at the start
         // of a range is normally done long before the piece that ends the previous range.)
         const int ug0 = cur->s.ug0;
         const int ug1 = ug0 + cur->s.n_kt;
@@ -904,14 +912,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           __threadfence();
           merge(cur, true, have_o ? m_run : -INFINITY, have_o ? l_run : 0.f);
         } else {
-          float* po = p.part_o + ((size_t)slot * 2 + t) * (128 * 128) + row;
+          float4* po = reinterpret_cast<float4*>(p.part_o + ((size_t)slot * 2 + t) * (128 * 128)) + row;
 #pragma unroll 1
           for (int c = 0; c < 4; ++c) {
             tmem_ld32(tO + (uint32_t)c * 32u, r);
             tmem_ld_wait();
             if (have_o) {
 #pragma unroll
-              for (int e = 0; e < 32; ++e) po[(size_t)(c * 32 + e) * 128] = __uint_as_float(r[e]);
+              for (int g = 0; g < 8; ++g)
+                po[(size_t)(c * 8 + g) * 128] = make_float4(__uint_as_float(r[4 * g]), __uint_as_float(r[4 * g + 1]),
+                                                            __uint_as_float(r[4 * g + 2]), __uint_as_float(r[4 * g + 3]));
             }
           }
           reinterpret_cast<float2*>(p.part_ml)[(size_t)slot * 256 + (size_t)t * 128 + row] =

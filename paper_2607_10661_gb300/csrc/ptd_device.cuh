@@ -164,6 +164,13 @@ __device__ __forceinline__ uint64_t l2_policy_evict_first() {
   return policy;
 }
 
+// The default L2 policy as an explicit one (for loads whose policy is chosen at run time).
+__device__ __forceinline__ uint64_t l2_policy_evict_normal() {
+  uint64_t policy;
+  asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(policy));
+  return policy;
+}
+
 // As tma_load_3d, with an L2 cache policy for the lines it brings in.
 __device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap* map, uint32_t bar, int c0, int c1,
                                                  int c2, uint64_t policy) {

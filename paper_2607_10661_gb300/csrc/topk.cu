@@ -339,6 +339,15 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
         if (rank == 0) row_tree = tree_of(r);
       }
     }
+    // with verification: warp 0 of rank 0 loads its row's tree (parents, tokens) while the copy is
+    // in flight, for the case that this cluster turns out to complete the tree
+    vt::TreeInputs tin;
+    if constexpr (kVerify) {
+      if (rank == 0 && warp == 0) {
+        const int b = __shfl_sync(0xffffffffu, row_tree, 0);
+        vt::load_tree_warp(va.node_offsets, va.parents, va.tokens, va.n_total, va.max_nodes, b, tin);
+      }
+    }
     // head / tail scalars while the copy is in flight
     float tmax = -INFINITY;
     if (own_head)
@@ -465,7 +474,7 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
         if (lane == 0) {
           const int b = row_tree;
           __threadfence();   // this row's top-k is visible before it is counted
-          const int node0 = va.node_offsets[b], T = va.node_offsets[b + 1] - node0;
+          const int T = tin.T;
           const int done = (int)atomicAdd(va.counters + b, 1u) + 1;
           if (done == T) vb = b;
         }
@@ -474,9 +483,7 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
           __shared__ vt::VerifyScratch vsc[1];
           __shared__ vt::TreeVerdict verdict[1];
           __threadfence();   // every other row's top-k of the tree was counted after it was written
-          vt::TreeInputs in;
-          vt::load_tree_warp(va.node_offsets, va.parents, va.tokens, va.n_total, va.max_nodes, vb, in);
-          vt::verify_tree_warp(in, out_idx, k, vsc[0], &verdict[0]);
+          vt::verify_tree_warp(tin, out_idx, k, vsc[0], &verdict[0]);
           __syncwarp();
           int len = verdict[0].len;
           if (len > va.max_nodes) len = va.max_nodes;

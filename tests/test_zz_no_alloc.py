@@ -21,7 +21,7 @@ from paper_2607_10661_gb300.harness import DeviceWorkload
 pytestmark = pytest.mark.gpu
 
 BF16_MAX, BF16_MEAN = 2e-2, 2e-3
-STATIC_SCRATCH_BYTES = 8 << 20     # PTD_STATIC_SCRATCH_BYTES in include/ptd.h
+STATIC_SCRATCH_BYTES = 48 << 20    # PTD_STATIC_SCRATCH_BYTES in include/ptd.h
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -48,14 +48,17 @@ def _case(cfg_name, seed, **over):
 def test_noalloc_matches_workspace_entry_on_consecutive_calls():
     """Bit-identical to the workspace call (the same kernel and schedule, and the merge of a
     unit's pieces runs in a fixed order), on two calls in a row per shape and across shapes,
-    so nothing left in the shared array by one call leaks into the next; the first case is
-    also checked against the oracle."""
+    so nothing left in the shared array by one call leaks into the next; the first case (a long
+    context over few KV heads: the balanced schedule, units cut into pieces whose partials go
+    through the array) is also checked against the oracle."""
     cases = [
-        _case("llama2-7b-layer", 71, hq=8, hkv=8, ctx=(333, 333), vocab=100),
-        _case("batched-paged", 72, batch=2, ctx=(300, 600), vocab=100, hq=8, hkv=2),
+        _case("long-context", 71, ctx=(3000, 3000), vocab=100),
+        _case("llama2-7b-layer", 72, hq=8, hkv=8, ctx=(333, 333), vocab=100),
+        _case("batched-paged", 73, batch=2, ctx=(300, 600), vocab=100, hq=8, hkv=2),
     ]
     for dw, need in cases:
-        assert 0 < need <= STATIC_SCRATCH_BYTES, need     # the split path (scratch) is exercised
+        assert 0 < need <= STATIC_SCRATCH_BYTES, need
+    assert cases[0][1] > (32 << 20)                       # the partials of one CTA per SM
     for dw, _ in cases:
         dw.dev_status.zero_()
         ref = torch.zeros_like(dw.q)
@@ -78,9 +81,14 @@ def test_noalloc_matches_workspace_entry_on_consecutive_calls():
 
 
 def test_noalloc_rejects_problems_beyond_its_scratch():
-    dw, need = _case("long-context", 73, ctx=(3000, 3000), vocab=100)
-    assert need > STATIC_SCRATCH_BYTES
-    out = torch.zeros_like(dw.q)
-    assert _noalloc(dw, out) == ptd.WORKSPACE
-    torch.cuda.synchronize()
-    assert float(out.float().abs().max()) == 0.0          # nothing was launched
+    """Shapes whose scratch exceeds the array (here 262144 (tree, KV head, M-tile pair) units:
+    their piece counters alone take 16 MB) are refused before anything is enqueued; the tree and
+    cache descriptions point at no memory the call may touch."""
+    A = 1 << 24
+    t = ptd._Tree(8192, 8192, 128, 100, A, A + 65536, A + 131072)
+    c = ptd._Cache(A * 2, A * 4, ptd.BF16, 1, 8, 128, 0, 1024, 0, None, 0)
+    need = ptd.lib().ptd_attention_workspace_size(ctypes.byref(t), ctypes.byref(c), 64, 1)
+    assert need > STATIC_SCRATCH_BYTES, need
+    st = ptd.lib().ptd_tree_attention_noalloc(ctypes.byref(t), ctypes.byref(c), 0, 1, A * 8, 64, ctypes.c_float(0.0),
+                                             A * 16, A * 32, ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert st == ptd.WORKSPACE
