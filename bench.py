@@ -358,6 +358,8 @@ def run_gpu(args, rank: int, world: int, dist):
                  [torch.empty((1, ptd.MAX_TREE_NODES), dtype=torch.int32, device=dev) for _ in range(3)] + \
                  [torch.empty((1, w.n_total), dtype=torch.int32, device=dev)]
 
+    attn_kernels = [1]   # kernels of one attention call: 2 when split units are merged after it
+
     def parts_step(d, ev=None, record=None):
         """One step of copy d through the entry points one by one; `record(event)` around the
         attention when timing it."""
@@ -366,7 +368,9 @@ def run_gpu(args, rank: int, world: int, dist):
             n += ptd.tree_rope_append(d.tree, d.cache, 0, d.q, cfg.hq, tree_k, tree_v, 500000.0, d.dev_status)
         if ev is not None:
             record(ev[0])
-        n += d.attention()
+        na = d.attention()
+        attn_kernels[0] = na
+        n += na
         if ev is not None:
             record(ev[1])
         if args.lm_head:
@@ -452,7 +456,7 @@ def run_gpu(args, rank: int, world: int, dist):
         return a.elapsed_time(b)
 
     main = Regions(dist, dev).run(graph_region if graphs is not None else eager_region)
-    launches_per_region = launches[0] if graphs is None else K * 3
+    launches_per_region = launches[0]   # the kernels of K steps (the captured steps, or the eager ones)
     eager = Regions(dist, dev).run(eager_region) if graphs is not None else main
     status = 0
     for d in copies:
@@ -538,6 +542,8 @@ def run_gpu(args, rank: int, world: int, dist):
                 "frac": round(achieved_gbs / hbm_peak, 4), "peak_kind": peak_kind,
                 "tensor_tflops": round(achieved_tf, 1), "tensor_frac": round(achieved_tf / tf_peak, 4)}
     kernel = "tree_attn_tc_kernel" if cfg.dtype == "bf16" else "tree_attn_simt_kernel"
+    if attn_kernels[0] == 2:   # timed from the attention's start to the end of the merge of split units
+        kernel += " + tree_attn_merge_kernel"
     roof.update({"kernel": kernel, "traffic": _profiled_traffic(PROFILED_ATTENTION_TRAFFIC, "attention_tc.cu",
                                                                  (cfg.name, cfg.layers)),
                  "bytes_per_launch": nb["attention"], "flops_per_launch": flops, "avg_launch_ms": round(attn_ms, 5),

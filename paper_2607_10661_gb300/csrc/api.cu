@@ -136,14 +136,22 @@ size_t tail_counters_bytes(int batch) { return ((size_t)batch * sizeof(unsigned 
 // One CTA per unit (no pieces, no merges) wins when units are few and short, e.g. a single
 // MHA layer over a short context; the balanced cut wins as soon as units are long or outnumber
 // the SMs.
+// Where the pieces of split units are merged: fewer units than CTAs means many pieces per
+// unit, merged best by tree_attn_merge_kernel over many CTAs after the attention; otherwise
+// the last piece of each unit merges inside the attention, overlapping other CTAs' tiles.
+bool defer_merge(int units, int ctas) { return units < ctas; }
+
 bool grid_schedule_cheaper(int units, int n_kt, int m_tiles, int sms) {
   const double t_tile = m_tiles >= 2 ? 1.75 : 1.2;
   const double waves = (double)((units + sms - 1) / sms);
   const double t_grid = 6.5 + waves * n_kt * t_tile;
   const double W = (double)units * n_kt;
-  const double w = W / (W < sms ? W : sms);
+  const int ctas = (int)(W < sms ? W : sms);
+  const double w = W / ctas;
   const int pieces = (int)((n_kt + w - 1e-9) / w);   // pieces of a unit, about
-  const double t_pers = 6.5 + w * t_tile + (pieces > 1 ? 9.0 + 4.0 * (pieces - 1) : 1.5);
+  double merge = 1.5;
+  if (pieces > 1) merge = defer_merge(units, ctas) ? 4.0 + 1.0 * pieces : 9.0 + 4.0 * (pieces - 1);
+  const double t_pers = 6.5 + w * t_tile + merge;
   return t_grid < t_pers;
 }
 
@@ -270,6 +278,8 @@ static ptd_status tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache
     p.epoch = next_epoch();
     p.part_o = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + counters_bytes(units));
     p.part_ml = p.part_o + (size_t)2 * ctas * 256 * D;
+    p.defer_merge = defer_merge(units, ctas) ? 1 : 0;
+    p.ctas = ctas;
     grid = dim3((unsigned)ctas, 1, 1);
   } else {
     p.persistent = 0;   // one CTA per unit, no scratch
@@ -310,6 +320,10 @@ static ptd_status tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache
   }
   if ((st = cuda_status(ptd::launch_tree_attn_tc(map_k, map_v, map_q, p, grid, s))) != PTD_OK) return st;
   g_last_launches = 1;
+  if (p.persistent && p.defer_merge) {
+    if ((st = cuda_status(ptd::launch_tree_attn_merge(p, units, sms, s))) != PTD_OK) return st;
+    g_last_launches = 2;
+  }
   return PTD_OK;
 }
 

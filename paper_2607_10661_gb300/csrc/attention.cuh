@@ -31,6 +31,8 @@ struct AttnParams {
   int n_total, max_nodes;
   int pairs;                   // 256-row M-tile pairs per (tree, KV head)
   int persistent;              // 1: balanced persistent schedule, one CTA per SM
+  int defer_merge;             // persistent: every piece leaves a partial; tree_attn_merge_kernel merges
+  int ctas;                    // persistent: the attention grid's CTAs (the cut the merge kernel follows)
   int q_tma;                   // 1: Q tiles arrive by TMA (map_q), else by per-thread loads
   int page_size, seq_capacity, num_pages, max_pages;
   float scale_log2;            // scale * log2(e)
@@ -44,5 +46,8 @@ size_t tc_smem_bytes();
 cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const CUtensorMap& map_q,
                                 const AttnParams& p, dim3 grid, cudaStream_t stream);
 cudaError_t launch_tree_attn_simt(const AttnParams& p, cudaStream_t stream);
+// The merge of the units the persistent cut split, after the attention kernel (programmatic
+// dependent launch): one CTA per unit, the pieces' partials combined in CTA order.
+cudaError_t launch_tree_attn_merge(const AttnParams& p, int units, int sms, cudaStream_t stream);
 
 }  // namespace ptd

@@ -844,7 +844,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // load overlaps the drain of this segment's last PV (the count only grows; a stale one
       // sends this warp down the partial path, which counts again).
       int seen = -1;
-      if (cur->s.slot >= 0 && lane == 0)
+      if (cur->s.slot >= 0 && lane == 0 && !p.defer_merge)
         seen = epoch_read(p.counters + (size_t)cur->s.unit * 8 + t * 4 + (warp & 3), p.epoch);
       // Every S_t GEMM of this segment has completed (its last s_full was seen), so the next
       // segment's Q can go in now: the tensor core starts on it while this epilogue runs.
@@ -907,7 +907,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = first; c <= last; ++c) pieces += range_start(wc, c + 1) > range_start(wc, c) ? 1 : 0;
           done = seen == pieces - 1;
         }
-        done = __shfl_sync(0xffffffffu, done, 0);
+        done = __shfl_sync(0xffffffffu, done, 0) && !p.defer_merge;
         if (done) {
           __threadfence();
           merge(cur, true, have_o ? m_run : -INFINITY, have_o ? l_run : 0.f);
@@ -926,15 +926,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           reinterpret_cast<float2*>(p.part_ml)[(size_t)slot * 256 + (size_t)t * 128 + row] =
               have_o ? make_float2(m_run, l_run) : make_float2(-INFINITY, 0.f);
-          __threadfence();
-          __syncwarp();
           int is_last = 0;
-          if (lane == 0) {
-            const int now = epoch_increment(counter, p.epoch);
-            if (now < 0) atomicMax(p.dev_status, (int)PTD_ERR_TIMEOUT);
-            is_last = now == pieces;
+          if (!p.defer_merge) {   // count in; the last piece merges (else the merge kernel does)
+            __threadfence();
+            __syncwarp();
+            if (lane == 0) {
+              const int now = epoch_increment(counter, p.epoch);
+              if (now < 0) atomicMax(p.dev_status, (int)PTD_ERR_TIMEOUT);
+              is_last = now == pieces;
+            }
+            is_last = __shfl_sync(0xffffffffu, is_last, 0);
           }
-          is_last = __shfl_sync(0xffffffffu, is_last, 0);
           if (is_last) {
             __threadfence();
             merge(cur, false, 0.f, 0.f);
@@ -954,10 +956,149 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ------------------------------------------------------------------- merge of split units
+// CTA (unit, column part) of the persistent cut, 256 threads = (M tile t, row); the unit's
+// 128 output columns are cut into `hsplit` parts (1, 2 or 4) of 128 / hsplit columns.  A unit
+// whose key tiles fall in one CTA's range was written whole by the attention; otherwise
+// every piece left a partial and the rows are
+//   O = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c   over the pieces in CTA order
+// (M the maximum over the pieces; a piece that saw no key has l_c = 0 and weight 0).
+constexpr int kMergeThreads = 256;
+constexpr int kMergeBatch = 2;   // pieces whose partial columns are in flight at a time
+constexpr int kMergeMl = 8;      // pieces whose (m, l) stay in registers
+
+__global__ void __launch_bounds__(kMergeThreads, 2) tree_attn_merge_kernel(const AttnParams p, int hsplit) {
+  if (threadIdx.x == 0) grid_launch_dependents();   // the next grid may be placed now; it waits for this one
+  grid_dependency_wait();   // the partials and the trees belong to the attention grid before this one
+  int u = blockIdx.x / hsplit;
+  const int hs = blockIdx.x - u * hsplit;
+  const int mp = u % p.pairs;
+  u /= p.pairs;
+  const int hkv = u % p.hkv;
+  u /= p.hkv;
+  const int b = u % p.batch;
+  const int lq = u / p.batch;
+  int node0, T, C, n_kt, pairs_b;
+  if (seq_info(p, nullptr, b, node0, T, C, n_kt, pairs_b) == 0 || mp >= pairs_b) return;
+  // the flattened (unit, key tile) position of the unit, as the attention's walk decodes it
+  int wl = 0, before = 0;
+  for (int bb = 0; bb < p.batch; ++bb) {
+    int n0, tt, cc, nk, pr;
+    const int w = seq_info(p, nullptr, bb, n0, tt, cc, nk, pr);
+    if (bb < b) before += w;
+    wl += w;
+  }
+  WalkConst wc;
+  wc.persistent = 1;
+  wc.Wl = wl;
+  wc.W = wl * p.layers;
+  wc.P = p.ctas;
+  wc.c = 0;
+  wc.r0 = wc.r1 = 0;
+  const int ug0 = lq * wl + before + (hkv * pairs_b + mp) * n_kt, ug1 = ug0 + n_kt;
+  const int first = owner_cta(wc, ug0), last = owner_cta(wc, ug1 - 1);
+  if (first == last) return;   // whole: written by the attention
+  const int t = threadIdx.x >> 7, row = threadIdx.x & 127;
+  const int nt = min(2, (T * p.group + 127) / 128 - 2 * mp);
+  if (t >= nt) return;
+  const int G = p.group;
+  const int grow = (2 * mp + t) * 128 + row;
+  const int node = grow / G, g = grow - node * G;
+  if (node >= T) return;   // padding row of the M tile: no output
+  const float2* pml = reinterpret_cast<const float2*>(p.part_ml) + (size_t)t * 128 + row;
+  auto has_piece = [&](int c) { return c <= last && range_start(wc, c + 1) > range_start(wc, c); };
+  auto piece_ml = [&](int c) -> float2 {
+    return has_piece(c) ? __ldcg(pml + (size_t)piece_slot(wc, c, ug0, ug1) * 256) : make_float2(-INFINITY, 0.f);
+  };
+  float2 mlc[kMergeMl];
+#pragma unroll
+  for (int q = 0; q < kMergeMl; ++q) mlc[q] = piece_ml(first + q);
+  float M = -INFINITY, L = 0.f;
+#pragma unroll
+  for (int q = 0; q < kMergeMl; ++q)
+    if (mlc[q].y > 0.f) M = fmaxf(M, mlc[q].x);
+  for (int c = first + kMergeMl; c <= last; ++c) {
+    const float2 ml = piece_ml(c);
+    if (ml.y > 0.f) M = fmaxf(M, ml.x);
+  }
+#pragma unroll
+  for (int q = 0; q < kMergeMl; ++q)
+    if (mlc[q].y > 0.f) L += mlc[q].y * ptx_exp2(mlc[q].x - M);
+  for (int c = first + kMergeMl; c <= last; ++c) {
+    const float2 ml = piece_ml(c);
+    if (ml.y > 0.f) L += ml.y * ptx_exp2(ml.x - M);
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  const size_t orow = (((size_t)lq * p.n_total + node0 + node) * p.hq + (size_t)hkv * G + g) * 128;
+  uint4* dst = reinterpret_cast<uint4*>(p.out) + orow / 8;
+  const int h_per = 4 / hsplit;
+#pragma unroll 1
+  for (int h = hs * h_per; h < (hs + 1) * h_per; ++h) {   // 32 output columns at a time
+    float acc[32];
+#pragma unroll
+    for (int d = 0; d < 32; ++d) acc[d] = 0.f;
+    for (int c0 = first; c0 <= last; c0 += kMergeBatch) {
+      float4 o[kMergeBatch][8];
+      float wgt[kMergeBatch];
+#pragma unroll
+      for (int q = 0; q < kMergeBatch; ++q) {
+        const int c = c0 + q;
+        wgt[q] = 0.f;
+        if (has_piece(c)) {
+          const size_t sl = (size_t)piece_slot(wc, c, ug0, ug1);
+          const float2 ml = __ldcg(pml + sl * 256);
+          const float4* po = reinterpret_cast<const float4*>(p.part_o + (sl * 2 + t) * (128 * 128)) +
+                             (size_t)(h * 8) * 128 + row;
+#pragma unroll
+          for (int gg = 0; gg < 8; ++gg) o[q][gg] = __ldcg(po + (size_t)gg * 128);
+          // rows of a piece that saw no key were not written: weight 0 and never read into acc
+          wgt[q] = ml.y > 0.f ? ptx_exp2(ml.x - M) : 0.f;
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < kMergeBatch; ++q) {
+        if (wgt[q] > 0.f) {
+#pragma unroll
+          for (int gg = 0; gg < 8; ++gg) {
+            acc[4 * gg] = fmaf(wgt[q], o[q][gg].x, acc[4 * gg]);
+            acc[4 * gg + 1] = fmaf(wgt[q], o[q][gg].y, acc[4 * gg + 1]);
+            acc[4 * gg + 2] = fmaf(wgt[q], o[q][gg].z, acc[4 * gg + 2]);
+            acc[4 * gg + 3] = fmaf(wgt[q], o[q][gg].w, acc[4 * gg + 3]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int c8 = 0; c8 < 4; ++c8) {
+      uint32_t w[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) w[e] = pack_bf16x2(acc[c8 * 8 + 2 * e] * inv, acc[c8 * 8 + 2 * e + 1] * inv);
+      dst[h * 4 + c8] = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+  }
+}
+
 }  // namespace tc
 
 // ------------------------------------------------------------------- host launchers
 size_t tc_smem_bytes() { return tc::kSmemBytes; }
+
+cudaError_t launch_tree_attn_merge(const AttnParams& p, int units, int sms, cudaStream_t stream) {
+  // column parts per unit: about two CTAs per SM over the grid (1, 2 or 4)
+  const int want = units > 0 ? 2 * sms / units : 1;
+  const int hsplit = want >= 4 ? 4 : (want >= 2 ? 2 : 1);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(units * hsplit), 1, 1);
+  cfg.blockDim = dim3(tc::kMergeThreads, 1, 1);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // placed while the attention drains
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, tc::tree_attn_merge_kernel, p, hsplit);
+}
 
 cudaError_t launch_tree_attn_tc(const CUtensorMap& map_k, const CUtensorMap& map_v, const CUtensorMap& map_q,
                                 const AttnParams& p, dim3 grid, cudaStream_t stream) {
