@@ -129,13 +129,18 @@ __global__ void __launch_bounds__(kCompactThreads)
   const int layer = blockIdx.x, b = blockIdx.y;
   uint8_t* base = blockIdx.z == 0 ? k_cache : v_cache;
   grid_dependency_wait();   // the path, its length and the cache belong to the stream's previous work
+  const int32_t* path = accepted + (size_t)b * max_nodes;
+  // the path's first entries are read together with its length and the context (one round
+  // trip for the common short path)
+  int head[kGroup];
+#pragma unroll
+  for (int q = 0; q < kGroup; ++q) head[q] = 1 + q < max_nodes ? path[1 + q] : 0;
   const int C = ctx_lens[b];
   int len = accept_len[b];
   if (len < 0) len = 0;
   if (len > max_nodes) len = max_nodes;
   if (layer == 0 && blockIdx.z == 0 && threadIdx.x == 0) new_ctx[b] = C + len;
   if (len <= 1 || C < 0) return;   // the root already sits at slot C
-  const int32_t* path = accepted + (size_t)b * max_nodes;
   const int cap = page_size > 0 ? max_pages * page_size : seq_capacity;
 
   auto row_ptr = [&](int slot) -> uint8_t* {
@@ -161,8 +166,9 @@ __global__ void __launch_bounds__(kCompactThreads)
         v[q] = make_uint4(0, 0, 0, 0);
         ok[q] = false;
         if (j < len) {
-          const int src = C + path[j];
-          const uint8_t* sp = (path[j] > j && src < cap) ? row_ptr(src) : nullptr;
+          const int pj = j0 == 1 ? head[q] : path[j];
+          const int src = C + pj;
+          const uint8_t* sp = (pj > j && src < cap) ? row_ptr(src) : nullptr;
           if (sp) {
             v[q] = reinterpret_cast<const uint4*>(sp)[c];
             ok[q] = true;
