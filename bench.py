@@ -52,8 +52,8 @@ METRIC = "tree-verify steps/sec (HBM GB/s and fraction of ~8 TB/s alongside)"
 # dram__bytes_read.sum + dram__bytes_write.sum per attention launch from one ncu capture,
 # keyed by (workload, the kernel source's sha256 prefix): a changed kernel reports null
 # until it is captured again
-PROFILED_ATTENTION_TRAFFIC = {(("llama3-8b-gqa", 32), "4167daf4590b1377"): 1112696832}
-PROFILED_LM_HEAD_TRAFFIC = {"541fa109411fd935": 1053963264}
+PROFILED_ATTENTION_TRAFFIC = {(("llama3-8b-gqa", 32), "230897d3805009aa"): 1112288000}
+PROFILED_LM_HEAD_TRAFFIC = {"541fa109411fd935": 1056455936}
 MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0

@@ -217,14 +217,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 // per warp and once more across the warps.
 constexpr int kMergeThreads = 128;
 
+// Largest key of the warp: the largest high word (one warp reduction), then the largest low
+// word among the lanes that hold it (a second one).
 template <int KM>
 __device__ __forceinline__ uint64_t warp_max_u64(uint64_t x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const uint64_t y = __shfl_xor_sync(0xffffffffu, x, o);
-    x = y > x ? y : x;
-  }
-  return x;
+  const uint32_t hi = (uint32_t)(x >> 32);
+  const uint32_t mhi = __reduce_max_sync(0xffffffffu, hi);
+  const uint32_t mlo = __reduce_max_sync(0xffffffffu, hi == mhi ? (uint32_t)x : 0u);
+  return ((uint64_t)mhi << 32) | mlo;
 }
 
 template <int KM>

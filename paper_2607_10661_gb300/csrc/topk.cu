@@ -45,13 +45,13 @@ __device__ __forceinline__ uint64_t make_key(uint32_t ord, uint32_t idx) {
   return ((uint64_t)ord << 32) | (uint64_t)(~idx);
 }
 
+// Largest key of the warp: the largest high word (one warp reduction), then the largest low
+// word among the lanes that hold it (a second one).
 __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const uint64_t w = __shfl_xor_sync(0xffffffffu, v, o);
-    v = w > v ? w : v;
-  }
-  return v;
+  const uint32_t hi = (uint32_t)(v >> 32);
+  const uint32_t mhi = __reduce_max_sync(0xffffffffu, hi);
+  const uint32_t mlo = __reduce_max_sync(0xffffffffu, hi == mhi ? (uint32_t)v : 0u);
+  return ((uint64_t)mhi << 32) | mlo;
 }
 
 // Sorted (descending) per-thread list of the KM best elements seen by this thread.
