@@ -109,8 +109,9 @@ typedef struct {
  * Passing less (even 0 with a NULL pointer) is allowed: the call then computes each (layer,
  * tree, KV head, 256-row block) in one CTA, which needs no scratch but leaves SMs idle when
  * such units are few or their count is not a multiple of the SM count.  With the scratch, the
- * call still takes one CTA per unit when an estimate from the shapes favours it (few, short
- * units, where the balanced cut would split each unit into many pieces to merge). */
+ * call still takes one CTA per unit when an estimate from the shapes favours it; with fewer
+ * units than SMs (every unit then cut into several pieces) the pieces' partials are merged by
+ * a second kernel launched right after the attention, otherwise inside it. */
 size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache,
                                     int32_t num_q_heads, int32_t num_layers);
 
@@ -137,7 +138,8 @@ size_t ptd_step_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache, 
  *   dev_status: device int32, atomicMax'ed with PTD_ERR_INVALID_TREE if a tree is
  *           invalid (that tree's outputs are zero) or PTD_ERR_TIMEOUT.
  * The tree's own K/V must already be in slots C_b .. C_b + T_b - 1 (position
- * encoding is applied by the caller before the call). */
+ * encoding is applied by the caller before the call).  One launch, or two when the partials
+ * of split units are merged by a kernel of their own (see ptd_attention_workspace_size). */
 ptd_status ptd_tree_attention(const ptd_tree* tree, const ptd_kv_cache* cache,
                               int32_t layer_begin, int32_t num_layers,
                               const void* q, int32_t num_q_heads, float scale, void* out,
@@ -345,7 +347,8 @@ ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_str
 /* One whole tree-verify step on device buffers: attention over all cache layers,
  * top-k of the logits, greedy verification on top-k column 0, KV compaction.
  * Equivalent to ptd_tree_attention, ptd_topk_draft and ptd_verify_and_compact in that
- * order on `stream` (three launches); when the workspace holds ptd_step_workspace_size
+ * order on `stream` (three launches, or four with the attention's merge kernel); when the
+ * workspace holds ptd_step_workspace_size
  * bytes and the logits are bf16 with vocab <= 262143, the top-k's CTAs verify the trees
  * instead and the third launch only copies the accepted rows (node_offsets must then run
  * from 0 to total_nodes without decreasing, as ptd_tree states; a tree with an empty or
