@@ -107,6 +107,15 @@ __device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity, unsign
   }
 }
 
+// Global atomic add with acquire-release semantics at GPU scope: the caller's earlier writes
+// (and those ordered before them by a barrier) are visible before the count, and reads after
+// it see what the counted writers wrote before theirs.
+__device__ __forceinline__ unsigned int atom_add_acq_rel_gpu(unsigned int* p, unsigned int v) {
+  unsigned int old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
 // ---------------------------------------------------------------- epoch-tagged counters
 // A counter that needs no clearing between launches: it holds (epoch << 32) | count, where the
 // epoch is unique to the launch (never 0), and a value left by another launch counts as 0.

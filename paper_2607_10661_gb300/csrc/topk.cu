@@ -471,18 +471,20 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
       if constexpr (kVerify) {
         // the last row of a tree to be written: this cluster verifies the tree
         int vb = -1;
+        __syncwarp();   // every lane's entries of this row are written before lane 0 counts the row
         if (lane == 0) {
           const int b = row_tree;
-          __threadfence();   // this row's top-k is visible before it is counted
           const int T = tin.T;
-          const int done = (int)atomicAdd(va.counters + b, 1u) + 1;
+          // release: this row's top-k before its count; acquire: the other rows' top-k (each
+          // written before its own count) before this cluster reads them
+          const int done = (int)atom_add_acq_rel_gpu(va.counters + b, 1u) + 1;
           if (done == T) vb = b;
         }
         vb = __shfl_sync(0xffffffffu, vb, 0);
         if (vb >= 0) {
           __shared__ vt::VerifyScratch vsc[1];
           __shared__ vt::TreeVerdict verdict[1];
-          __threadfence();   // every other row's top-k of the tree was counted after it was written
+          __syncwarp();   // lane 0's acquire precedes every lane's reads of the tree's rows
           vt::verify_tree_warp(tin, out_idx, k, vsc[0], &verdict[0]);
           __syncwarp();
           int len = verdict[0].len;
