@@ -512,6 +512,24 @@ def run_gpu(args, rank: int, world: int, dist):
 
     parts = Regions(dist, dev).run(parts_region)
     attn_ms = float(np.mean(attn_pairs))
+
+    # ---- the attention alone, K launches back to back on the stream (each placed by
+    # programmatic dependent launch while the one before drains): the roofline's second
+    # reading, with no timing event between launches
+    b2b_ms = float("nan")
+    if not extras:
+        def b2b_region():
+            j = turn[0] % n_graphs
+            turn[0] += 1
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for d in plan[j]:
+                d.attention()
+            b.record()
+            torch.cuda.synchronize()
+            return a.elapsed_time(b)
+
+        b2b_ms = Regions(dist, dev).run(b2b_region).median() / K
     lm_ms = float(np.mean([a.elapsed_time(b) for a, b in lm_evs])) if args.lm_head else None
     for d in copies:
         status |= int(d.dev_status.item())
@@ -525,7 +543,8 @@ def run_gpu(args, rank: int, world: int, dist):
     sampler.stop()
 
     ms_main, ms_eager, ms_parts = main.median(), eager.median(), parts.median()
-    ms_main, ms_eager, ms_parts, attn_ms = reduce_over_ranks(dist, [ms_main, ms_eager, ms_parts, attn_ms], dev)
+    ms_main, ms_eager, ms_parts, attn_ms, b2b_ms = reduce_over_ranks(
+        dist, [ms_main, ms_eager, ms_parts, attn_ms, b2b_ms], dev)
     hbm_peak, tf_peak, peak_kind = _peaks()
     ms_step = ms_main / K
     value = aggregate_rate(world, K, ms_main)
@@ -551,6 +570,13 @@ def run_gpu(args, rank: int, world: int, dist):
                  "timing": ("CUDA events recorded as graph nodes around every attention launch of the replayed "
                             "parts loop" if parts_graphs is not None else
                             "CUDA events around every attention launch of the eager parts loop")})
+    if b2b_ms == b2b_ms:   # the back-to-back reading (not NaN)
+        b2b_frac = ((flops / (b2b_ms * 1e-3) / 1e12) / tf_peak if tensor_bound else
+                    (nb["attention"] / (b2b_ms * 1e-3) / 1e9) / hbm_peak)
+        roof.update({"avg_launch_ms_back_to_back": round(b2b_ms, 5), "frac_back_to_back": round(b2b_frac, 4),
+                     "back_to_back_timing": f"{K} attention calls launched from the host back to back between "
+                                            "two CUDA events, divided by the launch count; median of the regions "
+                                            "(host-bound where a launch is shorter than the host's call)"})
     l2_note = (f"inputs larger than L2 ({nb['roofline'] / 1e9:.2f} GB read per step vs {l2 >> 20} MB L2)" if R == 1
                else f"{R} copies of every input rotated step by step ({R * nb['roofline'] / 1e6:.0f} MB in all vs "
                     f"{l2 >> 20} MB L2): no step finds its inputs in L2")
