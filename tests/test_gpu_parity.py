@@ -117,6 +117,27 @@ def test_attention_without_workspace_matches_oracle(case):
             _check_attn(got[l][w.nodes_of(b)], _attn_ref(w, l, b), w.cfg.dtype, f"{case} l{l} b{b}")
 
 
+@pytest.mark.parametrize("layers,ctx,launches", [
+    (12, 2000, 2),   # 96 units on 152 CTAs: pieces merged by the merge kernel, two column parts per unit
+    (4, 2000, 2),    # 32 units: four column parts per unit
+    (20, 1000, 1),   # 160 units: the last piece of each split unit merges inside the attention
+])
+def test_attention_merge_paths_match_oracle(layers, ctx, launches):
+    """Both merges of split units (in the attention kernel, or by the merge kernel with two or
+    four column parts per unit), every unit against the oracle."""
+    cfg = syn.shrink(syn.CONFIGS["llama3-8b-gqa"], layers=layers, ctx=(ctx, ctx), vocab=100)
+    w = syn.Workload(cfg, 23)
+    dw = DeviceWorkload(w, with_step_buffers=False)
+    n = dw.attention()
+    torch.cuda.synchronize()
+    assert int(dw.dev_status.item()) == 0
+    if torch.cuda.get_device_properties(0).multi_processor_count == 152:
+        assert n == launches
+    got = dw.attn_out.float().cpu().numpy()
+    for l in range(layers):
+        _check_attn(got[l][w.nodes_of(0)], _attn_ref(w, l, 0), cfg.dtype, f"layers {layers} l{l}")
+
+
 def test_attention_peaked_context_exposes_mask():
     """Committed-context keys made to score very low: outputs are dominated by the tree
     keys, so a wrongly (un)masked ancestor changes an output by O(1)."""
