@@ -413,6 +413,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool zero_tail = t0 + 128 > N;
         if (lane == 0) {
           const uint32_t dst = base + kOffRing + (uint32_t)st * kStageBytes;
+          // paged: the tile's page numbers, loaded together before the waits (K and V use the
+          // same pages), so that the copies do not each wait for their own block-table read
+          int phys[kPaged ? 8 : 1];
+          int nvalid = 0;
+          if (kPaged) {
+            const int ps = p.page_size;
+            const int first_page = t0 / ps;
+            nvalid = min(128 / ps, (N + ps - 1) / ps - first_page);
+            const int* bt = p.block_table + (size_t)b * p.max_pages + first_page;
+#pragma unroll
+            for (int pg = 0; pg < (kPaged ? 8 : 1); ++pg) phys[pg] = pg < nvalid ? bt[pg] : 0;
+          }
           for (int which = 0; which < 2 && ok; ++which) {
             ok = mbar_wait(which ? emptyv_bar(st) : emptyk_bar(st), ph ^ 1u, abort_flag, p.dev_status);
             if (ok) {
@@ -426,16 +438,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tma_load_3d_hint(d + kHalfBytes, map, fb, 64, hkv, row0, kv_policy);
               } else {
                 const int ps = p.page_size;
-                const int first_page = t0 / ps;
-                const int seq_pages = (N + ps - 1) / ps;
-                const int nvalid = min(128 / ps, seq_pages - first_page);
                 mbar_arrive_expect_tx(fb, (uint32_t)(nvalid * 2 * ps * 128));
-                for (int pg = 0; pg < nvalid; ++pg) {
-                  const int phys = p.block_table[(size_t)b * p.max_pages + first_page + pg];
-                  const int row0 = (layer * p.num_pages + phys) * ps;
-                  const uint32_t off = (uint32_t)(pg * ps * 128);
-                  tma_load_3d_hint(d + off, map, fb, 0, hkv, row0, kv_policy);
-                  tma_load_3d_hint(d + kHalfBytes + off, map, fb, 64, hkv, row0, kv_policy);
+#pragma unroll
+                for (int pg = 0; pg < (kPaged ? 8 : 1); ++pg) {
+                  if (pg < nvalid) {
+                    const int row0 = (layer * p.num_pages + phys[pg]) * ps;
+                    const uint32_t off = (uint32_t)(pg * ps * 128);
+                    tma_load_3d_hint(d + off, map, fb, 0, hkv, row0, kv_policy);
+                    tma_load_3d_hint(d + kHalfBytes + off, map, fb, 64, hkv, row0, kv_policy);
+                  }
                 }
               }
             }
