@@ -117,12 +117,17 @@ size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* ca
 
 /* Bytes of scratch the one-call step (ptd_tree_verify_step and the host-buffer and pipelined
  * steps built on it) wants as ptd_step_args.workspace: the attention's scratch
- * (ptd_attention_workspace_size, rounded up to 256 bytes) followed by one 4-byte counter per
- * tree (rounded up to 256 bytes).  With that much (and a bf16 cache), the top-k's CTAs also
- * verify every tree (the cluster that writes a tree's last row does it) and a copy kernel
- * compacts; with less, the top-k is followed by ptd_verify_and_compact, every CTA of which
- * verifies its tree before copying.  The scratch needs no clearing: the attention kernel
- * clears the tail's counters and tags its own with the launch.  0 for invalid arguments. */
+ * (ptd_attention_workspace_size, rounded up to 256 bytes) followed by the tail's: one 4-byte
+ * counter per tree and one per node row (together rounded up to 256 bytes), then one slot of
+ * 16 eight-byte keys per node row and two per SM of the current device (rounded up to 256
+ * bytes).  With that much (and a bf16 cache and bf16 logits whose rows start on 16 bytes,
+ * vocab a multiple of 8), a persistent top-k streams the rows back to back, one equal share
+ * per CTA, and also verifies every tree (the CTA that completes a tree's last row does it);
+ * a copy kernel compacts.  With the tree counters alone the clustered top-k (one cluster per
+ * row) verifies instead; with less, the top-k is followed by ptd_verify_and_compact, every
+ * CTA of which verifies its tree before copying.  The scratch needs no clearing: the
+ * attention kernel clears the tail's counters and tags its own with the launch.  0 for
+ * invalid arguments. */
 size_t ptd_step_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t num_q_heads);
 
 /* Tree-masked attention (Sec. 3.1 ancestor-only visibility; Sec. 3.2 one pass over
@@ -349,8 +354,8 @@ ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_str
  * Equivalent to ptd_tree_attention, ptd_topk_draft and ptd_verify_and_compact in that
  * order on `stream` (three launches, or four with the attention's merge kernel); when the
  * workspace holds ptd_step_workspace_size
- * bytes and the logits are bf16 with vocab <= 262143, the top-k's CTAs verify the trees
- * instead and the third launch only copies the accepted rows (node_offsets must then run
+ * bytes and the logits are bf16 (vocab a multiple of 8, or vocab <= 262143), the top-k's
+ * CTAs verify the trees instead and the third launch only copies the accepted rows (node_offsets must then run
  * from 0 to total_nodes without decreasing, as ptd_tree states; a tree with an empty or
  * out-of-range node range is reported as PTD_ERR_INVALID_TREE with accept_len 0, and when
  * the offsets decrease the outputs of the other trees are unspecified).  Each launch may be
@@ -380,6 +385,17 @@ typedef struct {
 
 ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
                                 const ptd_step_args* args, void* stream);
+
+/* Which top-k the one-call step (and the steps built on it) uses when its workspace allows
+ * both: AUTO streams the rows back to back when the clustered top-k (one cluster per row, at
+ * most three CTAs per SM) would take more than two waves of the device's SMs, and clusters
+ * otherwise (measured on GB300: 266 rows of 128256 logits stream faster, 128 rows of 152064
+ * and 63 or fewer rows of 128256 run faster clustered); CLUSTERED and STREAMED force one where
+ * it applies (streaming needs vocab a multiple of 8 and 16-byte aligned rows; clustering needs
+ * vocab <= 262143).  Process-wide; returns the previous policy, or -1 (nothing changed) for
+ * an unknown value.  Results are identical either way. */
+typedef enum { PTD_STEP_TOPK_AUTO = 0, PTD_STEP_TOPK_CLUSTERED = 1, PTD_STEP_TOPK_STREAMED = 2 } ptd_step_topk;
+int32_t ptd_step_topk_policy(int32_t policy);
 
 /* The same step fed from and drained to HOST memory (pinned for asynchronous copies):
  * copies the host inputs into the device buffers named by `tree`, `cache` and `args`,

@@ -126,8 +126,18 @@ size_t persistent_workspace_bytes(int units, int ctas, int head_dim) {
   return counters_bytes(units) + (size_t)2 * ctas * 256 * ((size_t)head_dim + 2) * sizeof(float);
 }
 
-// The step's tail counters (rows done per tree, epoch-tagged), after the attention's scratch.
+// The step's tail counters (rows done per tree, cleared by the attention's CTA 0), after the
+// attention's scratch.
 size_t tail_counters_bytes(int batch) { return ((size_t)batch * sizeof(unsigned int) + 255) / 256 * 256; }
+
+// The streaming top-k's tail: the counters per tree and per row (cleared together by the
+// attention's CTA 0), then its part slots.
+size_t stream_counters_bytes(int batch, int rows) {
+  return (((size_t)batch + (size_t)rows) * sizeof(unsigned int) + 255) / 256 * 256;
+}
+size_t stream_tail_bytes(int batch, int rows, int sms) {
+  return stream_counters_bytes(batch, rows) + (ptd::topk_stream_slot_bytes(rows, sms) + 255) / 256 * 256;
+}
 
 // Which schedule the shapes favour, from the host-known maxima (estimates in microseconds
 // measured on GB300 with these kernels): a key tile costs ~1.75 us for a unit of two 128-row
@@ -204,7 +214,7 @@ size_t ptd_attention_workspace_size(const ptd_tree* tree, const ptd_kv_cache* ca
 size_t ptd_step_workspace_size(const ptd_tree* tree, const ptd_kv_cache* cache, int32_t num_q_heads) {
   if (check_tree(tree) != PTD_OK || check_cache(cache) != PTD_OK) return 0;
   const size_t attn = ptd_attention_workspace_size(tree, cache, num_q_heads, cache->num_layers);
-  return (attn + 255) / 256 * 256 + tail_counters_bytes(tree->batch);
+  return (attn + 255) / 256 * 256 + stream_tail_bytes(tree->batch, tree->total_nodes, num_sms_of_current_device());
 }
 
 // ptd_tree_attention, and besides: the tensor-core kernel's CTA 0 clears zero_count words at
@@ -599,6 +609,15 @@ ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_str
   return st;
 }
 
+namespace {
+std::atomic<int> g_step_topk{PTD_STEP_TOPK_AUTO};
+}  // namespace
+
+int32_t ptd_step_topk_policy(int32_t policy) {
+  if (policy != PTD_STEP_TOPK_AUTO && policy != PTD_STEP_TOPK_CLUSTERED && policy != PTD_STEP_TOPK_STREAMED) return -1;
+  return g_step_topk.exchange(policy);
+}
+
 ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a,
                                 void* stream) {
   g_last_launches = 0;
@@ -618,16 +637,31 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
   // verification + compaction in one launch.  Each launch may be placed while the previous one
   // drains; it reads its inputs only after that one has completed (the top-k's logits come from
   // the step's forward pass).
+  // The streaming top-k needs rows back to back on 16-byte vectors and the whole tail of
+  // ptd_step_workspace_size; the clustered one only the per-tree counters.
   const size_t attn_ws = (ptd_attention_workspace_size(tree, cache, a->num_q_heads, cache->num_layers) + 255) /
                          256 * 256;
-  const bool fused = use_tensor_cores(cache) && a->logits_dtype == PTD_BF16 &&
-                     ptd::topk_can_verify(true, a->vocab) && a->workspace && aligned16(a->workspace) &&
-                     a->workspace_bytes >= attn_ws + tail_counters_bytes(tree->batch);
+  const int sms = num_sms_of_current_device();
+  const bool tail_ok = use_tensor_cores(cache) && a->logits_dtype == PTD_BF16 && a->workspace &&
+                       aligned16(a->workspace);
+  const bool can_stream = tail_ok && ptd::topk_stream_ok(a->logits, a->vocab) &&
+                          a->workspace_bytes >= attn_ws + stream_tail_bytes(tree->batch, tree->total_nodes, sms);
+  const bool can_cluster = tail_ok && ptd::topk_can_verify(true, a->vocab) &&
+                           a->workspace_bytes >= attn_ws + tail_counters_bytes(tree->batch);
+  const int policy = g_step_topk.load();
+  bool streamed = can_stream;
+  if (can_stream && can_cluster) {
+    const int64_t cluster_ctas = (int64_t)tree->total_nodes * ptd::topk_cluster_size(a->vocab);
+    streamed = policy == PTD_STEP_TOPK_STREAMED ||
+               (policy == PTD_STEP_TOPK_AUTO && cluster_ctas > 2 * 3 * (int64_t)sms);
+  }
+  const bool fused = streamed || can_cluster;
   unsigned int* tail_counters =
       fused ? reinterpret_cast<unsigned int*>(static_cast<uint8_t*>(a->workspace) + attn_ws) : nullptr;
+  const int zero_count = streamed ? tree->batch + tree->total_nodes : tree->batch;
   int total = 0;
   st = tree_attention(tree, cache, 0, cache->num_layers, a->q, a->num_q_heads, a->scale, a->attn_out, a->workspace,
-                      a->workspace_bytes, a->dev_status, tail_counters, tree->batch, stream);
+                      a->workspace_bytes, a->dev_status, tail_counters, zero_count, stream);
   if (st != PTD_OK) return st;
   total += g_last_launches;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -645,9 +679,16 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
     va.accept_len = a->accept_len;
     va.bonus = a->bonus_token;
     va.dev_status = a->dev_status;
-    if ((st = cuda_status(ptd::launch_topk(a->logits, true, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
-                                           a->topk_val, a->dev_status, &va, s))) != PTD_OK)
-      return st;
+    if (streamed) {
+      unsigned long long* slots = reinterpret_cast<unsigned long long*>(
+          static_cast<uint8_t*>(a->workspace) + attn_ws + stream_counters_bytes(tree->batch, tree->total_nodes));
+      st = cuda_status(ptd::launch_topk_stream(a->logits, tree->total_nodes, a->vocab, a->k, a->topk_idx, a->topk_val,
+                                               a->dev_status, va, tail_counters + tree->batch, slots, sms, s));
+    } else {
+      st = cuda_status(ptd::launch_topk(a->logits, true, tree->total_nodes, a->vocab, a->vocab, a->k, a->topk_idx,
+                                        a->topk_val, a->dev_status, &va, s));
+    }
+    if (st != PTD_OK) return st;
     const int row_bytes = cache->num_kv_heads * cache->head_dim * (int)dtype_size(cache->dtype);
     if ((st = cuda_status(ptd::launch_compact(cache->k, cache->v, row_bytes, cache->num_layers, tree->batch,
                                               cache->page_size, cache->seq_capacity, cache->num_pages,

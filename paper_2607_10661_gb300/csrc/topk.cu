@@ -235,6 +235,43 @@ __global__ void __launch_bounds__(kThreads) topk_cluster_kernel(const T* __restr
   }
 }
 
+// ------------------------------------------------------------------ the step's verification
+// Trees that no row can complete (an empty or out-of-range node range, or offsets that do not
+// run from 0 to n_total): their outputs and the status are written at once (one warp).
+__device__ __forceinline__ void flag_bad_trees_warp(const VerifyArgs& va) {
+  const int lane = threadIdx.x & 31;
+  for (int b = lane; b < va.batch; b += 32) {
+    const int n0 = va.node_offsets[b], n1 = va.node_offsets[b + 1];
+    const bool bad = n1 - n0 < 1 || n1 - n0 > va.max_nodes || n0 < 0 || n1 > va.n_total ||
+                     (b == 0 && n0 != 0) || (b == va.batch - 1 && n1 != va.n_total);
+    if (bad) {
+      for (int j = 0; j < va.max_nodes; ++j) va.accepted[(size_t)b * va.max_nodes + j] = -1;
+      va.accept_len[b] = 0;
+      va.bonus[b] = -1;
+      atomicMax(va.dev_status, (int)PTD_ERR_INVALID_TREE);
+    }
+  }
+}
+
+// Greedy verification of tree b on the calling warp, on column 0 of the top-k rows already
+// written (and made visible to this warp), and the tree's outputs.
+__device__ __forceinline__ void verify_and_write_warp(const VerifyArgs& va, int b, const vt::TreeInputs& tin,
+                                                      const int32_t* out_idx, int k, vt::VerifyScratch& sc,
+                                                      vt::TreeVerdict& vd) {
+  const int lane = threadIdx.x & 31;
+  vt::verify_tree_warp(tin, out_idx, k, sc, &vd);
+  __syncwarp();
+  int len = vd.len;
+  if (len > va.max_nodes) len = va.max_nodes;
+  int32_t* acc_row = va.accepted + (size_t)b * va.max_nodes;
+  for (int j = lane; j < va.max_nodes; j += 32) acc_row[j] = j < len ? vd.path[j] : -1;
+  if (lane == 0) {
+    va.accept_len[b] = len;
+    va.bonus[b] = vd.bonus;
+    if (vd.invalid) atomicMax(va.dev_status, (int)PTD_ERR_INVALID_TREE);
+  }
+}
+
 // ------------------------------------------------------------------ bf16 fast path
 // Each CTA stages its contiguous slice of the row (up to kSliceVec 16-byte vectors) into
 // shared memory with bulk asynchronous copies, so the row is read from HBM exactly once.
@@ -256,6 +293,13 @@ constexpr uint32_t kChunkBytes = 16384;    // bytes per bulk copy
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+// Lane-wise maximum of two bf16 pairs in one instruction (exact: a maximum only compares)
+__device__ __forceinline__ uint32_t bf16x2_max(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+constexpr uint32_t kBf16x2NegInf = 0xFF80FF80u;
 
 template <int KM, bool kVerify>
 __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16* __restrict__ logits,
@@ -297,19 +341,7 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
     // Trees that no row completes (an empty or out-of-range node range, or offsets that do not
     // run from 0 to n_total): their outputs and the status are written here, by warp 1 of the
     // first CTA, while its copy is in flight; a tree whose rows all arrive is verified below.
-    if (blockIdx.x == 0 && blockIdx.y == 0 && warp == 1) {
-      for (int b = lane; b < va.batch; b += 32) {
-        const int n0 = va.node_offsets[b], n1 = va.node_offsets[b + 1];
-        const bool bad = n1 - n0 < 1 || n1 - n0 > va.max_nodes || n0 < 0 || n1 > va.n_total ||
-                         (b == 0 && n0 != 0) || (b == va.batch - 1 && n1 != va.n_total);
-        if (bad) {
-          for (int j = 0; j < va.max_nodes; ++j) va.accepted[(size_t)b * va.max_nodes + j] = -1;
-          va.accept_len[b] = 0;
-          va.bonus[b] = -1;
-          atomicMax(va.dev_status, (int)PTD_ERR_INVALID_TREE);
-        }
-      }
-    }
+    if (blockIdx.x == 0 && blockIdx.y == 0 && warp == 1) flag_bad_trees_warp(va);
   }
   uint32_t phase = 0;
 
@@ -356,9 +388,9 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
       for (int i = a1; i < vocab; ++i) tmax = fmaxf(tmax, Vec<__nv_bfloat16>::scalar(row + i));
     mbar_wait(bar, phase, &abort_s, dev_status);   // bounded: a lost copy only flags PTD_ERR_TIMEOUT
 
-    // 1. lane maximum (four vectors in flight, two chains)
+    // 1. lane maximum (four vectors in flight, two chains of packed pair maxima)
     {
-      float t1 = -INFINITY;
+      uint32_t h0 = kBf16x2NegInf, h1 = kBf16x2NegInf;
       int v = tid;
       for (; v + 3 * kThreads < nv; v += 4 * kThreads) {
         uint4 x[4];
@@ -366,20 +398,17 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
         for (int u = 0; u < 4; ++u) x[u] = slice[v + u * kThreads];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          tmax = fmax3(tmax, bf16_lo(x[u].x), bf16_hi(x[u].x));
-          t1 = fmax3(t1, bf16_lo(x[u].y), bf16_hi(x[u].y));
-          tmax = fmax3(tmax, bf16_lo(x[u].z), bf16_hi(x[u].z));
-          t1 = fmax3(t1, bf16_lo(x[u].w), bf16_hi(x[u].w));
+          h0 = bf16x2_max(h0, bf16x2_max(x[u].x, x[u].y));
+          h1 = bf16x2_max(h1, bf16x2_max(x[u].z, x[u].w));
         }
       }
       for (; v < nv; v += kThreads) {
         const uint4 x = slice[v];
-        tmax = fmax3(tmax, bf16_lo(x.x), bf16_hi(x.x));
-        t1 = fmax3(t1, bf16_lo(x.y), bf16_hi(x.y));
-        tmax = fmax3(tmax, bf16_lo(x.z), bf16_hi(x.z));
-        t1 = fmax3(t1, bf16_lo(x.w), bf16_hi(x.w));
+        h0 = bf16x2_max(h0, bf16x2_max(x.x, x.y));
+        h1 = bf16x2_max(h1, bf16x2_max(x.z, x.w));
       }
-      tmax = fmaxf(tmax, t1);
+      h0 = bf16x2_max(h0, h1);
+      tmax = fmax3(tmax, bf16_lo(h0), bf16_hi(h0));
     }
     const bool has_elems = tid < nv || (own_head && a0 > 0) || (own_tail && a1 < vocab);
 
@@ -404,13 +433,12 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
         const float f = Vec<__nv_bfloat16>::scalar(row + i);
         if (f >= thr) list.push(ordered_bits(f), (uint32_t)i);
       }
-    for (int v = tid; v < nv; v += kThreads) {
-      const uint4 x = slice[v];
-      float vm = fmax3(bf16_lo(x.x), bf16_hi(x.x), bf16_lo(x.y));
-      vm = fmax3(vm, bf16_hi(x.y), bf16_lo(x.z));
-      vm = fmax3(vm, bf16_hi(x.z), bf16_lo(x.w));
-      vm = fmaxf(vm, bf16_hi(x.w));
-      if (vm >= thr) {
+    {
+      auto vec_max = [](const uint4& x) {
+        const uint32_t h = bf16x2_max(bf16x2_max(x.x, x.y), bf16x2_max(x.z, x.w));
+        return fmaxf(bf16_lo(h), bf16_hi(h));
+      };
+      auto push_vec = [&](const uint4& x, int v) {
         const uint32_t gi = (uint32_t)(a0 + (v_begin + v) * 8);
         const uint32_t w[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
@@ -419,6 +447,25 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
           if (f0 >= thr) list.push(ordered_bits(f0), gi + 2 * q);
           if (f1 >= thr) list.push(ordered_bits(f1), gi + 2 * q + 1);
         }
+      };
+      // four vectors in flight; the few that reach T_w are read again and pushed, in index order
+      int v = tid;
+      for (; v + 3 * kThreads < nv; v += 4 * kThreads) {
+        uint4 x[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) x[u] = slice[v + u * kThreads];
+        uint32_t hits = 0u;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) hits |= (vec_max(x[u]) >= thr ? 1u : 0u) << u;
+#pragma unroll 1
+        for (; hits != 0u; hits &= hits - 1u) {   // rare: read the vector again
+          const int vu = v + (__ffs(hits) - 1) * kThreads;
+          push_vec(slice[vu], vu);
+        }
+      }
+      for (; v < nv; v += kThreads) {
+        const uint4 x = slice[v];
+        if (vec_max(x) >= thr) push_vec(x, v);
       }
     }
     if (own_tail)
@@ -485,22 +532,335 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
           __shared__ vt::VerifyScratch vsc[1];
           __shared__ vt::TreeVerdict verdict[1];
           __syncwarp();   // lane 0's acquire precedes every lane's reads of the tree's rows
-          vt::verify_tree_warp(tin, out_idx, k, vsc[0], &verdict[0]);
-          __syncwarp();
-          int len = verdict[0].len;
-          if (len > va.max_nodes) len = va.max_nodes;
-          int32_t* acc_row = va.accepted + (size_t)vb * va.max_nodes;
-          for (int j = lane; j < va.max_nodes; j += 32) acc_row[j] = j < len ? verdict[0].path[j] : -1;
-          if (lane == 0) {
-            va.accept_len[vb] = len;
-            va.bonus[vb] = verdict[0].bonus;
-            if (verdict[0].invalid) atomicMax(va.dev_status, (int)PTD_ERR_INVALID_TREE);
-          }
+          verify_and_write_warp(va, vb, tin, out_idx, k, vsc[0], verdict[0]);
         }
       }
     }
     cluster.sync();   // keep every CTA's shared memory alive until rank 0 has read it
   }
+}
+
+// ------------------------------------------------------------------ streaming top-k of the step
+// The step's rows (its trees' nodes) lie back to back in memory: as one sequence of 16-byte
+// vectors (8 logits), CTA c of a persistent grid takes vectors [c L, (c + 1) L) of it, so every
+// CTA moves the same number of bytes however many rows there are.  One producer warp streams
+// the CTA's range through a ring of shared-memory chunks (bulk copies, one mbarrier pair per
+// stage); copy and selection overlap across row boundaries and the grid never waits between
+// waves.  The piece of a row that falls in one CTA's range (a row part) is selected by the 8
+// selection warps as in the clustered kernel: T_w is taken on the part's first chunk (every
+// lane's maximum over its vectors of that chunk; the k lanes holding the k largest maxima own
+// k elements >= T_w), each lane keeps its elements >= T_w of the whole part in an exact sorted
+// list, and at the part's end the warps' lists are merged into the part's top-k, which goes to
+// a global slot.  The part that completes its row (a per-row counter) merges the row's slots
+// and writes the row; the row that completes its tree (a per-tree counter) has the tree
+// verified on the same warp.  The part ends (the CTA merge, the global slot, the counters, a
+// row's merge and a tree's verification: a chain of L2 round trips) run on a merge warp of
+// their own, fed through a double buffer of the selection warps' keys, so that the stream
+// never waits for them.  Counters are cleared by the launch before this one (the step's
+// attention); slots are written before they are read within the launch.
+// The k-th largest of the warp's 32 order-preserving values (0 = a lane without one), or 0 when
+// fewer than k lanes hold one: one warp maximum and one ballot per distinct value, equal values
+// counted together.  Any x with k elements >= x bounds the warp's top-k from below.
+__device__ __forceinline__ uint32_t kth_largest_ord(uint32_t v, int k) {
+  int count = 0;
+  for (int s = 0; s < k; ++s) {
+    const uint32_t m = __reduce_max_sync(0xffffffffu, v);
+    if (m == 0u) return 0u;
+    count += __popc(__ballot_sync(0xffffffffu, v == m));
+    if (count >= k) return m;
+    if (v == m) v = 0u;
+  }
+  return 0u;
+}
+
+constexpr int kSelWarps = 8;
+constexpr int kSelThreads = kSelWarps * 32;
+constexpr int kProducerWarp = kSelWarps;
+constexpr int kMergeWarp = kSelWarps + 1;
+constexpr int kStreamThreads = kSelThreads + 64;   // + the producer and merge warps
+constexpr int kStreamStages = 6;
+constexpr int kStreamChunkVec = 1024;              // 16 KB of logits per chunk
+constexpr int kStreamMinVec = 2048;                // at least 32 KB per CTA
+constexpr int kPartSlot = 16;                      // keys per part slot (the largest k)
+constexpr int kCachedOffsets = 257;                // trees whose node offsets sit in shared memory
+constexpr int kRaiseAfter = 8;                     // new candidate lanes before T_w is raised
+
+struct StreamArgs {
+  const __nv_bfloat16* logits;      // [rows][nvec_row * 8], back to back, 16-byte aligned
+  int64_t rows;
+  int nvec_row;
+  int k;
+  int64_t total_vec, per_cta;       // rows * nvec_row; vectors per CTA (the last may have fewer)
+  int32_t* out_idx;                 // [rows][k]
+  float* out_val;                   // [rows][k]
+  unsigned int* row_counters;       // [rows], zero before the launch
+  unsigned long long* part_keys;    // [(rows + gridDim.x) * kPartSlot]: slot of row r in CTA c = r + c
+  int32_t* dev_status;
+};
+
+template <int KM>
+__global__ void __launch_bounds__(kStreamThreads, 2) topk_stream_kernel(const StreamArgs a, const VerifyArgs va) {
+  extern __shared__ __align__(128) uint4 ring[];
+  __shared__ __align__(8) uint64_t bars_s[2 * kStreamStages + 4];
+  __shared__ uint64_t warp_keys[2][kSelWarps][KM];
+  __shared__ int offsets_s[kCachedOffsets];
+  __shared__ int abort_s;
+  __shared__ vt::VerifyScratch vsc;
+  __shared__ vt::TreeVerdict verdict;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t full0 = smem_u32(&bars_s[0]), empty0 = smem_u32(&bars_s[kStreamStages]);
+  auto full_bar = [&](int st) { return full0 + 8u * (uint32_t)st; };
+  auto empty_bar = [&](int st) { return empty0 + 8u * (uint32_t)st; };
+  // the selection warps' keys of a part: buffer pb full (8 warps) / empty (the merge warp)
+  auto kfull_bar = [&](int pb) { return smem_u32(&bars_s[2 * kStreamStages + pb]); };
+  auto kempty_bar = [&](int pb) { return smem_u32(&bars_s[2 * kStreamStages + 2 + pb]); };
+  if (threadIdx.x == 0) {
+    for (int st = 0; st < kStreamStages; ++st) {
+      mbar_init(full_bar(st), 1);
+      mbar_init(empty_bar(st), kSelWarps);
+    }
+    for (int pb = 0; pb < 2; ++pb) {
+      mbar_init(kfull_bar(pb), kSelWarps);
+      mbar_init(kempty_bar(pb), 1);
+    }
+    abort_s = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) grid_launch_dependents();   // the next grid may be placed now; it waits for this one
+  const int64_t vbeg = (int64_t)blockIdx.x * a.per_cta;
+  const int64_t vend = vbeg + a.per_cta < a.total_vec ? vbeg + a.per_cta : a.total_vec;
+  const int nvr = a.nvec_row;
+  // the chunk at vector position pos: its row, offset in the row and length (never across a row)
+  auto chunk_at = [&](int64_t pos, int64_t& row, int& off, int& n) {
+    row = pos / nvr;
+    off = (int)(pos - row * nvr);
+    int64_t m = vend - pos;
+    if (m > kStreamChunkVec) m = kStreamChunkVec;
+    if (m > nvr - off) m = nvr - off;
+    n = (int)m;
+  };
+  grid_dependency_wait();   // the logits, the trees and the outputs belong to the stream's previous work
+
+  if (warp == kProducerWarp) {
+    // ================================================================ producer (one lane)
+    if (lane == 0) {
+      bool ok = true;
+      int j = 0;
+      for (int64_t pos = vbeg; pos < vend; ++j) {
+        int64_t row;
+        int off, n;
+        chunk_at(pos, row, off, n);
+        const int st = j % kStreamStages;
+        ok = mbar_wait(empty_bar(st), (uint32_t)(((j / kStreamStages) & 1) ^ 1), &abort_s, a.dev_status);
+        if (!ok) break;
+        // (the selection warps only read the stage: their arrivals on its empty barrier order
+        // those reads before this copy; no proxy fence, which would also wait for the copies
+        // still in flight)
+        mbar_arrive_expect_tx(full_bar(st), (uint32_t)n * 16u);
+        bulk_load(smem_u32(ring) + (uint32_t)st * (kStreamChunkVec * 16u),
+                  reinterpret_cast<const uint4*>(a.logits) + pos, (uint32_t)n * 16u, full_bar(st));
+        pos += n;
+      }
+      if (!ok) {
+        // drain the copies already issued (bounded) before the CTA can exit
+        for (int back = 1; back <= kStreamStages && j - back >= 0; ++back) {
+          const int j2 = j - back;
+          mbar_drain(full_bar(j2 % kStreamStages), (uint32_t)((j2 / kStreamStages) & 1), 100000000ull);
+        }
+      }
+    }
+    return;
+  }
+
+  const int k = a.k;
+  if (warp == kMergeWarp) {
+    // ================================================================ merge warp
+    const bool cached = va.batch + 1 <= kCachedOffsets;
+    if (cached)
+      for (int i = lane; i <= va.batch; i += 32) offsets_s[i] = va.node_offsets[i];
+    if (blockIdx.x == 0) flag_bad_trees_warp(va);
+    __syncwarp();
+    auto tree_of = [&](int64_t r) {
+      int lo = 0, hi = va.batch;
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if ((cached ? offsets_s[mid] : va.node_offsets[mid]) <= r) lo = mid; else hi = mid;
+      }
+      return lo;
+    };
+    int part = 0;
+    for (int64_t pos = vbeg; pos < vend;) {
+      int64_t row;
+      int off, n;
+      chunk_at(pos, row, off, n);
+      pos += n;
+      if (!(pos == vend || off + n == nvr)) continue;   // not the end of a row part
+      const int pb = part & 1;
+      if (!mbar_wait_warp(kfull_bar(pb), (uint32_t)((part >> 1) & 1), &abort_s, a.dev_status)) break;
+      // the CTA's top-k of the part: lane w (< 8) owns warp w's sorted keys
+      int cur = 0;
+      uint64_t pk = 0ull;
+      for (int s = 0; s < k; ++s) {
+        const uint64_t mine = (lane < kSelWarps && cur < k) ? warp_keys[pb][lane][cur] : 0ull;
+        const uint64_t best = warp_max_u64(mine);
+        if (lane < kSelWarps && mine == best && best != 0ull) ++cur;
+        if (lane == s) pk = best;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(kempty_bar(pb));   // the buffer is read (the keys are in registers)
+      ++part;
+      const int64_t c_first = row * nvr / a.per_cta;
+      int64_t c_last = ((row + 1) * nvr - 1) / a.per_cta;
+      if (c_last > (int64_t)gridDim.x - 1) c_last = gridDim.x - 1;
+      const int nparts = (int)(c_last - c_first + 1);
+      int last_part = 1;   // a row that lies in this CTA alone has the part's top-k
+      if (nparts > 1) {
+        if (lane < k) a.part_keys[(size_t)(row + blockIdx.x) * kPartSlot + lane] = pk;
+        __syncwarp();   // every lane's key of this part is written before lane 0 counts the part
+        if (lane == 0) last_part = (int)atom_add_acq_rel_gpu(a.row_counters + row, 1u) + 1 == nparts;
+        last_part = __shfl_sync(0xffffffffu, last_part, 0);
+      }
+      if (!last_part) continue;
+      if (nparts > 1) {
+        // the row's top-k from its parts' slots (each written before its part was counted)
+        ThreadList<KM> ml;
+        ml.init();
+        __syncwarp();   // lane 0's acquire precedes every lane's reads of the slots
+        for (int q = lane; q < nparts * k; q += 32) {
+          const uint64_t key = __ldcg(a.part_keys + (size_t)(row + c_first + q / k) * kPartSlot + q % k);
+          if (key != 0ull) ml.push_key(key);
+        }
+        pk = 0ull;
+        for (int s = 0; s < k; ++s) {
+          const uint64_t mine = ml.head();
+          const uint64_t best = warp_max_u64(mine);
+          if (mine == best && best != 0ull) ml.pop();
+          if (lane == s) pk = best;
+        }
+      }
+      if (lane < k) {
+        a.out_idx[row * k + lane] = (int32_t)(~(uint32_t)(pk & 0xFFFFFFFFull));
+        a.out_val[row * k + lane] = from_ordered((uint32_t)(pk >> 32));
+      }
+      // count the row for its tree; the tree's last row verifies it (its parents and tokens
+      // are loaded while the count is in flight)
+      const int b = tree_of(row);
+      vt::TreeInputs tin;
+      vt::load_tree_warp(va.node_offsets, va.parents, va.tokens, va.n_total, va.max_nodes, b, tin);
+      int vb = -1;
+      __syncwarp();   // every lane's entries of this row are written before lane 0 counts the row
+      if (lane == 0) {
+        // release: this row's top-k before its count; acquire: the other rows' top-k (each
+        // written before its own count) before this warp reads them
+        if ((int)atom_add_acq_rel_gpu(va.counters + b, 1u) + 1 == tin.T) vb = b;
+      }
+      vb = __shfl_sync(0xffffffffu, vb, 0);
+      if (vb >= 0) {
+        __syncwarp();   // lane 0's acquire precedes every lane's reads of the tree's rows
+        verify_and_write_warp(va, vb, tin, a.out_idx, k, vsc, verdict);
+      }
+    }
+    return;
+  }
+
+  // ================================================================ selection warps
+  const int tid = threadIdx.x;
+  ThreadList<KM> list;
+  list.init();
+  float thr = -INFINITY;
+  int fresh = 0;   // lanes that pushed since T_w was last set (summed over chunks)
+  int part = 0;
+  // After a failed wait (timeout, or another warp's) a warp stops reading; the others and the
+  // merge warp see the abort flag within their own bounded waits.
+  int j = 0;
+  for (int64_t pos = vbeg; pos < vend; ++j) {
+    int64_t row;
+    int off, n;
+    chunk_at(pos, row, off, n);
+    const bool first = pos == vbeg || off == 0;
+    const bool last = pos + n == vend || off + n == nvr;
+    const int st = j % kStreamStages;
+    if (!mbar_wait_warp(full_bar(st), (uint32_t)((j / kStreamStages) & 1), &abort_s, a.dev_status)) break;
+    const uint4* chunk = ring + (size_t)st * kStreamChunkVec;
+    uint32_t hv[4];   // per vector: the packed maximum of its four pairs
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int vi = tid + u * kSelThreads;
+      const uint4 x = vi < n ? chunk[vi] : make_uint4(kBf16x2NegInf, kBf16x2NegInf, kBf16x2NegInf, kBf16x2NegInf);
+      hv[u] = bf16x2_max(bf16x2_max(x.x, x.y), bf16x2_max(x.z, x.w));
+    }
+    if (first) {
+      // a new row part: T_w from this chunk (lanes without a vector here hold no element)
+      list.init();
+      fresh = 0;
+      const uint32_t h = bf16x2_max(bf16x2_max(hv[0], hv[1]), bf16x2_max(hv[2], hv[3]));
+      const uint32_t kth = kth_largest_ord(tid < n ? ordered_bits(fmaxf(bf16_lo(h), bf16_hi(h))) : 0u, k);
+      thr = kth != 0u ? from_ordered(kth) : -INFINITY;
+    }
+    uint32_t hits = 0u;
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      hits |= (tid + u * kSelThreads < n && fmaxf(bf16_lo(hv[u]), bf16_hi(hv[u])) >= thr ? 1u : 0u) << u;
+    // the few vectors that reach the threshold: read again and pushed, in index order
+    fresh += __popc(__ballot_sync(0xffffffffu, hits != 0u));
+#pragma unroll 1
+    for (; hits != 0u; hits &= hits - 1u) {
+      const int vi = tid + (__ffs(hits) - 1) * kSelThreads;
+      const uint4 x = chunk[vi];
+      const uint32_t gi = (uint32_t)(off + vi) * 8u;
+      const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float f0 = bf16_lo(w[q]), f1 = bf16_hi(w[q]);
+        if (f0 >= thr) list.push(ordered_bits(f0), gi + 2 * q);
+        if (f1 >= thr) list.push(ordered_bits(f1), gi + 2 * q + 1);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty_bar(st));   // this warp is done with the stage
+    if (!last && fresh >= kRaiseAfter) {
+      // raise T_w once enough new candidates came in: if k lanes hold candidates >= x, no
+      // element below x is among the warp's top-k; x = the k-th largest of the lanes' largest
+      fresh = 0;
+      const uint32_t kth = kth_largest_ord(list.ord[0], k);
+      if (kth != 0u) thr = fmaxf(thr, from_ordered(kth));
+    }
+    pos += n;
+    if (!last) continue;
+    // ---- the end of a row part: the warp's top-k into buffer part % 2 (free once the merge
+    // warp has read the part two before this one)
+    const int pb = part & 1;
+    if (!mbar_wait_warp(kempty_bar(pb), (uint32_t)(((part >> 1) & 1) ^ 1), &abort_s, a.dev_status)) break;
+    for (int s = 0; s < k; ++s) {
+      const uint64_t mine = list.head();
+      const uint64_t best = warp_max_u64(mine);
+      if (mine == best) list.pop();
+      if (lane == 0) warp_keys[pb][warp][s] = best;
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(kfull_bar(pb));
+    ++part;
+  }
+}
+
+template <int KM>
+cudaError_t launch_stream_km(const StreamArgs& a, int grid, const VerifyArgs& va, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);
+  cfg.blockDim = dim3(kStreamThreads, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)kStreamStages * kStreamChunkVec * 16;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // set-up overlaps the previous kernel
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaFuncSetAttribute(topk_stream_kernel<KM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)cfg.dynamicSmemBytes);
+  if (e != cudaSuccess) return e;
+  return cudaLaunchKernelEx(&cfg, topk_stream_kernel<KM>, a, va);
 }
 
 template <int KM, typename T, bool kFast, bool kVerify>
@@ -560,6 +920,49 @@ cudaError_t launch_t(const T* logits, int64_t rows, int vocab, int64_t row_strid
 }
 
 }  // namespace topk
+
+bool topk_stream_ok(const void* logits, int vocab) {
+  return vocab >= 8 && vocab % 8 == 0 && (reinterpret_cast<uintptr_t>(logits) & 15u) == 0;
+}
+
+size_t topk_stream_slot_bytes(int64_t rows, int sms) {
+  return (size_t)(rows + 2 * (int64_t)sms) * topk::kPartSlot * sizeof(unsigned long long);
+}
+
+cudaError_t launch_topk_stream(const void* logits, int64_t rows, int vocab, int k, int32_t* out_idx, float* out_val,
+                               int32_t* dev_status, const VerifyArgs& va, unsigned int* row_counters,
+                               unsigned long long* part_keys, int sms, cudaStream_t stream) {
+  if (!topk_stream_ok(logits, vocab) || rows < 1 || k < 1 || k > topk::kPartSlot || sms < 1)
+    return cudaErrorInvalidValue;
+  topk::StreamArgs a = {};
+  a.logits = static_cast<const __nv_bfloat16*>(logits);
+  a.rows = rows;
+  a.nvec_row = vocab / 8;
+  a.k = k;
+  a.total_vec = rows * (int64_t)a.nvec_row;
+  // two CTAs per SM, each with at least kStreamMinVec vectors; equal ranges
+  int64_t grid = (a.total_vec + topk::kStreamMinVec - 1) / topk::kStreamMinVec;
+  if (grid > 2 * (int64_t)sms) grid = 2 * (int64_t)sms;
+  if (grid < 1) grid = 1;
+  a.per_cta = (a.total_vec + grid - 1) / grid;
+  grid = (a.total_vec + a.per_cta - 1) / a.per_cta;
+  a.out_idx = out_idx;
+  a.out_val = out_val;
+  a.row_counters = row_counters;
+  a.part_keys = part_keys;
+  a.dev_status = dev_status;
+  if (k <= 1) return topk::launch_stream_km<1>(a, (int)grid, va, stream);
+  if (k <= 2) return topk::launch_stream_km<2>(a, (int)grid, va, stream);
+  if (k <= 4) return topk::launch_stream_km<4>(a, (int)grid, va, stream);
+  if (k <= 8) return topk::launch_stream_km<8>(a, (int)grid, va, stream);
+  return topk::launch_stream_km<16>(a, (int)grid, va, stream);
+}
+
+int topk_cluster_size(int vocab) {
+  const int nvec = vocab / 8 + 1;
+  int cluster = (nvec + topk::kSliceVec - 1) / topk::kSliceVec;
+  return cluster < 1 ? 1 : (cluster > topk::kMaxCluster ? topk::kMaxCluster : cluster);
+}
 
 bool topk_can_verify(bool bf16, int vocab) {
   return bf16 && (int64_t)vocab / 8 + 1 <= (int64_t)topk::kMaxCluster * topk::kSliceVec;

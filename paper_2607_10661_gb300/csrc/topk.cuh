@@ -2,6 +2,7 @@
 #pragma once
 #include <cuda_runtime.h>
 
+#include <cstddef>
 #include <cstdint>
 
 namespace ptd {
@@ -19,6 +20,19 @@ struct VerifyArgs {
   int32_t* bonus;                // [batch]
   int32_t* dev_status;
 };
+
+// The step's streaming top-k with verification (bf16 rows back to back, vocab a multiple of 8,
+// logits 16-byte aligned): a persistent grid of at most 2 * sms CTAs, each over an equal share
+// of the rows' bytes.  row_counters [rows] (and va.counters) must be zero before the launch;
+// part_keys holds topk_stream_slot_bytes(rows, sms) bytes of scratch (no clearing needed).
+bool topk_stream_ok(const void* logits, int vocab);
+size_t topk_stream_slot_bytes(int64_t rows, int sms);
+cudaError_t launch_topk_stream(const void* logits, int64_t rows, int vocab, int k, int32_t* out_idx, float* out_val,
+                               int32_t* dev_status, const VerifyArgs& va, unsigned int* row_counters,
+                               unsigned long long* part_keys, int sms, cudaStream_t stream);
+
+// CTAs per row of the clustered bf16 top-k (one cluster per row).
+int topk_cluster_size(int vocab);
 
 // Whether launch_topk can verify for these logits (bf16 rows within the clustered fast path).
 bool topk_can_verify(bool bf16, int vocab);

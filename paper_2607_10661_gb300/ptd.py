@@ -31,7 +31,7 @@ EXPORTED = (
     "ptd_draft_tree_update", "ptd_pool_bytes", "ptd_pool_init", "ptd_pool_merge", "ptd_pool_retrieve",
     "ptd_tree_rope_append", "ptd_lm_head_topk_workspace_size", "ptd_lm_head_topk", "ptd_pipeline_create",
     "ptd_pipeline_submit", "ptd_pipeline_wait", "ptd_pipeline_destroy", "ptd_check_bounded_wait",
-    "ptd_step_workspace_size",
+    "ptd_step_workspace_size", "ptd_step_topk_policy",
 )
 
 
@@ -86,6 +86,8 @@ def lib() -> ctypes.CDLL:
         L.ptd_status_string.argtypes = [ctypes.c_int]
         L.ptd_last_launch_count.restype = i32
         L.ptd_last_launch_count.argtypes = []
+        L.ptd_step_topk_policy.restype = i32
+        L.ptd_step_topk_policy.argtypes = [i32]
         L.ptd_attention_workspace_size.restype = sz
         L.ptd_attention_workspace_size.argtypes = [P(_Tree), P(_Cache), i32, i32]
         L.ptd_step_workspace_size.restype = sz
@@ -141,6 +143,17 @@ def lib() -> ctypes.CDLL:
 
 def status_string(status: int) -> str:
     return lib().ptd_status_string(int(status)).decode()
+
+
+STEP_TOPK_AUTO, STEP_TOPK_CLUSTERED, STEP_TOPK_STREAMED = 0, 1, 2
+
+
+def step_topk_policy(policy: int) -> int:
+    """ptd_step_topk_policy: which top-k the one-call step uses (process-wide); returns the previous one."""
+    prev = int(lib().ptd_step_topk_policy(int(policy)))
+    if prev < 0:
+        raise ValueError(f"unknown step top-k policy {policy}")
+    return prev
 
 
 def last_launch_count() -> int:

@@ -253,3 +253,19 @@ def test_host_step_rejects_a_tree_above_max_nodes(lib):
     _, c, a = _step_structs(ptd)
     assert lib.ptd_tree_verify_step_host(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a), ctypes.byref(io),
                                          None) == ptd.INVALID_ARG
+
+
+def test_step_topk_policy_round_trip(lib):
+    """ptd_step_topk_policy (host only): each known policy is taken and the previous one is
+    returned; an unknown one changes nothing and returns -1."""
+    lib.ptd_step_topk_policy.restype = ctypes.c_int32
+    lib.ptd_step_topk_policy.argtypes = [ctypes.c_int32]
+    start = lib.ptd_step_topk_policy(0)
+    try:
+        assert lib.ptd_step_topk_policy(2) == 0
+        assert lib.ptd_step_topk_policy(1) == 2
+        assert lib.ptd_step_topk_policy(7) == -1
+        assert lib.ptd_step_topk_policy(-1) == -1
+        assert lib.ptd_step_topk_policy(0) == 1
+    finally:
+        lib.ptd_step_topk_policy(start)

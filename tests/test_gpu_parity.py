@@ -826,3 +826,117 @@ def test_step_fused_tail_equals_three_launch_tail(base, over, seed):
         else:
             assert torch.equal(a[key], b[key]), key
     assert int(a["alen"].max()) > 2
+
+
+# ------------------------------------------------------------------------------ streamed top-k of the step
+
+# With the step's workspace and bf16 rows of a multiple of 8 logits, the step's top-k is the
+# persistent streaming kernel: the rows back to back, one equal share per CTA, so a row is cut
+# into parts that end in different CTAs and meet in a merge by the part that completes it.
+STREAM_CASES = {
+    # one row of 128256 logits in eight CTAs
+    "one-row": ("llama3-8b-gqa", dict(layers=1, ctx=(64, 64), tree="chain", nodes=(1, 1)), 91),
+    # three rows, CTA shares crossing the row boundaries
+    "three-rows": ("llama3-8b-gqa", dict(layers=1, ctx=(64, 64), tree="chain", nodes=(3, 3)), 92),
+    # forty trees of 1-16 nodes with 1000 logits a row: several rows in one CTA's share
+    "many-short-rows": ("batched-paged", dict(batch=40, ctx=(16, 200), nodes=(1, 16), depth_range=(1, 4),
+                                              vocab=1000, hq=8, hkv=2), 93),
+    # 128 rows of 152064 logits, k = 6
+    "long-context-rows": ("long-context", dict(layers=1, ctx=(200, 200)), 94),
+    # eight trees of 16-64 nodes, 128256 logits a row (the batched workload's rows)
+    "batched-rows": ("batched-paged", dict(ctx=(64, 300)), 97),
+    # the largest k, and k = 1
+    "k16": ("batched-paged", dict(batch=3, ctx=(64, 200), vocab=20000, k=16, hq=8, hkv=2), 95),
+    "k1": ("llama3-8b-gqa", dict(layers=1, ctx=(64, 64), vocab=4096, k=1), 96),
+}
+
+
+def _plant_ties(w):
+    """Every other row gets four equal maxima (one at each end, two adjacent in the middle,
+    which straddle a CTA boundary in the one-row case); returns the bf16 bit patterns."""
+    logits = w.logits.copy()
+    f = syn.bf16_to_f32(logits)
+    V = w.cfg.vocab
+    cols = [5, V // 2 - 1, V // 2, V - 1]
+    for r in range(0, logits.shape[0], 2):
+        top = syn.bf16_bits(np.array([f[r].max() + 1.0], np.float32))[0]
+        logits[r, cols] = top
+    return logits
+
+
+def _tree_counter_workspace(dw, cfg):
+    """The attention's scratch and the per-tree counters only: the step's clustered top-k."""
+    small = ptd.attention_workspace_size(dw.tree, dw.cache, cfg.hq)
+    return (small + 255) // 256 * 256 + (4 * cfg.batch + 255) // 256 * 256
+
+
+@pytest.mark.parametrize("case", list(STREAM_CASES))
+def test_step_streamed_topk_matches_oracle(case):
+    """Every top-k row (indices and values, ties to the lower index across CTA parts), every
+    verified path and the compacted caches equal the oracle's, with the streamed top-k forced,
+    with the clustered one forced, and with the clustered one chosen by a workspace that holds
+    only the per-tree counters: identical outputs all three ways."""
+    base, over, seed = STREAM_CASES[case]
+    cfg = syn.shrink(syn.CONFIGS[base], **over)
+    outs = []
+    for kind in ("streamed", "clustered", "tree-counters"):
+        w = syn.Workload(cfg, seed)
+        dw = DeviceWorkload(w)
+        logits = _plant_ties(w)
+        dw.logits.copy_(to_torch(logits, cfg.dtype))
+        if kind == "tree-counters":
+            ws = torch.empty(_tree_counter_workspace(dw, cfg), dtype=torch.uint8, device="cuda")
+            dw.bufs = ptd.StepBuffers(dw.q, cfg.hq, dw.attn_out, dw.logits, cfg.k, dw.tokens, dw.topk_idx,
+                                      dw.topk_val, dw.accepted, dw.accept_len, dw.bonus, dw.new_ctx, dw.dev_status,
+                                      ws)
+        prev = ptd.step_topk_policy(ptd.STEP_TOPK_CLUSTERED if kind == "clustered" else ptd.STEP_TOPK_STREAMED)
+        idx_ref, val_ref = oracle.topk_rows(syn.bf16_to_f32(logits), cfg.k)
+        greedy = idx_ref[:, 0]
+        rng = np.random.default_rng(seed)
+        tokens = w.tokens.copy()
+        for b, par in enumerate(w.trees):
+            o = int(w.node_offsets[b])
+            for i in range(1, len(par)):
+                tokens[o + i] = greedy[o + par[i]] if rng.random() < 0.8 else int(rng.integers(cfg.vocab))
+        dw.tokens.copy_(torch.tensor(tokens, dtype=torch.int32))
+        k_before = dw.k.cpu().view(torch.int16).numpy()
+        try:
+            launches = dw.step()
+            torch.cuda.synchronize()
+        finally:
+            ptd.step_topk_policy(prev)
+        assert launches in (3, 4)
+        assert int(dw.dev_status.item()) == 0
+        assert np.array_equal(dw.topk_idx.cpu().numpy(), idx_ref)
+        assert np.array_equal(dw.topk_val.cpu().numpy(), val_ref.astype(np.float32))
+        ka = dw.k.cpu().view(torch.int16).numpy()
+        for b, par in enumerate(w.trees):
+            sl = w.nodes_of(b)
+            path, nacc, bonus = oracle.verify_greedy(par, tokens[sl], greedy[sl])
+            assert int(dw.accept_len[b]) == nacc and int(dw.bonus[b]) == bonus
+            acc = dw.accepted[b].cpu().tolist()
+            assert acc[:nacc] == path and all(x == -1 for x in acc[nacc:])
+            for l in range(cfg.layers):
+                ref, new_ctx = oracle.kv_compact(w.seq_view(k_before[l], b), path, int(w.ctx_lens[b]))
+                assert int(dw.new_ctx[b]) == new_ctx
+                assert np.array_equal(w.seq_view(ka[l], b)[:new_ctx], ref[:new_ctx])
+        first = _step_outputs(dw)
+        # a second step on the same buffers (the counters are cleared per step): the same top-k
+        # and verdicts
+        prev = ptd.step_topk_policy(ptd.STEP_TOPK_CLUSTERED if kind == "clustered" else ptd.STEP_TOPK_STREAMED)
+        try:
+            assert dw.step() == launches
+            torch.cuda.synchronize()
+        finally:
+            ptd.step_topk_policy(prev)
+        second = _step_outputs(dw)
+        for key in ("idx", "val", "acc", "alen", "bonus", "status"):
+            assert (first[key] == second[key]) if isinstance(first[key], int) else torch.equal(first[key], second[key])
+        outs.append(second)
+    a = outs[0]
+    for b in outs[1:]:
+        for key in a:
+            if isinstance(a[key], int):
+                assert a[key] == b[key], key
+            else:
+                assert torch.equal(a[key], b[key]), key
