@@ -388,9 +388,9 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
 
 /* Which top-k the one-call step (and the steps built on it) uses when its workspace allows
  * both: AUTO streams the rows back to back when the clustered top-k (one cluster per row, at
- * most three CTAs per SM) would take more than two waves of the device's SMs, and clusters
- * otherwise (measured on GB300: 266 rows of 128256 logits stream faster, 128 rows of 152064
- * and 63 or fewer rows of 128256 run faster clustered); CLUSTERED and STREAMED force one where
+ * most three CTAs per SM) would take more than one wave of the device's SMs, and clusters
+ * otherwise (measured on GB300: 266 rows of 128256 logits and 128 rows of 152064 stream
+ * faster, 63 rows of 128256 and 31 of 32000 run faster clustered); CLUSTERED and STREAMED force one where
  * it applies (streaming needs vocab a multiple of 8 and 16-byte aligned rows; clustering needs
  * vocab <= 262143).  Process-wide; returns the previous policy, or -1 (nothing changed) for
  * an unknown value.  Results are identical either way. */

@@ -653,7 +653,7 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
   if (can_stream && can_cluster) {
     const int64_t cluster_ctas = (int64_t)tree->total_nodes * ptd::topk_cluster_size(a->vocab);
     streamed = policy == PTD_STEP_TOPK_STREAMED ||
-               (policy == PTD_STEP_TOPK_AUTO && cluster_ctas > 2 * 3 * (int64_t)sms);
+               (policy == PTD_STEP_TOPK_AUTO && cluster_ctas > 3 * (int64_t)sms);
   }
   const bool fused = streamed || can_cluster;
   unsigned int* tail_counters =

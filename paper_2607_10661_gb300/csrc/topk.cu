@@ -573,6 +573,27 @@ __device__ __forceinline__ uint32_t kth_largest_ord(uint32_t v, int k) {
   return 0u;
 }
 
+// The k-th largest of the 256 values v[0..7] of the warp's lanes (0 = none), or 0 when fewer
+// than k are nonzero: per distinct value one warp maximum and one warp sum of its copies.
+__device__ __forceinline__ uint32_t kth_largest_ord8(uint32_t (&v)[8], int k) {
+  int count = 0;
+  for (int s = 0; s < k; ++s) {
+    uint32_t lmax = 0u;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) lmax = v[i] > lmax ? v[i] : lmax;
+    const uint32_t m = __reduce_max_sync(0xffffffffu, lmax);
+    if (m == 0u) return 0u;
+    int c = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) c += v[i] == m ? 1 : 0;
+    count += (int)__reduce_add_sync(0xffffffffu, (unsigned)c);
+    if (count >= k) return m;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = v[i] == m ? 0u : v[i];
+  }
+  return 0u;
+}
+
 constexpr int kSelWarps = 8;
 constexpr int kSelThreads = kSelWarps * 32;
 constexpr int kProducerWarp = kSelWarps;
@@ -603,6 +624,7 @@ __global__ void __launch_bounds__(kStreamThreads, 2) topk_stream_kernel(const St
   extern __shared__ __align__(128) uint4 ring[];
   __shared__ __align__(8) uint64_t bars_s[2 * kStreamStages + 4];
   __shared__ uint64_t warp_keys[2][kSelWarps][KM];
+  __shared__ uint32_t lane_max_s[2][kSelThreads];   // a row part's first-chunk lane maxima
   __shared__ int offsets_s[kCachedOffsets];
   __shared__ int abort_s;
   __shared__ vt::VerifyScratch vsc;
@@ -772,8 +794,10 @@ __global__ void __launch_bounds__(kStreamThreads, 2) topk_stream_kernel(const St
   float thr = -INFINITY;
   int fresh = 0;   // lanes that pushed since T_w was last set (summed over chunks)
   int part = 0;
-  // After a failed wait (timeout, or another warp's) a warp stops reading; the others and the
-  // merge warp see the abort flag within their own bounded waits.
+  // After a failed wait (timeout, or another warp's) a warp keeps walking the schedule without
+  // data, so that every selection warp meets every part's barrier; the merge warp sees the
+  // abort flag within its own bounded waits.
+  bool ok = true;
   int j = 0;
   for (int64_t pos = vbeg; pos < vend; ++j) {
     int64_t row;
@@ -782,27 +806,35 @@ __global__ void __launch_bounds__(kStreamThreads, 2) topk_stream_kernel(const St
     const bool first = pos == vbeg || off == 0;
     const bool last = pos + n == vend || off + n == nvr;
     const int st = j % kStreamStages;
-    if (!mbar_wait_warp(full_bar(st), (uint32_t)((j / kStreamStages) & 1), &abort_s, a.dev_status)) break;
+    if (ok) ok = mbar_wait_warp(full_bar(st), (uint32_t)((j / kStreamStages) & 1), &abort_s, a.dev_status);
     const uint4* chunk = ring + (size_t)st * kStreamChunkVec;
     uint32_t hv[4];   // per vector: the packed maximum of its four pairs
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int vi = tid + u * kSelThreads;
-      const uint4 x = vi < n ? chunk[vi] : make_uint4(kBf16x2NegInf, kBf16x2NegInf, kBf16x2NegInf, kBf16x2NegInf);
+      const uint4 x =
+          ok && vi < n ? chunk[vi] : make_uint4(kBf16x2NegInf, kBf16x2NegInf, kBf16x2NegInf, kBf16x2NegInf);
       hv[u] = bf16x2_max(bf16x2_max(x.x, x.y), bf16x2_max(x.z, x.w));
     }
     if (first) {
-      // a new row part: T_w from this chunk (lanes without a vector here hold no element)
+      // a new row part: T from this chunk, the k-th largest of the CTA's 256 lane maxima
+      // (lanes without a vector here hold none): k elements of the part are >= T, so no
+      // element below T is among the CTA's top-k of the part (a warp's own T_w is never above)
       list.init();
       fresh = 0;
       const uint32_t h = bf16x2_max(bf16x2_max(hv[0], hv[1]), bf16x2_max(hv[2], hv[3]));
-      const uint32_t kth = kth_largest_ord(tid < n ? ordered_bits(fmaxf(bf16_lo(h), bf16_hi(h))) : 0u, k);
+      lane_max_s[part & 1][tid] = ok && tid < n ? ordered_bits(fmaxf(bf16_lo(h), bf16_hi(h))) : 0u;
+      asm volatile("bar.sync 1, %0;" ::"n"(kSelThreads) : "memory");   // the 8 selection warps only
+      uint32_t v[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[i] = lane_max_s[part & 1][lane * 8 + i];
+      const uint32_t kth = kth_largest_ord8(v, k);
       thr = kth != 0u ? from_ordered(kth) : -INFINITY;
     }
     uint32_t hits = 0u;
 #pragma unroll
     for (int u = 0; u < 4; ++u)
-      hits |= (tid + u * kSelThreads < n && fmaxf(bf16_lo(hv[u]), bf16_hi(hv[u])) >= thr ? 1u : 0u) << u;
+      hits |= (ok && tid + u * kSelThreads < n && fmaxf(bf16_lo(hv[u]), bf16_hi(hv[u])) >= thr ? 1u : 0u) << u;
     // the few vectors that reach the threshold: read again and pushed, in index order
     fresh += __popc(__ballot_sync(0xffffffffu, hits != 0u));
 #pragma unroll 1
@@ -819,7 +851,7 @@ __global__ void __launch_bounds__(kStreamThreads, 2) topk_stream_kernel(const St
       }
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(empty_bar(st));   // this warp is done with the stage
+    if (ok && lane == 0) mbar_arrive(empty_bar(st));   // this warp is done with the stage
     if (!last && fresh >= kRaiseAfter) {
       // raise T_w once enough new candidates came in: if k lanes hold candidates >= x, no
       // element below x is among the warp's top-k; x = the k-th largest of the lanes' largest
@@ -832,15 +864,17 @@ __global__ void __launch_bounds__(kStreamThreads, 2) topk_stream_kernel(const St
     // ---- the end of a row part: the warp's top-k into buffer part % 2 (free once the merge
     // warp has read the part two before this one)
     const int pb = part & 1;
-    if (!mbar_wait_warp(kempty_bar(pb), (uint32_t)(((part >> 1) & 1) ^ 1), &abort_s, a.dev_status)) break;
-    for (int s = 0; s < k; ++s) {
-      const uint64_t mine = list.head();
-      const uint64_t best = warp_max_u64(mine);
-      if (mine == best) list.pop();
-      if (lane == 0) warp_keys[pb][warp][s] = best;
+    if (ok) ok = mbar_wait_warp(kempty_bar(pb), (uint32_t)(((part >> 1) & 1) ^ 1), &abort_s, a.dev_status);
+    if (ok) {
+      for (int s = 0; s < k; ++s) {
+        const uint64_t mine = list.head();
+        const uint64_t best = warp_max_u64(mine);
+        if (mine == best) list.pop();
+        if (lane == 0) warp_keys[pb][warp][s] = best;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(kfull_bar(pb));
     }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(kfull_bar(pb));
     ++part;
   }
 }
