@@ -547,17 +547,20 @@ __global__ void __launch_bounds__(kThreads) topk_bf16_kernel(const __nv_bfloat16
 // the CTA's range through a ring of shared-memory chunks (bulk copies, one mbarrier pair per
 // stage); copy and selection overlap across row boundaries and the grid never waits between
 // waves.  The piece of a row that falls in one CTA's range (a row part) is selected by the 8
-// selection warps as in the clustered kernel: T_w is taken on the part's first chunk (every
-// lane's maximum over its vectors of that chunk; the k lanes holding the k largest maxima own
-// k elements >= T_w), each lane keeps its elements >= T_w of the whole part in an exact sorted
-// list, and at the part's end the warps' lists are merged into the part's top-k, which goes to
-// a global slot.  The part that completes its row (a per-row counter) merges the row's slots
+// selection warps much as in the clustered kernel: a threshold T is taken on the part's first
+// chunk (the k-th largest of the CTA's 256 lane maxima over that chunk: the lanes holding the
+// k largest own k elements >= T, so no element below T is among the CTA's top-k of the part),
+// each warp raises its own threshold as its lanes' candidates grow, each lane keeps its
+// elements at or above the threshold in an exact sorted list, and at the part's end the warps'
+// lists are merged into the part's top-k, which goes to a global slot.  The part that
+// completes its row (a per-row counter) merges the row's slots
 // and writes the row; the row that completes its tree (a per-tree counter) has the tree
 // verified on the same warp.  The part ends (the CTA merge, the global slot, the counters, a
 // row's merge and a tree's verification: a chain of L2 round trips) run on a merge warp of
 // their own, fed through a double buffer of the selection warps' keys, so that the stream
 // never waits for them.  Counters are cleared by the launch before this one (the step's
 // attention); slots are written before they are read within the launch.
+
 // The k-th largest of the warp's 32 order-preserving values (0 = a lane without one), or 0 when
 // fewer than k lanes hold one: one warp maximum and one ballot per distinct value, equal values
 // counted together.  Any x with k elements >= x bounds the warp's top-k from below.
@@ -604,7 +607,7 @@ constexpr int kStreamChunkVec = 1024;              // 16 KB of logits per chunk
 constexpr int kStreamMinVec = 2048;                // at least 32 KB per CTA
 constexpr int kPartSlot = 16;                      // keys per part slot (the largest k)
 constexpr int kCachedOffsets = 257;                // trees whose node offsets sit in shared memory
-constexpr int kRaiseAfter = 8;                     // new candidate lanes before T_w is raised
+constexpr int kRaiseAfter = 8;                     // new candidate lanes before a warp's threshold is raised
 
 struct StreamArgs {
   const __nv_bfloat16* logits;      // [rows][nvec_row * 8], back to back, 16-byte aligned
@@ -853,7 +856,7 @@ __global__ void __launch_bounds__(kStreamThreads, 2) topk_stream_kernel(const St
     __syncwarp();
     if (ok && lane == 0) mbar_arrive(empty_bar(st));   // this warp is done with the stage
     if (!last && fresh >= kRaiseAfter) {
-      // raise T_w once enough new candidates came in: if k lanes hold candidates >= x, no
+      // raise the threshold once enough new candidates came in: if k lanes hold candidates >= x, no
       // element below x is among the warp's top-k; x = the k-th largest of the lanes' largest
       fresh = 0;
       const uint32_t kth = kth_largest_ord(list.ord[0], k);
