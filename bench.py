@@ -55,6 +55,10 @@ METRIC = "tree-verify steps/sec (HBM GB/s and fraction of ~8 TB/s alongside)"
 PROFILED_ATTENTION_TRAFFIC = {(("llama3-8b-gqa", 32), "766310cc72ef5798"): 1112748032}
 PROFILED_LM_HEAD_TRAFFIC = {"c177b463ccbf468a": 1056910592}
 MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
+# the tail of the one-call step (ptd_step_tail)
+STEP_TAILS = {0: "top-k, then verification + compaction in one launch",
+              1: "clustered top-k (one cluster per row) verifying the trees, then a compaction kernel",
+              2: "streamed top-k (rows back to back, one share per CTA) verifying the trees, then a compaction kernel"}
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
 NOMINAL_HBM_GBS = 8000.0
@@ -584,6 +588,7 @@ def run_gpu(args, rank: int, world: int, dist):
         "verify": "sampling (Alg. 2, temperature 1)" if sampling else "greedy",
         "draft_update": "top-1 expansion, width 4, depth 6 (Alg. 1 step 3)" if args.draft_update else None,
         "top_k_source": ("LM head from hidden states (logits not written)" if args.lm_head else "resident logits"),
+        "step_tail": None if sampling else STEP_TAILS[ptd.step_tail(dw.tree, dw.cache, dw.bufs)],
         "ptd_step": ("tree positions + rotary encoding + K/V append, attention, top-k, verification + compaction, "
                      "draft update, pool merge, pool retrieval") if args.ptd_step else None,
         "parallelism": f"replicas x{world}" if world > 1 else "single GPU", "l2": l2_note}

@@ -397,6 +397,13 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
 typedef enum { PTD_STEP_TOPK_AUTO = 0, PTD_STEP_TOPK_CLUSTERED = 1, PTD_STEP_TOPK_STREAMED = 2 } ptd_step_topk;
 int32_t ptd_step_topk_policy(int32_t policy);
 
+/* The tail ptd_tree_verify_step would run for these arguments under the current policy (host
+ * only; reads the sizes, the pointers' presence and alignment, and the device's SM count;
+ * enqueues nothing): 2 = the streamed top-k verifies the trees, 1 = the clustered top-k does,
+ * 0 = the top-k is followed by ptd_verify_and_compact; -1 for a missing or invalid tree,
+ * cache or argument block. */
+int32_t ptd_step_tail(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* args);
+
 /* The same step fed from and drained to HOST memory (pinned for asynchronous copies):
  * copies the host inputs into the device buffers named by `tree`, `cache` and `args`,
  * runs ptd_tree_verify_step, and copies the small results back.  Contiguous caches only.

@@ -611,7 +611,45 @@ ptd_status ptd_lm_head_topk(const void* hidden, int32_t rows, int64_t hidden_str
 
 namespace {
 std::atomic<int> g_step_topk{PTD_STEP_TOPK_AUTO};
+
+constexpr int kTailSeparate = 0, kTailClustered = 1, kTailStreamed = 2;
+
+// The step's tail for checked arguments.  The streaming top-k needs rows back to back on
+// 16-byte vectors and the whole tail of ptd_step_workspace_size; the clustered one only the
+// per-tree counters; both need the tensor-core attention (which clears the counters) and bf16
+// logits.  With both possible the policy decides (auto: stream when the clustered grid, at
+// three CTAs per SM, would need more than one wave).
+int step_tail(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a, size_t* attn_ws_out,
+              int* sms_out) {
+  const size_t attn_ws = (ptd_attention_workspace_size(tree, cache, a->num_q_heads, cache->num_layers) + 255) /
+                         256 * 256;
+  const int sms = num_sms_of_current_device();
+  *attn_ws_out = attn_ws;
+  *sms_out = sms;
+  const bool tail_ok = use_tensor_cores(cache) && a->logits_dtype == PTD_BF16 && a->workspace &&
+                       aligned16(a->workspace);
+  const bool can_stream = tail_ok && ptd::topk_stream_ok(a->logits, a->vocab) &&
+                          a->workspace_bytes >= attn_ws + stream_tail_bytes(tree->batch, tree->total_nodes, sms);
+  const bool can_cluster = tail_ok && ptd::topk_can_verify(true, a->vocab) &&
+                           a->workspace_bytes >= attn_ws + tail_counters_bytes(tree->batch);
+  if (can_stream && can_cluster) {
+    const int policy = g_step_topk.load();
+    const int64_t cluster_ctas = (int64_t)tree->total_nodes * ptd::topk_cluster_size(a->vocab);
+    const bool stream = policy == PTD_STEP_TOPK_STREAMED ||
+                        (policy == PTD_STEP_TOPK_AUTO && cluster_ctas > 3 * (int64_t)sms);
+    return stream ? kTailStreamed : kTailClustered;
+  }
+  return can_stream ? kTailStreamed : (can_cluster ? kTailClustered : kTailSeparate);
+}
 }  // namespace
+
+int32_t ptd_step_tail(const ptd_tree* tree, const ptd_kv_cache* cache, const ptd_step_args* a) {
+  if (!a || !tree || !cache || check_tree(tree) != PTD_OK || check_cache(cache) != PTD_OK || a->num_q_heads < 1)
+    return -1;
+  size_t attn_ws = 0;
+  int sms = 0;
+  return step_tail(tree, cache, a, &attn_ws, &sms);
+}
 
 int32_t ptd_step_topk_policy(int32_t policy) {
   if (policy != PTD_STEP_TOPK_AUTO && policy != PTD_STEP_TOPK_CLUSTERED && policy != PTD_STEP_TOPK_STREAMED) return -1;
@@ -637,25 +675,11 @@ ptd_status ptd_tree_verify_step(const ptd_tree* tree, const ptd_kv_cache* cache,
   // verification + compaction in one launch.  Each launch may be placed while the previous one
   // drains; it reads its inputs only after that one has completed (the top-k's logits come from
   // the step's forward pass).
-  // The streaming top-k needs rows back to back on 16-byte vectors and the whole tail of
-  // ptd_step_workspace_size; the clustered one only the per-tree counters.
-  const size_t attn_ws = (ptd_attention_workspace_size(tree, cache, a->num_q_heads, cache->num_layers) + 255) /
-                         256 * 256;
-  const int sms = num_sms_of_current_device();
-  const bool tail_ok = use_tensor_cores(cache) && a->logits_dtype == PTD_BF16 && a->workspace &&
-                       aligned16(a->workspace);
-  const bool can_stream = tail_ok && ptd::topk_stream_ok(a->logits, a->vocab) &&
-                          a->workspace_bytes >= attn_ws + stream_tail_bytes(tree->batch, tree->total_nodes, sms);
-  const bool can_cluster = tail_ok && ptd::topk_can_verify(true, a->vocab) &&
-                           a->workspace_bytes >= attn_ws + tail_counters_bytes(tree->batch);
-  const int policy = g_step_topk.load();
-  bool streamed = can_stream;
-  if (can_stream && can_cluster) {
-    const int64_t cluster_ctas = (int64_t)tree->total_nodes * ptd::topk_cluster_size(a->vocab);
-    streamed = policy == PTD_STEP_TOPK_STREAMED ||
-               (policy == PTD_STEP_TOPK_AUTO && cluster_ctas > 3 * (int64_t)sms);
-  }
-  const bool fused = streamed || can_cluster;
+  size_t attn_ws = 0;
+  int sms = 0;
+  const int tail = step_tail(tree, cache, a, &attn_ws, &sms);
+  const bool streamed = tail == kTailStreamed;
+  const bool fused = tail != kTailSeparate;
   unsigned int* tail_counters =
       fused ? reinterpret_cast<unsigned int*>(static_cast<uint8_t*>(a->workspace) + attn_ws) : nullptr;
   const int zero_count = streamed ? tree->batch + tree->total_nodes : tree->batch;

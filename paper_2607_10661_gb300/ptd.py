@@ -31,7 +31,7 @@ EXPORTED = (
     "ptd_draft_tree_update", "ptd_pool_bytes", "ptd_pool_init", "ptd_pool_merge", "ptd_pool_retrieve",
     "ptd_tree_rope_append", "ptd_lm_head_topk_workspace_size", "ptd_lm_head_topk", "ptd_pipeline_create",
     "ptd_pipeline_submit", "ptd_pipeline_wait", "ptd_pipeline_destroy", "ptd_check_bounded_wait",
-    "ptd_step_workspace_size", "ptd_step_topk_policy",
+    "ptd_step_workspace_size", "ptd_step_topk_policy", "ptd_step_tail",
 )
 
 
@@ -88,6 +88,8 @@ def lib() -> ctypes.CDLL:
         L.ptd_last_launch_count.argtypes = []
         L.ptd_step_topk_policy.restype = i32
         L.ptd_step_topk_policy.argtypes = [i32]
+        L.ptd_step_tail.restype = i32
+        L.ptd_step_tail.argtypes = [P(_Tree), P(_Cache), P(_StepArgs)]
         L.ptd_attention_workspace_size.restype = sz
         L.ptd_attention_workspace_size.argtypes = [P(_Tree), P(_Cache), i32, i32]
         L.ptd_step_workspace_size.restype = sz
@@ -154,6 +156,18 @@ def step_topk_policy(policy: int) -> int:
     if prev < 0:
         raise ValueError(f"unknown step top-k policy {policy}")
     return prev
+
+
+STEP_TAIL_SEPARATE, STEP_TAIL_CLUSTERED, STEP_TAIL_STREAMED = 0, 1, 2
+
+
+def step_tail(tree: Tree, cache: KVCache, bufs: "StepBuffers") -> int:
+    """ptd_step_tail: which tail tree_verify_step would run (0 separate verify + compact,
+    1 clustered top-k verifying, 2 streamed top-k verifying)."""
+    t = int(lib().ptd_step_tail(ctypes.byref(tree.c), ctypes.byref(cache.c), ctypes.byref(bufs.c)))
+    if t < 0:
+        raise ValueError("ptd_step_tail: invalid tree, cache or step arguments")
+    return t
 
 
 def last_launch_count() -> int:

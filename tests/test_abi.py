@@ -269,3 +269,45 @@ def test_step_topk_policy_round_trip(lib):
         assert lib.ptd_step_topk_policy(0) == 1
     finally:
         lib.ptd_step_topk_policy(start)
+
+
+@host_only
+def test_step_tail_choice(lib):
+    """ptd_step_tail (host only) gives the tail ptd_tree_verify_step would run: the clustered
+    top-k for a one-wave step (63 rows of 128256), the streamed one for more than one wave
+    (266 rows), either when forced, the clustered one where streaming cannot apply (vocab not a
+    multiple of 8, logits off 16 bytes, a workspace holding only the per-tree counters), the
+    separate verification without a workspace or with fp32 logits, and -1 for a missing tree."""
+    from paper_2607_10661_gb300 import ptd
+
+    A = 1 << 20
+
+    def tail(tree=None, **kw):
+        t, c, a = _step_structs(ptd, **kw)
+        if tree is not None:
+            t = tree
+        return lib.ptd_step_tail(ctypes.byref(t), ctypes.byref(c), ctypes.byref(a)), t, c
+
+    _, t, c = tail()
+    full = lib.ptd_step_workspace_size(ctypes.byref(t), ctypes.byref(c), 32)
+    attn = lib.ptd_attention_workspace_size(ctypes.byref(t), ctypes.byref(c), 32, 32)
+    ws = dict(workspace=A * 64, workspace_bytes=full)
+    assert tail()[0] == ptd.STEP_TAIL_SEPARATE
+    assert tail(**ws)[0] == ptd.STEP_TAIL_CLUSTERED
+    many = ptd._Tree(8, 266, 64, 4096, A, A + 1024, A + 2048)
+    full_many = lib.ptd_step_workspace_size(ctypes.byref(many), ctypes.byref(c), 32)
+    assert tail(many, workspace=A * 64, workspace_bytes=full_many)[0] == ptd.STEP_TAIL_STREAMED
+    prev = ptd.step_topk_policy(ptd.STEP_TOPK_STREAMED)
+    try:
+        assert tail(**ws)[0] == ptd.STEP_TAIL_STREAMED
+        assert tail(vocab=128250, **ws)[0] == ptd.STEP_TAIL_CLUSTERED
+        assert tail(logits=A * 32 + 8, **ws)[0] == ptd.STEP_TAIL_CLUSTERED
+        counters_only = (attn + 255) // 256 * 256 + 256
+        assert tail(workspace=A * 64, workspace_bytes=counters_only)[0] == ptd.STEP_TAIL_CLUSTERED
+        ptd.step_topk_policy(ptd.STEP_TOPK_CLUSTERED)
+        assert tail(many, workspace=A * 64, workspace_bytes=full_many)[0] == ptd.STEP_TAIL_CLUSTERED
+    finally:
+        ptd.step_topk_policy(prev)
+    assert tail(logits_dtype=ptd.F32, **ws)[0] == ptd.STEP_TAIL_SEPARATE
+    t, c, a = _step_structs(ptd)
+    assert lib.ptd_step_tail(None, ctypes.byref(c), ctypes.byref(a)) == -1
